@@ -1,0 +1,423 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+None of these tests compares the oracle with itself: each checks a closed
+form, an invariant, a special case that reduces to a textbook routine (SVD,
+symmetric eigendecomposition), a published known-answer value, or brute force
+on tiny inputs.  CPU only.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle as O
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+# Muon's published quintic, typed here independently of the oracle's constant.
+A_COEF, B_COEF, C_COEF = 3.4445, -4.7750, 2.0315
+
+
+def _rng(s):
+    return np.random.default_rng(s)
+
+
+# ---------------------------------------------------------------------------
+# Philox4x32-10 and the Gaussian sketch matrix (Algorithm 2, Omega sample)
+# ---------------------------------------------------------------------------
+def test_philox_known_answers():
+    kat = json.load(open(os.path.join(GOLD, "philox4x32_10_kat.json")))
+    for v in kat["vectors"]:
+        ctr = tuple(np.array([int(x, 16)], dtype=np.uint64) for x in v["ctr"])
+        key = tuple(int(x, 16) for x in v["key"])
+        out = O.philox4x32_10(ctr, key)
+        assert ["%08x" % int(w[0]) for w in out] == v["out"]
+
+
+def test_philox_uniform_is_open_interval_and_exact():
+    x = np.array([0, 511, 512, 0xFFFFFFFF], dtype=np.uint32)
+    u = O.philox_uniform(x)
+    assert u[0] == 2.0 ** -24 and u[1] == u[0]
+    assert u[2] == 3.0 * 2.0 ** -24
+    assert u[3] == 1.0 - 2.0 ** -24
+    assert np.all((u > 0) & (u < 1))
+    # odd multiples of 2^-24 below 1 have <= 24 significant bits: exact in fp32
+    xs = np.random.default_rng(0).integers(0, 2 ** 32, 100000, dtype=np.uint64).astype(np.uint32)
+    us = O.philox_uniform(xs)
+    assert np.all(us.astype(np.float32).astype(np.float64) == us)
+
+
+def test_omega_counter_layout():
+    """Element e of Omega uses block e // 4 with counter (block, id, t_lo, t_hi)."""
+    seed, mid, t = 0x1234_5678_9ABC_DEF0, 5, (3 << 32) + 7
+    om = O.sketch_omega(seed, mid, t, 6, 10)          # 60 elements, 15 blocks
+    blk = 9
+    ctr = tuple(np.array([c], dtype=np.uint64) for c in (blk, mid, 7, 3))
+    words = O.philox4x32_10(ctr, (0x9ABCDEF0, 0x12345678))
+    u = [O.philox_uniform(w)[0] for w in words]
+    z = [math.sqrt(-2 * math.log(u[0])) * math.cos(2 * math.pi * u[1]),
+         math.sqrt(-2 * math.log(u[0])) * math.sin(2 * math.pi * u[1]),
+         math.sqrt(-2 * math.log(u[2])) * math.cos(2 * math.pi * u[3]),
+         math.sqrt(-2 * math.log(u[2])) * math.sin(2 * math.pi * u[3])]
+    flat = om.reshape(-1)
+    np.testing.assert_allclose(flat[36:40], z, rtol=0, atol=1e-15)
+    # a different step or matrix gives an independent stream
+    assert not np.allclose(om, O.sketch_omega(seed, mid, t + 1, 6, 10))
+    assert not np.allclose(om, O.sketch_omega(seed, mid + 1, t, 6, 10))
+
+
+def test_omega_is_standard_normal():
+    from scipy import stats
+    z = O.sketch_omega(42, 0, 0, 20000, 10).reshape(-1)
+    assert abs(z.mean()) < 0.01
+    assert abs(z.var() - 1) < 0.01
+    assert abs(stats.skew(z)) < 0.03
+    assert abs(stats.kurtosis(z)) < 0.06
+    assert stats.kstest(z, "norm").pvalue > 1e-3
+
+
+# ---------------------------------------------------------------------------
+# Momentum, relaxed tangent momentum, diagonal-Gram normalization (Alg. 1, Eq. 3)
+# ---------------------------------------------------------------------------
+def test_hand_worked_2x3_both_orientations():
+    """A 2x3 example worked by hand from Algorithm 1 with mu = 1/2."""
+    W = np.array([[1.0, 0, 0], [0, 2.0, 0]])
+    Mp = np.array([[2.0, 0, 0], [0, 0, 2.0]])
+    G = np.array([[0, 3.0, 0], [1.0, 0, 0]])
+    M = O.momentum_update(Mp, G, 0.5)
+    np.testing.assert_array_equal(M, [[1, 3, 0], [1, 0, 1]])
+    # row-active: row0 m=(1,3,0), w=(1,0,0): <m,w>=1, x=(0,3,0);
+    #             row1 m=(1,0,1), w=(0,2,0): <m,w>=0, x=(1,0,1)
+    X = O.relaxed_tangent(O.orient(M, 0), O.orient(W, 0))
+    np.testing.assert_array_equal(X, [[0, 3, 0], [1, 0, 1]])
+    Psi, d = O.diag_gram_normalize(X)
+    np.testing.assert_allclose(d, [3, math.sqrt(2)], rtol=1e-15)
+    r = 1 / math.sqrt(2)
+    np.testing.assert_allclose(Psi, [[0, 1, 0], [r, 0, r]], rtol=0, atol=1e-16)
+    # column-active: columns of M (1,1),(3,0),(0,1); of W (1,0),(0,2),(0,0)
+    #   c0: a=1 -> x=(0,1); c1: a=0 -> x=(3,0); c2: w=0 -> x=(0,1)
+    X1 = O.relaxed_tangent(O.orient(M, 1), O.orient(W, 1))
+    np.testing.assert_array_equal(X1, [[0, 1], [3, 0], [0, 1]])
+    Psi1, _ = O.diag_gram_normalize(X1)
+    np.testing.assert_array_equal(Psi1, [[0, 1], [1, 0], [0, 1]])
+
+
+def test_orientation_parity():
+    assert [O.orientation_of(t) for t in range(5)] == [0, 1, 0, 1, 0]
+    assert O.orientation_of(3, mode=1) == 0 and O.orientation_of(2, mode=2) == 1
+
+
+def test_tangent_decomposition_identity():
+    """x = g_tan + (1 - ||w||^2) g_rad and ||x||^2 = ||g||^2 [sin^2 + (1-||w||^2)^2 cos^2]
+    (App. D.2, relaxed tangent gradient and Lemma 1)."""
+    rng = _rng(1)
+    g = rng.standard_normal((7, 40))
+    w = rng.standard_normal((7, 40)) * rng.uniform(0.1, 2.0, (7, 1)) / math.sqrt(40)
+    x = O.relaxed_tangent(g, w)
+    wn2 = (w * w).sum(1, keepdims=True)
+    g_rad = (g * w).sum(1, keepdims=True) / wn2 * w
+    g_tan = g - g_rad
+    np.testing.assert_allclose(x, g_tan + (1 - wn2) * g_rad, rtol=1e-12, atol=1e-12)
+    cos2 = (g * w).sum(1) ** 2 / ((g * g).sum(1) * wn2[:, 0])
+    lhs = (x * x).sum(1)
+    rhs = (g * g).sum(1) * ((1 - cos2) + (1 - wn2[:, 0]) ** 2 * cos2)
+    np.testing.assert_allclose(lhs, rhs, rtol=1e-11)
+
+
+def test_tangent_special_cases():
+    rng = _rng(2)
+    g = rng.standard_normal((5, 30))
+    # W = 0: x = m
+    np.testing.assert_array_equal(O.relaxed_tangent(g, np.zeros_like(g)), g)
+    # unit-norm rows: strict tangent projection, x orthogonal to w
+    w = rng.standard_normal((5, 30))
+    w /= np.linalg.norm(w, axis=1, keepdims=True)
+    x = O.relaxed_tangent(g, w)
+    np.testing.assert_allclose((x * w).sum(1), 0, atol=1e-13)
+
+
+def test_normalize_unit_rows_and_inner_product():
+    """Gamma_ii = 1 (Sec. 2.2) and <X, Psi>_F = sum_i ||x_i|| (Lemma 1)."""
+    X = _rng(3).standard_normal((9, 33)) * np.exp(_rng(4).standard_normal((9, 1)))
+    Psi, d = O.diag_gram_normalize(X)
+    np.testing.assert_allclose(np.diag(Psi @ Psi.T), 1, rtol=1e-14)
+    np.testing.assert_allclose((X * Psi).sum(), np.linalg.norm(X, axis=1).sum(), rtol=1e-13)
+    # D(X) is the square root of the Gram diagonal
+    np.testing.assert_allclose(d ** 2, np.diag(X @ X.T), rtol=1e-13)
+
+
+def test_normalize_zero_row_reading():
+    X = _rng(5).standard_normal((4, 8))
+    X[2] = 0
+    Psi, d = O.diag_gram_normalize(X)
+    assert d[2] == 0 and np.all(Psi[2] == 0)
+    np.testing.assert_allclose(np.linalg.norm(Psi, axis=1)[[0, 1, 3]], 1, rtol=1e-14)
+
+
+def test_extreme_scale_example():
+    """Sec. 1: one row norm 1e4, the rest 1e-3, fixed directions.  The raw Gram's
+    leading eigenvector is the big row's axis; Psi is scale-free."""
+    g = json.load(open(os.path.join(GOLD, "extreme_scale.json")))
+    rng = _rng(g["direction_seed"])
+    base = rng.standard_normal(g["cols"])
+    dirs = g["correlation"] * base + (1 - g["correlation"]) * rng.standard_normal((g["rows"], g["cols"]))
+    dirs /= np.linalg.norm(dirs, axis=1, keepdims=True)
+    norms = np.full(g["rows"], g["small_norm"])
+    norms[g["big_row"]] = g["big_norm"]
+    X = dirs * norms[:, None]
+    lam, U = np.linalg.eigh(X @ X.T)
+    lead = U[:, -1]
+    assert abs(lead[g["big_row"]]) > 1 - 1e-9
+    Psi, _ = O.diag_gram_normalize(X)
+    Psi_eq, _ = O.diag_gram_normalize(dirs)
+    np.testing.assert_allclose(Psi, Psi_eq, rtol=0, atol=1e-14)
+    # after normalization the correlated rows dominate the leading mode
+    lamG, UG = np.linalg.eigh(Psi @ Psi.T)
+    assert abs(UG[g["big_row"], -1]) < 0.6
+
+
+def test_step_invariant_to_row_rescaling():
+    """With M_{t-1} = 0 and a row-active step, positive per-row rescaling of G
+    leaves Psi, T and the weight update unchanged (A3 is linear per row, Eq. 3
+    divides the scale out).  Column rescaling plays the same role for k = 1."""
+    rng = _rng(6)
+    m, n = 12, 40
+    W = rng.standard_normal((m, n)) * 0.05
+    G = rng.standard_normal((m, n))
+    Z = np.zeros((m, n))
+    s_row = np.exp(2 * rng.standard_normal((m, 1)))
+    s_col = np.exp(2 * rng.standard_normal((1, n)))
+    for variant in ("G", "L"):
+        cfg = O.OracleConfig(variant=variant, rank=4, oversample=3)
+        a = O.normpre_step(W, G, Z, 0, 1e-2, cfg)
+        b = O.normpre_step(W, G * s_row, Z, 0, 1e-2, cfg)
+        np.testing.assert_allclose(b["Psi"], a["Psi"], atol=1e-13)
+        np.testing.assert_allclose(b["W"], a["W"], atol=1e-12)
+        a1 = O.normpre_step(W, G, Z, 1, 1e-2, cfg)
+        b1 = O.normpre_step(W, G * s_col, Z, 1, 1e-2, cfg)
+        np.testing.assert_allclose(b1["W"], a1["W"], atol=1e-12)
+    # and the overall momentum scale has no effect
+    cfgG = O.OracleConfig(variant="G")
+    Mp = rng.standard_normal((m, n))
+    a = O.normpre_step(W, G, Mp, 0, 1e-2, cfgG)
+    b = O.normpre_step(W, 3.0 * G, 3.0 * Mp, 0, 1e-2, cfgG)
+    np.testing.assert_allclose(b["W"], a["W"], atol=1e-12)
+
+
+def test_orientation_is_transpose_symmetric():
+    """A column-active step on W is the row-active step on W^T, transposed."""
+    rng = _rng(7)
+    W = rng.standard_normal((10, 24)) * 0.05
+    G = rng.standard_normal((10, 24))
+    Mp = rng.standard_normal((10, 24))
+    for variant in ("G", "L_exact"):
+        cfg = O.OracleConfig(variant=variant, rank=5)
+        col = O.normpre_step(W, G, Mp, 1, 1e-2, cfg)
+        row_t = O.normpre_step(W.T, G.T, Mp.T, 0, 1e-2, cfg)
+        np.testing.assert_allclose(col["W"], row_t["W"].T, atol=1e-13)
+        np.testing.assert_allclose(col["Psi"], row_t["Psi"], atol=1e-14)
+
+
+# ---------------------------------------------------------------------------
+# NormPre-G: Newton-Schulz (Sec. 3.2, App. B/C)
+# ---------------------------------------------------------------------------
+def _scalar_quintic(x, steps):
+    for _ in range(steps):
+        x = A_COEF * x + B_COEF * x ** 3 + C_COEF * x ** 5
+    return x
+
+
+@pytest.mark.parametrize("shape", [(16, 48), (48, 16), (20, 20), (1, 9)])
+def test_ns_singular_value_map(shape):
+    """NS acts on each singular value alone: svd(NS_q(Psi)) = p^q(sigma/||Psi||_F)
+    with the singular vectors of Psi (checked with an independent SVD)."""
+    rng = _rng(8)
+    X = rng.standard_normal(shape) * np.exp(rng.standard_normal((shape[0], 1)))
+    Psi, _ = O.diag_gram_normalize(X)
+    T = O.newton_schulz(Psi, 5, eps=0.0)
+    U, s, Vt = np.linalg.svd(Psi, full_matrices=False)
+    expect = U @ np.diag(_scalar_quintic(s / np.linalg.norm(Psi), 5)) @ Vt
+    np.testing.assert_allclose(T, expect, atol=1e-12)
+
+
+def test_ns_band_of_the_polynomial():
+    """After 5 quintic steps every singular value from [sigma_min/||Psi||, 1] lands in
+    the band the scalar map implies (Muon's quintic oscillates around ~0.7-1.2)."""
+    rng = _rng(9)
+    Psi, _ = O.diag_gram_normalize(rng.standard_normal((64, 256)))
+    s_in = np.linalg.svd(Psi, compute_uv=False) / np.linalg.norm(Psi)
+    grid = np.linspace(s_in.min(), 1.0, 20001)
+    band = _scalar_quintic(grid, 5)
+    s_out = np.linalg.svd(O.newton_schulz(Psi, 5, eps=0.0), compute_uv=False)
+    assert s_out.min() >= band.min() - 1e-9 and s_out.max() <= band.max() + 1e-9
+    assert 0.6 < s_out.min() and s_out.max() < 1.25
+
+
+def test_cubic_ns_converges_to_polar_factor():
+    """With the classical cubic (1.5, -0.5, 0) iterated to convergence, NS gives
+    msign(Psi) = U V^T (Sec. 2.1), which has ||T||_F^2 = min(m, n)."""
+    rng = _rng(10)
+    Psi, _ = O.diag_gram_normalize(rng.standard_normal((12, 30)))
+    T = O.newton_schulz(Psi, 80, coef=(1.5, -0.5, 0.0), eps=0.0)
+    U, s, Vt = np.linalg.svd(Psi, full_matrices=False)
+    np.testing.assert_allclose(T, U @ Vt, atol=1e-10)
+    assert abs((T * T).sum() - 12) < 1e-9
+
+
+def test_ns_transpose_rule():
+    rng = _rng(11)
+    Psi = rng.standard_normal((40, 12))
+    np.testing.assert_allclose(O.newton_schulz(Psi), O.newton_schulz(Psi.T).T, atol=1e-13)
+
+
+def test_orthogonal_rows_are_fixed_points():
+    """App. A.3: orthogonal rows normalize to Gamma = I; msign(Psi) = Psi and the
+    localized preconditioner selects nothing (T = Psi)."""
+    g = json.load(open(os.path.join(GOLD, "orthogonal_rows.json")))
+    Qm, _ = np.linalg.qr(_rng(12).standard_normal((g["cols"], g["rows"])))
+    X = Qm.T * np.array(g["row_norms"])[:, None]
+    Psi, _ = O.diag_gram_normalize(X)
+    np.testing.assert_allclose(Psi @ Psi.T, np.eye(g["rows"]), atol=1e-14)
+    ex = O.exact_interaction_eigs(Psi, r=32)
+    # every eigenvalue is one (up to rounding, which may put some a few ulps above
+    # the strict lam > 1 cut; such a mode is scaled by lam^{-1/2} - 1 ~ 1e-16)
+    np.testing.assert_allclose(ex["lam"], 1.0, atol=1e-14)
+    np.testing.assert_allclose(O.localized_apply(Psi, ex["U_C"], ex["lam_C"]), Psi, atol=1e-14)
+    T = O.newton_schulz(Psi, 80, coef=(1.5, -0.5, 0.0), eps=0.0)
+    np.testing.assert_allclose(T, Psi, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# NormPre-L: Props. 1-2, Algorithm 2 (App. B, App. D.1)
+# ---------------------------------------------------------------------------
+def _psi(m, n, seed, corr=0.0):
+    rng = _rng(seed)
+    X = rng.standard_normal((m, n)) + corr * rng.standard_normal((1, n))
+    X *= np.exp(rng.standard_normal((m, 1)))
+    return O.diag_gram_normalize(X)[0]
+
+
+def test_prop1_clipped_singular_values():
+    """r >= |A|: sigma_i(T) = min(sigma_i(Psi), 1) with Psi's singular vectors (Prop. 1)."""
+    Psi = _psi(10, 30, 13, corr=0.6)
+    ex = O.exact_interaction_eigs(Psi, r=10)
+    T = O.localized_apply(Psi, ex["U_C"], ex["lam_C"])
+    U, s, Vt = np.linalg.svd(Psi, full_matrices=False)
+    np.testing.assert_allclose(T, U @ np.diag(np.minimum(s, 1.0)) @ Vt, atol=1e-12)
+    # and T_+ is the projection of Psi onto the unit spectral ball: nearest
+    # feasible point beats random feasible perturbations
+    base = np.linalg.norm(T - Psi)
+    rng = _rng(14)
+    for _ in range(20):
+        D = rng.standard_normal(T.shape) * 1e-3
+        Tp = T + D
+        Tp /= max(1.0, np.linalg.norm(Tp, 2))
+        assert np.linalg.norm(Tp - Psi) >= base - 1e-12
+
+
+def test_prop2_rank_budget_and_trace_identity():
+    """r < |A|: singular values are 1 on the r largest active modes and unchanged
+    elsewhere (Prop. 2); ||T||_F^2 = m - sum_C (lam_i - 1) and eig(P) in (0, 1]
+    (Lemma 2)."""
+    Psi = _psi(30, 40, 15, corr=0.0)
+    U, s, Vt = np.linalg.svd(Psi, full_matrices=False)
+    n_act = int((s ** 2 > 1).sum())
+    assert n_act >= 3
+    r = n_act - 1
+    ex = O.exact_interaction_eigs(Psi, r=r)
+    assert ex["n_active"] == r
+    T = O.localized_apply(Psi, ex["U_C"], ex["lam_C"])
+    s_exp = s.copy()
+    s_exp[:r] = 1.0
+    np.testing.assert_allclose(T, U @ np.diag(s_exp) @ Vt, atol=1e-12)
+    m = Psi.shape[0]
+    assert abs((T * T).sum() - (m - (ex["lam_C"] - 1).sum())) < 1e-11
+    P = np.eye(m) + ex["U_C"] @ np.diag(ex["lam_C"] ** -0.5 - 1) @ ex["U_C"].T
+    ev = np.linalg.eigvalsh(P)
+    assert ev.min() > 0 and ev.max() <= 1 + 1e-12
+
+
+def test_sketch_full_width_equals_exact():
+    """l = m: the sketch spans the whole row space, Rayleigh-Ritz is exact."""
+    Psi = _psi(10, 50, 16, corr=0.7)
+    om = O.sketch_omega(3, 0, 0, 50, 10)
+    sk = O.interaction_sketch(Psi, r=6, o=8, p=1, Omega=om)
+    assert sk["ell"] == 10
+    ex = O.exact_interaction_eigs(Psi, r=6)
+    assert sk["n_active"] == ex["n_active"]
+    np.testing.assert_allclose(sk["lam_C"], ex["lam_C"], rtol=1e-12)
+    P1 = sk["U_C"] @ sk["U_C"].T
+    P2 = ex["U_C"] @ ex["U_C"].T
+    np.testing.assert_allclose(P1, P2, atol=1e-10)
+
+
+def test_sketch_recovers_exact_low_rank():
+    """Rank-rho Psi with rho <= l: the Gaussian sketch captures range(Psi) and the
+    Ritz pairs are the exact eigenpairs (Halko et al. 2011)."""
+    rng = _rng(17)
+    m, n, rho = 60, 200, 5
+    X = rng.standard_normal((m, rho)) @ rng.standard_normal((rho, n))
+    Psi, _ = O.diag_gram_normalize(X)
+    sk = O.interaction_sketch(Psi, r=8, o=4, p=1, Omega=O.sketch_omega(1, 0, 0, n, 12))
+    lam = np.linalg.eigvalsh(Psi @ Psi.T)[::-1]
+    np.testing.assert_allclose(sk["ritz"][:rho], lam[:rho], rtol=1e-10)
+    ex = O.exact_interaction_eigs(Psi, r=8)
+    assert sk["n_active"] == ex["n_active"]
+    np.testing.assert_allclose(sk["U_C"] @ sk["U_C"].T, ex["U_C"] @ ex["U_C"].T, atol=1e-9)
+
+
+def test_sketch_ritz_values_interlace():
+    """Rayleigh-Ritz values satisfy lam_hat_i <= lam_i (Cauchy interlacing), so the
+    sketch never selects more modes than the exact preconditioner."""
+    Psi = _psi(64, 128, 18, corr=0.5)
+    lam = np.linalg.eigvalsh(Psi @ Psi.T)[::-1]
+    for seed in range(4):
+        sk = O.interaction_sketch(Psi, r=8, o=4, p=1, Omega=O.sketch_omega(seed, 0, 0, 128, 12))
+        assert np.all(sk["ritz"] <= lam[:12] + 1e-12)
+        assert sk["n_active"] <= O.exact_interaction_eigs(Psi, 8)["n_active"]
+
+
+def test_sketch_basis_orthonormal_and_selection_order():
+    Psi = _psi(40, 90, 19, corr=0.8)
+    sk = O.interaction_sketch(Psi, r=5, o=6, p=1, Omega=O.sketch_omega(9, 2, 4, 90, 11))
+    np.testing.assert_allclose(sk["Q"].T @ sk["Q"], np.eye(11), atol=1e-13)
+    lam = sk["ritz"]
+    assert np.all(np.diff(lam) <= 0)
+    # top-r then lam > 1 equals active-then-top-r (App. B)
+    active_then_top = lam[lam > 1][:5]
+    np.testing.assert_array_equal(sk["lam_C"], active_then_top)
+
+
+# ---------------------------------------------------------------------------
+# Consistent update RMS and the weight update (Sec. 3.1, Algorithm 1)
+# ---------------------------------------------------------------------------
+def test_rms_matching_and_weight_update():
+    rng = _rng(20)
+    T = rng.standard_normal((8, 20))
+    for k in (0, 1):
+        Ta = T if k == 0 else T.T
+        R = O.rms_matched(Ta, k, 0.2)
+        assert R.shape == (8, 20)
+        assert abs(np.sqrt((R * R).mean()) - 0.2) < 1e-15
+        np.testing.assert_allclose(R / np.linalg.norm(R), T / np.linalg.norm(T), atol=1e-15)
+    W = rng.standard_normal((8, 20))
+    R = O.rms_matched(T, 0, 0.2)
+    np.testing.assert_array_equal(O.weight_update(W, R, 0.0, 0.1), W)
+    np.testing.assert_allclose(O.weight_update(W, R, 0.5, 0.1), W - 0.5 * R - 0.05 * W, rtol=1e-13, atol=1e-15)
+    # zero update reading: only weight decay acts
+    Z = O.rms_matched(np.zeros((8, 20)), 0, 0.2)
+    assert np.all(Z == 0)
+
+
+def test_full_step_shapes_and_rms():
+    rng = _rng(21)
+    for variant in ("G", "L", "L_exact"):
+        cfg = O.OracleConfig(variant=variant, rank=4, oversample=4)
+        for t in (0, 1):
+            W = rng.standard_normal((16, 28)) * 0.02
+            out = O.normpre_step(W, rng.standard_normal((16, 28)), np.zeros((16, 28)), t, 0.1, cfg)
+            dW = (W - out["W"]) / 0.1 - 0.1 * W
+            assert dW.shape == W.shape
+            assert abs(np.sqrt((dW * dW).mean()) - 0.2) < 1e-12
