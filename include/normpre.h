@@ -1,0 +1,232 @@
+/*
+ * normpre.h — C ABI of the GB300 (sm_103a) NormPre optimizer-step library.
+ *
+ * The library computes the per-matrix update step of NormPre
+ * ("Normalize-Then-Precondition", Algorithm 1 of the paper) for a list of 2-D
+ * weight matrices on one GPU:
+ *
+ *   M_t   = mu M_{t-1} + G_t                                  (Sec. 3.1)
+ *   k_t   = t mod 2, Wbar = O_k(W), Mbar = O_k(M)             (Sec. 3.1)
+ *   x_i   = mbar_i - <mbar_i, wbar_i> wbar_i                  (relaxed tangent momentum, Sec. 3.1)
+ *   Psi   = D(X)^{-1} X                                       (Eq. 3, Sec. 2.2)
+ *   T     = msign(Psi) by Newton-Schulz        (NormPre-G, Sec. 3.2, App. B)
+ *         | (I + U_C (Lam_C^{-1/2} - I) U_C^T) Psi
+ *           with (U_C, Lam_C) from the randomized interaction sketch
+ *                                              (NormPre-L, Sec. 2.3, Alg. 2)
+ *   W    <- W - eta (0.2 O_k^{-1}(T) / RMS(T) + lambda_wd W)  (Sec. 3.1)
+ *
+ * Conventions shared by every call:
+ *   - Matrices are dense, row-major, contiguous, `rows x cols` as stored.
+ *   - Device pointers are CUDA device addresses on the current device and must
+ *     be 16-byte aligned.  Host pointers are ordinary host addresses.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Calls enqueue work on it and return without synchronizing unless the
+ *     description says otherwise.
+ *   - Every int-returning call returns a normpre_status.  A text message for
+ *     the last failure of a handle is available from normpre_last_error();
+ *     failures of calls without a handle are reported by
+ *     normpre_last_error(NULL) (thread-local).
+ *   - Argument, shape, dtype and alignment errors are found on the host before
+ *     any work is enqueued.  Conditions found on the device (non-finite
+ *     momentum, numerical breakdown, a bounded wait that gave up) set a flag in
+ *     device memory; it is reported by normpre_sync_status().  No kernel traps.
+ */
+#ifndef NORMPRE_H
+#define NORMPRE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct normpre_handle normpre_handle;
+
+/* Variant of the spectral preconditioner (Algorithm 1). */
+enum normpre_variant {
+  NORMPRE_G = 0,   /* global: T = msign(Psi) by Newton-Schulz (Sec. 3.2) */
+  NORMPRE_L = 1    /* localized: randomized interaction sketch (Alg. 2) */
+};
+
+/* Storage dtypes of caller tensors. */
+enum normpre_dtype {
+  NORMPRE_F32 = 0,
+  NORMPRE_BF16 = 1
+};
+
+/* Status codes. */
+enum normpre_status {
+  NORMPRE_OK = 0,
+  NORMPRE_ERR_ARG = 1,        /* null pointer, bad count or bad hyperparameter */
+  NORMPRE_ERR_SHAPE = 2,      /* a dimension <= 0 or beyond the supported range */
+  NORMPRE_ERR_DTYPE = 3,      /* dtype not supported for that tensor */
+  NORMPRE_ERR_ALIGN = 4,      /* a device pointer is not 16-byte aligned */
+  NORMPRE_ERR_CUDA = 5,       /* a CUDA runtime call failed (message has the CUDA error) */
+  NORMPRE_ERR_NONFINITE = 6,  /* NaN or Inf met in the momentum or weights (device flag) */
+  NORMPRE_ERR_NUMERIC = 7,    /* CholeskyQR breakdown or Jacobi sweep cap reached (device flag) */
+  NORMPRE_ERR_TIMEOUT = 8     /* a bounded device-side wait gave up (device flag) */
+};
+
+/* Which precision the spectral stage computes in. */
+enum normpre_precision {
+  NORMPRE_PREC_BF16 = 0,   /* NormPre-G: Psi and the Newton-Schulz operands in bf16 with fp32
+                              accumulation on the tensor cores; normalization in fp32 */
+  NORMPRE_PREC_F32 = 1     /* everything in fp32 (parity mode) */
+};
+
+/* Hyperparameters (defaults: Table 4 / App. A of the paper). */
+typedef struct normpre_config {
+  int variant;            /* normpre_variant */
+  float momentum;         /* mu = 0.95 */
+  float weight_decay;     /* lambda_wd = 0.1 (multiplied by the learning rate) */
+  float target_rms;       /* 0.2 (consistent update RMS, Sec. 3.1) */
+  int ns_steps;           /* q = 5 Newton-Schulz iterations */
+  float ns_coef[3];       /* (a, b, c) of X <- aX + b(XX^T)X + c(XX^T)^2 X; default Muon's
+                             quintic (3.4445, -4.7750, 2.0315) */
+  float ns_eps;           /* 1e-7: X is divided by ||X||_F + eps before the iteration */
+  int rank;               /* r = 32 (interaction rank budget) */
+  int oversample;         /* o = 8 */
+  int power_iters;        /* p = 1 */
+  uint64_t seed;          /* Philox4x32-10 key of the sketch matrix Omega */
+  int precision;          /* normpre_precision */
+  int orientation;        /* 0: alternate rows/columns with t (paper); 1: rows only; 2: columns only */
+} normpre_config;
+
+/* Fills `cfg` with the paper's defaults (NormPre-G, bf16 Newton-Schulz). */
+void normpre_default_config(normpre_config* cfg);
+
+/*
+ * Creates a handle for a fixed list of matrices.
+ *   cfg       hyperparameters (copied).
+ *   n_mats    number of matrices (>= 1).
+ *   rows/cols host arrays[n_mats] of stored shapes (each >= 1, <= 65536).
+ *   w_dtype   host array[n_mats] of normpre_dtype for W (F32 or BF16).
+ *   g_dtype   host array[n_mats] of normpre_dtype for G (F32 or BF16).
+ *             M is always F32.
+ *   out       receives the handle.
+ * The handle owns all device workspaces (allocated here with cudaMalloc on the
+ * current device) and precomputed launch plans; matrices of equal shape and
+ * dtypes are grouped so that one launch serves a whole group.
+ * Errors: ARG (null / bad count / bad hyperparameter), SHAPE, DTYPE, CUDA.
+ */
+int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, const int64_t* cols,
+                 const int* w_dtype, const int* g_dtype, normpre_handle** out);
+
+/*
+ * One optimizer step (Algorithm 1) for every matrix of the handle.
+ *   t        number of steps completed before this one (0 for the first);
+ *            selects the orientation k_t = t mod 2 and the sketch stream.
+ *   lr       eta_t.
+ *   W, G, M  host arrays[n_mats] of DEVICE pointers: W (w_dtype, updated in
+ *            place), G (g_dtype, read only), M (fp32 momentum M_{t-1} on
+ *            entry, M_t on return).
+ *   stream   cudaStream_t.
+ * Asynchronous: enqueues the whole step on `stream`.  Workspaces of the
+ * handle are reused by the next step, so two steps of one handle must not run
+ * concurrently.  Device-detected conditions: see normpre_sync_status().
+ * Errors: ARG, ALIGN, CUDA.
+ */
+int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const void* const* G,
+                 void* const* M, void* stream);
+
+/*
+ * The same step on HOST buffers: copies W, G and M from host memory to device
+ * staging buffers owned by the handle (allocated on the first call), runs
+ * normpre_step, copies W and M back, and synchronizes `stream`.  Host buffers
+ * should be pinned (cudaHostAlloc / torch pin_memory) for full copy speed.
+ * Errors: as normpre_step, plus the device-detected conditions of the step.
+ */
+int normpre_step_host(normpre_handle* h, int64_t t, float lr, void* const* W_host,
+                      const void* const* G_host, void* const* M_host, void* stream);
+
+/*
+ * Synchronizes `stream`, then reports and clears the device-side flags set
+ * since the last call: NONFINITE, NUMERIC or TIMEOUT (the first one found, in
+ * that order), else OK.
+ */
+int normpre_sync_status(normpre_handle* h, void* stream);
+
+/* What normpre_read / normpre_buffer_info can return for one matrix. */
+enum normpre_buffer {
+  NORMPRE_BUF_PSI = 0,    /* Psi in the stored layout (rows x cols): the normalized update of the
+                             last step; bf16 in NORMPRE_PREC_BF16 with NORMPRE_G, else fp32 */
+  NORMPRE_BUF_T = 1,      /* NormPre-G: Newton-Schulz result T in the stored layout (rows x cols),
+                             same dtype as PSI */
+  NORMPRE_BUF_Q = 2,      /* NormPre-L: orthonormal basis Q of the sketch, m_a x l, fp32 */
+  NORMPRE_BUF_RITZ = 3,   /* NormPre-L: all l Ritz values, descending, fp32 (1 x l) */
+  NORMPRE_BUF_Z = 4,      /* NormPre-L: Ritz vectors Z (l x l, column j = j-th Ritz value), fp32 */
+  NORMPRE_BUF_OMEGA = 5,  /* NormPre-L: sketch matrix Omega of the last step, n_a x l, fp32 */
+  NORMPRE_BUF_STATS = 6   /* 1 x 8 fp32: [k, m', ||T||_F^2, |C|, l, n_a, m_a, 0] of the last step */
+};
+
+/*
+ * Shape and dtype of a readable buffer of matrix `mat` (after at least one
+ * step).  Errors: ARG (bad mat / what / buffer absent for this variant).
+ */
+int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* rows, int64_t* cols,
+                        int* dtype);
+
+/*
+ * Synchronizes the device and copies buffer `what` of matrix `mat` into the
+ * host array `dst` (row-major, `capacity_bytes` long).  Intended for tests and
+ * diagnostics.  Errors: ARG (too small / absent), CUDA.
+ */
+int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capacity_bytes);
+
+/*
+ * Stand-alone Newton-Schulz (the NormPre-G preconditioner of Sec. 3.2 and
+ * App. B; also Muon's orthogonalization):
+ *   T_b = NS_q(X_b) for b < batch, X_b rows x cols, contiguous [batch][rows][cols].
+ * X and T are device pointers of dtype BF16 when cfg->precision is
+ * NORMPRE_PREC_BF16 and F32 otherwise.  X is scaled by 1/(||X_b||_F + eps)
+ * first (the scale is computed on the device) and transposed internally when
+ * rows > cols.  Uses cfg->ns_steps and cfg->ns_coef.  Allocates its workspace
+ * per call and synchronizes `stream` before returning.
+ * Errors: ARG, SHAPE, ALIGN, CUDA, TIMEOUT.
+ */
+int normpre_newton_schulz(const normpre_config* cfg, int batch, int64_t rows, int64_t cols,
+                          const void* X, void* T, void* stream);
+
+/*
+ * Per-phase timing of this library's kernels (tests and benchmarks).
+ * normpre_profile(h, 1) makes every later step record a pair of CUDA events
+ * around each launch group on the step's stream (a few microseconds per step);
+ * 0 turns it off.  Kernel launches are always counted.
+ */
+int normpre_profile(normpre_handle* h, int enable);
+
+/* Kernel classes of normpre_profile_read. */
+enum normpre_profile_class {
+  NORMPRE_PROF_NORMALIZE = 0,  /* momentum + tangent + normalization (all passes) */
+  NORMPRE_PROF_NS_GRAM = 1,    /* Newton-Schulz A = X X^T (or X^T X) */
+  NORMPRE_PROF_NS_POLY = 2,    /* Newton-Schulz B = b A + c A^2 */
+  NORMPRE_PROF_NS_UPDATE = 3,  /* Newton-Schulz X <- a X + B X (or a X + X B) */
+  NORMPRE_PROF_APPLY_G = 4,    /* NormPre-G RMS-matched weight update */
+  NORMPRE_PROF_OMEGA = 5,      /* Philox sketch matrix */
+  NORMPRE_PROF_CONTRACT = 6,   /* sketch contractions Psi V and Psi^T U */
+  NORMPRE_PROF_QR = 7,         /* CholeskyQR passes */
+  NORMPRE_PROF_EIG = 8,        /* Rayleigh-Ritz Gram, Jacobi eigensolver, Q K */
+  NORMPRE_PROF_APPLY_L = 9,    /* NormPre-L projector apply + weight update */
+  NORMPRE_PROF_PRESCALE = 10,  /* Newton-Schulz input scale 1/(sqrt(m') + eps) */
+  NORMPRE_PROF_CLASSES = 11
+};
+
+/*
+ * Synchronizes on the recorded events and writes, for each of the first
+ * `n_classes` kernel classes, the summed event time in ms (`ms`, zero when
+ * profiling was off) and the number of kernel launches (`launches`) since the
+ * previous read; then resets both.  Errors: ARG.
+ */
+int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* launches);
+
+/* Releases the handle and every device buffer it owns.  NULL is ignored. */
+void normpre_free(normpre_handle* h);
+
+/* Message of the last failure of `h` (or of the calling thread when h is NULL). */
+const char* normpre_last_error(const normpre_handle* h);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* NORMPRE_H */

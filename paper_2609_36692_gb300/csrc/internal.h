@@ -1,0 +1,235 @@
+// Host-side declarations shared by the translation units of libnormpre.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+namespace normpre {
+
+// Bits of the device status word (see normpre_sync_status).
+constexpr int kFlagNonfinite = 1;
+constexpr int kFlagNumeric = 2;
+constexpr int kFlagTimeout = 4;
+
+constexpr int kMaxBatch = 32;    // matrices served by one normalize/apply launch
+constexpr int kMaxGroups = 8;    // shape groups served by one Newton-Schulz GEMM launch
+
+inline int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+// Kernel classes of the per-phase profile (normpre_profile_read).
+enum ProfClass {
+  kProfNormalize = 0, kProfNsGram = 1, kProfNsPoly = 2, kProfNsUpdate = 3, kProfApplyG = 4,
+  kProfOmega = 5, kProfContract = 6, kProfQR = 7, kProfEig = 8, kProfApplyL = 9,
+  kProfPrescale = 10, kProfClasses = 11
+};
+
+// Counts kernel launches and, when enabled, brackets launch groups with CUDA
+// events recorded on the launch stream.
+class ProfileHook {
+ public:
+  bool on = false;
+  int64_t launches[kProfClasses] = {};
+  double ms[kProfClasses] = {};
+  void begin(int cls, cudaStream_t s) {
+    if (!on) return;
+    open_cls_ = cls;
+    open_ = take();
+    cudaEventRecord(open_, s);
+  }
+  void end(int cls, cudaStream_t s, int n_launches) {
+    launches[cls] += n_launches;
+    if (!on || !open_) return;
+    cudaEvent_t e = take();
+    cudaEventRecord(e, s);
+    marks_.push_back({open_cls_, open_, e});
+    open_ = nullptr;
+  }
+  // Waits for the recorded events and folds them into ms[].
+  void collect() {
+    for (auto& m : marks_) {
+      cudaEventSynchronize(m.b);
+      float t = 0.f;
+      cudaEventElapsedTime(&t, m.a, m.b);
+      ms[m.cls] += t;
+      pool_.push_back(m.a);
+      pool_.push_back(m.b);
+    }
+    marks_.clear();
+  }
+  void reset() {
+    collect();
+    for (int i = 0; i < kProfClasses; ++i) { ms[i] = 0; launches[i] = 0; }
+  }
+  ~ProfileHook() {
+    for (auto& m : marks_) { cudaEventDestroy(m.a); cudaEventDestroy(m.b); }
+    for (auto e : pool_) cudaEventDestroy(e);
+  }
+
+ private:
+  struct Mark { int cls; cudaEvent_t a, b; };
+  cudaEvent_t take() {
+    if (!pool_.empty()) { cudaEvent_t e = pool_.back(); pool_.pop_back(); return e; }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+  }
+  std::vector<Mark> marks_;
+  std::vector<cudaEvent_t> pool_;
+  cudaEvent_t open_ = nullptr;
+  int open_cls_ = 0;
+};
+inline int64_t cdiv(int64_t x, int64_t m) { return (x + m - 1) / m; }
+
+// ----------------------------------------------------------------------------
+// K1: momentum + relaxed tangent + diagonal-Gram normalization (normalize.cu)
+// ----------------------------------------------------------------------------
+struct NormLaunch {
+  int n = 0;                      // matrices in this launch (<= kMaxBatch)
+  int64_t rows = 0, cols = 0;     // stored shape
+  int g_dtype = 0, w_dtype = 0;   // 0 = f32, 1 = bf16
+  int psi_dtype = 0;              // dtype of the written Psi
+  const void* G[kMaxBatch] = {};
+  float* M[kMaxBatch] = {};       // in: M_{t-1}, out: M_t
+  const void* W[kMaxBatch] = {};
+  void* psi[kMaxBatch] = {};      // Psi in the stored layout, row stride psi_ld
+  int mat_id[kMaxBatch] = {};     // global matrix index (into count[])
+  int64_t psi_ld = 0;
+  float mu = 0.95f;
+  int* count = nullptr;           // [n_mats] nonzero active rows, accumulated
+  int* flags = nullptr;
+  // column-active scratch (see normalize_cols_scratch_bytes)
+  double* col_part = nullptr;
+  float2* col_coef = nullptr;
+};
+cudaError_t launch_normalize_rows(const NormLaunch& a, cudaStream_t s);
+cudaError_t launch_normalize_cols(const NormLaunch& a, cudaStream_t s);
+size_t normalize_cols_scratch_bytes(int64_t rows, int64_t cols, int n);
+
+// ----------------------------------------------------------------------------
+// K7: NormPre-G apply: W <- W - lr (target * sqrt(mn)/||T|| T + wd W) (apply.cu)
+// ----------------------------------------------------------------------------
+struct ApplyLaunch {
+  int n = 0;
+  int64_t rows = 0, cols = 0;
+  int w_dtype = 0, t_dtype = 0;
+  void* W[kMaxBatch] = {};
+  const void* T[kMaxBatch] = {};      // stored layout, row stride t_ld
+  const float* sq_part[kMaxBatch] = {};  // n_part partial sums of ||T||^2 per matrix
+  float* stats[kMaxBatch] = {};       // optional: receives [k, m', ||T||_F^2]
+  int mat_id[kMaxBatch] = {};
+  const int* count = nullptr;         // nonzero active rows per matrix (m')
+  int k = 0;                          // orientation of this step
+  int64_t t_ld = 0;
+  int n_part = 0;
+  float lr = 0, wd = 0, target = 0.2f;
+};
+cudaError_t launch_apply_g(const ApplyLaunch& a, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// Newton-Schulz (ns.cu)
+// ----------------------------------------------------------------------------
+struct NSGroupSpec {
+  int batch = 0;
+  int64_t rows = 0, cols = 0;   // stored logical shape of every matrix of the group
+};
+
+struct NSGroupBuf {
+  NSGroupSpec spec;
+  bool tall = false;            // rows > cols: the Gram matrix is X^T X
+  int64_t s = 0, big = 0;       // s = min(rows, cols), big = max(rows, cols)
+  int64_t s_pad = 0, big_pad = 0;
+  int64_t rows_pad = 0, cols_pad = 0;   // padded stored layout of X buffers
+  int bn_s = 256, bn_big = 256;         // N tile of the s x s GEMMs / of the update GEMM
+  void* X[3] = {};              // [batch][rows_pad][cols_pad]; X[0] receives Psi
+  void* A = nullptr;            // [batch][s_pad][s_pad]
+  void* B = nullptr;            // [batch][s_pad][s_pad]
+  float* inscale = nullptr;     // [batch] 1/(||Psi||_F + eps)
+  float* sq_part = nullptr;     // [batch][n_part] partial ||T||_F^2 of the last update
+  int n_part = 0;
+  size_t elem = 2;              // element size of X, A, B
+};
+
+class NSPlan {
+ public:
+  NSPlan() = default;
+  ~NSPlan();
+  // Allocates the buffers of every group and prepares launch descriptors.
+  // bf16 = true: tcgen05 tensor-core path; false: fp32 SIMT path.
+  cudaError_t init(bool bf16, const std::vector<NSGroupSpec>& groups, std::string* err);
+  // q iterations of X <- aX + (b A + c A^2) X on X[0] of every group, with
+  // X[0] scaled by inscale[] in the first iteration.  Leaves T in out_index().
+  cudaError_t run(int steps, const float coef[3], cudaStream_t s, int* flags,
+                  ProfileHook* prof = nullptr);
+  // Computes inscale[] = 1/(sqrt(count[mat_id]) + eps) for matrices whose Psi
+  // rows are unit or zero (Eq. 3), i.e. ||Psi||_F^2 = number of nonzero rows.
+  cudaError_t scale_from_count(const int* count, const int* const* group_mat_ids, float eps,
+                               cudaStream_t s, ProfileHook* prof = nullptr);
+  // Computes inscale[] = 1/(||X0||_F + eps) directly from X[0].
+  cudaError_t scale_from_norm(float eps, cudaStream_t s);
+  static int out_index(int steps) { return (steps % 2 == 1) ? 1 : 2; }
+  std::vector<NSGroupBuf>& groups() { return groups_; }
+  bool bf16() const { return bf16_; }
+  void release();
+
+ private:
+  bool bf16_ = true;
+  std::vector<NSGroupBuf> groups_;
+  std::vector<void*> allocs_;
+  void* tc_args_host_ = nullptr;   // prepared kernel arguments (opaque)
+  int num_sms_ = 0;
+  int* mat_ids_dev_ = nullptr;
+};
+
+// ----------------------------------------------------------------------------
+// NormPre-L (sketch.cu)
+// ----------------------------------------------------------------------------
+struct SketchGroup {
+  int batch = 0;
+  int64_t rows = 0, cols = 0;   // stored shape
+  int w_dtype = 0;
+  int64_t ld = 0;               // row stride of Psi (fp32)
+  int ell_rows = 0;             // l when rows are active
+  int ell_cols = 0;             // l when columns are active
+  // device buffers, all [batch][...] contiguous, fp32 unless noted
+  float* psi = nullptr;         // [rows][ld]
+  float* omega = nullptr;       // [max(rows, cols)][lmax]
+  float* y0 = nullptr;          // [max(rows, cols)][lmax]  (Y0 / Z^T / Y / Q scratch)
+  float* zt = nullptr;
+  float* y = nullptr;
+  float* q = nullptr;           // [m_a][l]
+  float* bt = nullptr;          // [n_a][l]  B^T = Psi_a^T Q
+  float* qk = nullptr;          // [m_a][l]  Q K
+  double* part = nullptr;       // split-K partial Gram sums
+  double* small = nullptr;      // [l][l] Gram / R^{-1} workspace per matrix (fp64)
+  float* kmat = nullptr;        // [l][l] K = Z_C (Lam_C^{-1/2} - I) Z_C^T
+  float* ritz = nullptr;        // [l]
+  float* zvec = nullptr;        // [l][l]
+  float* stats = nullptr;       // [8] per matrix
+  int lmax = 0;
+  int max_part = 0;
+};
+
+struct SketchParams {
+  int rank = 32, oversample = 8, power_iters = 1;
+  uint64_t seed = 0;
+  int64_t t = 0;
+  int k = 0;                    // orientation of this step
+  float lr = 0, wd = 0, target = 0.2f;
+};
+
+cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::vector<void*>& allocs);
+cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* mat_ids,
+                             const int* count, void* const* W, int* flags, cudaStream_t s,
+                             ProfileHook* prof);
+
+// Device properties cached per process.
+int device_sm_count();
+bool driver_encode_tiled(CUtensorMap* map, CUtensorMapDataType dt, uint32_t rank, void* addr,
+                         const uint64_t* dims, const uint64_t* strides_bytes, const uint32_t* box,
+                         std::string* err);
+
+}  // namespace normpre

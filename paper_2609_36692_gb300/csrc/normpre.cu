@@ -1,0 +1,551 @@
+// C ABI of the NormPre optimizer-step library: handle, shape groups,
+// workspaces and the orchestration of one step (Algorithm 1 of the paper).
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <map>
+#include <memory>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "../../include/normpre.h"
+#include "internal.h"
+
+using namespace normpre;
+
+namespace {
+
+thread_local std::string g_thread_error;
+
+struct MatInfo {
+  int64_t rows, cols;
+  int w_dtype, g_dtype;
+  int group;     // index into groups
+  int slot;      // index inside the group
+};
+
+struct Group {
+  int64_t rows, cols;
+  int w_dtype, g_dtype;
+  std::vector<int> mats;       // global matrix ids
+  int* mat_ids_dev = nullptr;  // device copy of mats
+  // NormPre-L
+  SketchGroup sk;
+};
+
+}  // namespace
+
+struct normpre_handle {
+  normpre_config cfg;
+  int device = 0;
+  int n_mats = 0;
+  std::vector<MatInfo> mats;
+  std::vector<Group> groups;
+  std::vector<void*> allocs;
+  int* count = nullptr;        // [n_mats]
+  int* flags = nullptr;        // [1]
+  float* stats = nullptr;      // [n_mats][8] (NormPre-G)
+  double* col_part = nullptr;  // column-active scratch
+  float2* col_coef = nullptr;
+  std::unique_ptr<NSPlan> ns;  // NormPre-G
+  int last_k = -1;
+  bool stepped = false;
+  // host-buffer entry point staging
+  std::vector<void*> stage_w, stage_g, stage_m;
+  ProfileHook prof;
+  std::string err;
+};
+
+namespace {
+
+int fail(normpre_handle* h, int code, const std::string& msg) {
+  if (h) h->err = msg; else g_thread_error = msg;
+  return code;
+}
+int cuda_fail(normpre_handle* h, cudaError_t e, const char* what) {
+  return fail(h, NORMPRE_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+size_t dsize(int dt) { return dt == NORMPRE_BF16 ? 2 : 4; }
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_config(const normpre_config* c, std::string* msg) {
+  if (c->variant != NORMPRE_G && c->variant != NORMPRE_L) { *msg = "variant must be NORMPRE_G or NORMPRE_L"; return NORMPRE_ERR_ARG; }
+  if (!std::isfinite(c->momentum) || !std::isfinite(c->weight_decay) || !std::isfinite(c->target_rms)) {
+    *msg = "momentum, weight_decay and target_rms must be finite"; return NORMPRE_ERR_ARG;
+  }
+  if (c->precision != NORMPRE_PREC_BF16 && c->precision != NORMPRE_PREC_F32) { *msg = "bad precision"; return NORMPRE_ERR_ARG; }
+  if (c->orientation < 0 || c->orientation > 2) { *msg = "orientation must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
+  if (c->variant == NORMPRE_G) {
+    if (c->ns_steps < 1 || c->ns_steps > 100) { *msg = "ns_steps must be in [1, 100]"; return NORMPRE_ERR_ARG; }
+    if (!std::isfinite(c->ns_coef[0]) || !std::isfinite(c->ns_coef[1]) || !std::isfinite(c->ns_coef[2]) ||
+        !(c->ns_eps >= 0.f)) { *msg = "bad Newton-Schulz coefficients or eps"; return NORMPRE_ERR_ARG; }
+  } else {
+    if (c->rank < 1 || c->oversample < 0 || c->rank + c->oversample > 64) {
+      *msg = "need rank >= 1, oversample >= 0 and rank + oversample <= 64"; return NORMPRE_ERR_ARG;
+    }
+    if (c->power_iters < 0 || c->power_iters > 8) { *msg = "power_iters must be in [0, 8]"; return NORMPRE_ERR_ARG; }
+  }
+  return NORMPRE_OK;
+}
+
+int orientation_of(const normpre_config& c, int64_t t) {
+  if (c.orientation == 1) return 0;
+  if (c.orientation == 2) return 1;
+  return static_cast<int>(((t % 2) + 2) % 2);
+}
+
+template <typename T>
+cudaError_t dalloc(normpre_handle* h, T** p, size_t bytes) {
+  void* v = nullptr;
+  cudaError_t e = cudaMalloc(&v, bytes);
+  if (e != cudaSuccess) return e;
+  h->allocs.push_back(v);
+  *p = static_cast<T*>(v);
+  return cudaMemset(v, 0, bytes);
+}
+
+}  // namespace
+
+extern "C" {
+
+void normpre_default_config(normpre_config* c) {
+  if (!c) return;
+  std::memset(c, 0, sizeof(*c));
+  c->variant = NORMPRE_G;
+  c->momentum = 0.95f;
+  c->weight_decay = 0.1f;
+  c->target_rms = 0.2f;
+  c->ns_steps = 5;
+  c->ns_coef[0] = 3.4445f;
+  c->ns_coef[1] = -4.7750f;
+  c->ns_coef[2] = 2.0315f;
+  c->ns_eps = 1e-7f;
+  c->rank = 32;
+  c->oversample = 8;
+  c->power_iters = 1;
+  c->seed = 0;
+  c->precision = NORMPRE_PREC_BF16;
+  c->orientation = 0;
+}
+
+const char* normpre_last_error(const normpre_handle* h) {
+  return h ? h->err.c_str() : g_thread_error.c_str();
+}
+
+void normpre_free(normpre_handle* h) {
+  if (!h) return;
+  cudaSetDevice(h->device);
+  cudaDeviceSynchronize();
+  h->ns.reset();
+  for (void* p : h->allocs) cudaFree(p);
+  for (auto* v : {&h->stage_w, &h->stage_g, &h->stage_m})
+    for (void* p : *v) cudaFree(p);
+  delete h;
+}
+
+int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, const int64_t* cols,
+                 const int* w_dtype, const int* g_dtype, normpre_handle** out) {
+  if (!cfg || !rows || !cols || !w_dtype || !g_dtype || !out) return fail(nullptr, NORMPRE_ERR_ARG, "null argument");
+  *out = nullptr;
+  if (n_mats < 1) return fail(nullptr, NORMPRE_ERR_ARG, "n_mats must be >= 1");
+  std::string msg;
+  int rc = check_config(cfg, &msg);
+  if (rc) return fail(nullptr, rc, msg);
+  for (int i = 0; i < n_mats; ++i) {
+    if (rows[i] < 1 || cols[i] < 1 || rows[i] > 65536 || cols[i] > 65536)
+      return fail(nullptr, NORMPRE_ERR_SHAPE, "matrix " + std::to_string(i) + ": each dimension must be in [1, 65536]");
+    if ((w_dtype[i] != NORMPRE_F32 && w_dtype[i] != NORMPRE_BF16) || (g_dtype[i] != NORMPRE_F32 && g_dtype[i] != NORMPRE_BF16))
+      return fail(nullptr, NORMPRE_ERR_DTYPE, "matrix " + std::to_string(i) + ": dtype must be NORMPRE_F32 or NORMPRE_BF16");
+  }
+  std::unique_ptr<normpre_handle> h(new normpre_handle());
+  h->cfg = *cfg;
+  h->n_mats = n_mats;
+  cudaError_t e = cudaGetDevice(&h->device);
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "cudaGetDevice");
+  // shape groups: equal (rows, cols, w dtype, g dtype)
+  std::map<std::tuple<int64_t, int64_t, int, int>, int> key2g;
+  h->mats.resize(n_mats);
+  for (int i = 0; i < n_mats; ++i) {
+    auto key = std::make_tuple(rows[i], cols[i], w_dtype[i], g_dtype[i]);
+    auto it = key2g.find(key);
+    int gi;
+    if (it == key2g.end()) {
+      gi = static_cast<int>(h->groups.size());
+      key2g[key] = gi;
+      Group g;
+      g.rows = rows[i]; g.cols = cols[i]; g.w_dtype = w_dtype[i]; g.g_dtype = g_dtype[i];
+      h->groups.push_back(g);
+    } else {
+      gi = it->second;
+    }
+    h->mats[i] = MatInfo{rows[i], cols[i], w_dtype[i], g_dtype[i], gi, static_cast<int>(h->groups[gi].mats.size())};
+    h->groups[gi].mats.push_back(i);
+  }
+  if (cfg->variant == NORMPRE_G && h->groups.size() > static_cast<size_t>(kMaxGroups))
+    return fail(nullptr, NORMPRE_ERR_SHAPE, "NormPre-G supports at most " + std::to_string(kMaxGroups) + " distinct (shape, dtype) groups per handle");
+  normpre_handle* hp = h.get();
+  if ((e = dalloc(hp, &h->count, sizeof(int) * n_mats))) return cuda_fail(nullptr, e, "cudaMalloc");
+  if ((e = dalloc(hp, &h->flags, sizeof(int) * 4))) return cuda_fail(nullptr, e, "cudaMalloc");
+  if ((e = dalloc(hp, &h->stats, sizeof(float) * 8 * n_mats))) return cuda_fail(nullptr, e, "cudaMalloc");
+  size_t scratch = 0;
+  for (Group& g : h->groups) {
+    if ((e = dalloc(hp, &g.mat_ids_dev, sizeof(int) * g.mats.size()))) return cuda_fail(nullptr, e, "cudaMalloc");
+    e = cudaMemcpy(g.mat_ids_dev, g.mats.data(), sizeof(int) * g.mats.size(), cudaMemcpyHostToDevice);
+    if (e) return cuda_fail(nullptr, e, "cudaMemcpy");
+    const int chunk = std::min<int>(kMaxBatch, static_cast<int>(g.mats.size()));
+    scratch = std::max(scratch, normalize_cols_scratch_bytes(g.rows, g.cols, chunk));
+  }
+  if ((e = dalloc(hp, &h->col_part, scratch))) return cuda_fail(nullptr, e, "cudaMalloc");
+  {
+    int64_t maxc = 1;
+    for (Group& g : h->groups) maxc = std::max<int64_t>(maxc, g.cols * std::min<int>(kMaxBatch, static_cast<int>(g.mats.size())));
+    if ((e = dalloc(hp, &h->col_coef, sizeof(float2) * maxc))) return cuda_fail(nullptr, e, "cudaMalloc");
+  }
+  if (cfg->variant == NORMPRE_G) {
+    std::vector<NSGroupSpec> specs;
+    for (Group& g : h->groups) specs.push_back(NSGroupSpec{static_cast<int>(g.mats.size()), g.rows, g.cols});
+    h->ns.reset(new NSPlan());
+    e = h->ns->init(cfg->precision == NORMPRE_PREC_BF16, specs, &msg);
+    if (e != cudaSuccess) return fail(nullptr, NORMPRE_ERR_CUDA, "Newton-Schulz plan: " + (msg.empty() ? std::string(cudaGetErrorString(e)) : msg));
+  } else {
+    for (Group& g : h->groups) {
+      g.sk.batch = static_cast<int>(g.mats.size());
+      g.sk.rows = g.rows; g.sk.cols = g.cols; g.sk.w_dtype = g.w_dtype;
+      g.sk.ld = round_up(g.cols, 8);
+      e = sketch_group_alloc(g.sk, cfg->rank, cfg->oversample, h->allocs);
+      if (e != cudaSuccess) return cuda_fail(nullptr, e, "sketch workspace");
+    }
+  }
+  e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "init");
+  *out = h.release();
+  return NORMPRE_OK;
+}
+
+int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const void* const* G, void* const* M,
+                 void* stream) {
+  if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
+  if (!W || !G || !M) return fail(h, NORMPRE_ERR_ARG, "null pointer array");
+  if (!std::isfinite(lr)) return fail(h, NORMPRE_ERR_ARG, "lr must be finite");
+  for (int i = 0; i < h->n_mats; ++i) {
+    if (!W[i] || !G[i] || !M[i]) return fail(h, NORMPRE_ERR_ARG, "matrix " + std::to_string(i) + ": null tensor pointer");
+    if (!aligned16(W[i]) || !aligned16(G[i]) || !aligned16(M[i]))
+      return fail(h, NORMPRE_ERR_ALIGN, "matrix " + std::to_string(i) + ": tensors must be 16-byte aligned");
+  }
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const normpre_config& c = h->cfg;
+  const int k = orientation_of(c, t);
+  cudaError_t e = cudaMemsetAsync(h->count, 0, sizeof(int) * h->n_mats, s);
+  if (e) return cuda_fail(h, e, "cudaMemsetAsync");
+  const bool is_g = (c.variant == NORMPRE_G);
+  const bool psi_bf16 = is_g && c.precision == NORMPRE_PREC_BF16;
+
+  // (1) momentum + relaxed tangent + diagonal-Gram normalization
+  h->prof.begin(kProfNormalize, s);
+  int n_norm = 0;
+  for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+    Group& g = h->groups[gi];
+    const int B = static_cast<int>(g.mats.size());
+    char* psi_base;
+    int64_t psi_ld, psi_bs;
+    if (is_g) {
+      NSGroupBuf& nb = h->ns->groups()[gi];
+      psi_base = static_cast<char*>(nb.X[0]);
+      psi_ld = nb.cols_pad;
+      psi_bs = nb.rows_pad * nb.cols_pad * static_cast<int64_t>(nb.elem);
+    } else {
+      psi_base = reinterpret_cast<char*>(g.sk.psi);
+      psi_ld = g.sk.ld;
+      psi_bs = g.rows * g.sk.ld * static_cast<int64_t>(sizeof(float));
+    }
+    for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
+      NormLaunch a;
+      a.n = std::min(kMaxBatch, B - c0);
+      a.rows = g.rows; a.cols = g.cols;
+      a.g_dtype = g.g_dtype; a.w_dtype = g.w_dtype; a.psi_dtype = psi_bf16 ? 1 : 0;
+      for (int i = 0; i < a.n; ++i) {
+        const int mid = g.mats[c0 + i];
+        a.G[i] = G[mid]; a.M[i] = static_cast<float*>(M[mid]); a.W[i] = W[mid];
+        a.psi[i] = psi_base + static_cast<int64_t>(c0 + i) * psi_bs;
+        a.mat_id[i] = mid;
+      }
+      a.psi_ld = psi_ld;
+      a.mu = c.momentum;
+      a.count = h->count;
+      a.flags = h->flags;
+      a.col_part = h->col_part;
+      a.col_coef = h->col_coef;
+      e = (k == 0) ? launch_normalize_rows(a, s) : launch_normalize_cols(a, s);
+      if (e) return cuda_fail(h, e, "normalize launch");
+      n_norm += (k == 0) ? 1 : 3;
+    }
+  }
+  h->prof.end(kProfNormalize, s, n_norm);
+
+  if (is_g) {
+    // (2) Newton-Schulz on every group, prescaled by 1/(sqrt(m') + eps)
+    std::vector<const int*> ids;
+    for (Group& g : h->groups) ids.push_back(g.mat_ids_dev);
+    e = h->ns->scale_from_count(h->count, ids.data(), c.ns_eps, s, &h->prof);
+    if (e) return cuda_fail(h, e, "prescale launch");
+    e = h->ns->run(c.ns_steps, c.ns_coef, s, h->flags, &h->prof);
+    if (e) return cuda_fail(h, e, "Newton-Schulz launch");
+    // (3) RMS-matched update with weight decay
+    const int oi = NSPlan::out_index(c.ns_steps);
+    h->prof.begin(kProfApplyG, s);
+    int n_apply = 0;
+    for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+      Group& g = h->groups[gi];
+      NSGroupBuf& nb = h->ns->groups()[gi];
+      const int B = static_cast<int>(g.mats.size());
+      const int64_t xs = nb.rows_pad * nb.cols_pad * static_cast<int64_t>(nb.elem);
+      for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
+        ApplyLaunch a;
+        a.n = std::min(kMaxBatch, B - c0);
+        a.rows = g.rows; a.cols = g.cols;
+        a.w_dtype = g.w_dtype; a.t_dtype = psi_bf16 ? 1 : 0;
+        for (int i = 0; i < a.n; ++i) {
+          const int mid = g.mats[c0 + i];
+          a.W[i] = W[mid];
+          a.T[i] = static_cast<char*>(nb.X[oi]) + static_cast<int64_t>(c0 + i) * xs;
+          a.sq_part[i] = nb.sq_part + static_cast<int64_t>(c0 + i) * nb.n_part;
+          a.stats[i] = h->stats + 8 * mid;
+          a.mat_id[i] = mid;
+        }
+        a.count = h->count;
+        a.k = k;
+        a.t_ld = nb.cols_pad;
+        a.n_part = nb.n_part;
+        a.lr = lr; a.wd = c.weight_decay; a.target = c.target_rms;
+        e = launch_apply_g(a, s);
+        if (e) return cuda_fail(h, e, "apply launch");
+        ++n_apply;
+      }
+    }
+    h->prof.end(kProfApplyG, s, n_apply);
+  } else {
+    SketchParams p;
+    p.rank = c.rank; p.oversample = c.oversample; p.power_iters = c.power_iters;
+    p.seed = c.seed; p.t = t; p.k = k;
+    p.lr = lr; p.wd = c.weight_decay; p.target = c.target_rms;
+    for (Group& g : h->groups) {
+      std::vector<void*> wp;
+      for (int mid : g.mats) wp.push_back(W[mid]);
+      e = run_sketch_group(g.sk, p, g.mat_ids_dev, h->count, wp.data(), h->flags, s, &h->prof);
+      if (e) return cuda_fail(h, e, "sketch launch");
+    }
+  }
+  h->last_k = k;
+  h->stepped = true;
+  return NORMPRE_OK;
+}
+
+int normpre_profile(normpre_handle* h, int enable) {
+  if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
+  h->prof.collect();
+  h->prof.on = enable != 0;
+  return NORMPRE_OK;
+}
+
+int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* launches) {
+  if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
+  if (n_classes < 0 || (n_classes > 0 && (!ms || !launches))) return fail(h, NORMPRE_ERR_ARG, "bad output arrays");
+  cudaSetDevice(h->device);
+  h->prof.collect();
+  for (int i = 0; i < n_classes; ++i) {
+    ms[i] = i < kProfClasses ? h->prof.ms[i] : 0.0;
+    launches[i] = i < kProfClasses ? h->prof.launches[i] : 0;
+  }
+  h->prof.reset();
+  return NORMPRE_OK;
+}
+
+int normpre_sync_status(normpre_handle* h, void* stream) {
+  if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
+  cudaSetDevice(h->device);
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e) return cuda_fail(h, e, "cudaStreamSynchronize");
+  int flags = 0;
+  e = cudaMemcpy(&flags, h->flags, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e) return cuda_fail(h, e, "cudaMemcpy");
+  if (flags) {
+    e = cudaMemset(h->flags, 0, sizeof(int));
+    if (e) return cuda_fail(h, e, "cudaMemset");
+  }
+  if (flags & kFlagNonfinite) return fail(h, NORMPRE_ERR_NONFINITE, "non-finite value in the momentum or the weights");
+  if (flags & kFlagNumeric) return fail(h, NORMPRE_ERR_NUMERIC, "CholeskyQR breakdown or Jacobi sweep cap reached");
+  if (flags & kFlagTimeout) return fail(h, NORMPRE_ERR_TIMEOUT, "a bounded device wait gave up");
+  return NORMPRE_OK;
+}
+
+int normpre_step_host(normpre_handle* h, int64_t t, float lr, void* const* W_host, const void* const* G_host,
+                      void* const* M_host, void* stream) {
+  if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
+  if (!W_host || !G_host || !M_host) return fail(h, NORMPRE_ERR_ARG, "null pointer array");
+  cudaSetDevice(h->device);
+  cudaError_t e;
+  if (h->stage_w.empty()) {
+    for (int i = 0; i < h->n_mats; ++i) {
+      const MatInfo& m = h->mats[i];
+      const size_t n = static_cast<size_t>(m.rows * m.cols);
+      void *pw, *pg, *pm;
+      if ((e = cudaMalloc(&pw, n * dsize(m.w_dtype)))) return cuda_fail(h, e, "cudaMalloc staging");
+      h->stage_w.push_back(pw);
+      if ((e = cudaMalloc(&pg, n * dsize(m.g_dtype)))) return cuda_fail(h, e, "cudaMalloc staging");
+      h->stage_g.push_back(pg);
+      if ((e = cudaMalloc(&pm, n * 4))) return cuda_fail(h, e, "cudaMalloc staging");
+      h->stage_m.push_back(pm);
+    }
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  for (int i = 0; i < h->n_mats; ++i) {
+    const MatInfo& m = h->mats[i];
+    const size_t n = static_cast<size_t>(m.rows * m.cols);
+    if (!W_host[i] || !G_host[i] || !M_host[i]) return fail(h, NORMPRE_ERR_ARG, "null host tensor pointer");
+    if ((e = cudaMemcpyAsync(h->stage_w[i], W_host[i], n * dsize(m.w_dtype), cudaMemcpyHostToDevice, s))) return cuda_fail(h, e, "H2D");
+    if ((e = cudaMemcpyAsync(h->stage_g[i], G_host[i], n * dsize(m.g_dtype), cudaMemcpyHostToDevice, s))) return cuda_fail(h, e, "H2D");
+    if ((e = cudaMemcpyAsync(h->stage_m[i], M_host[i], n * 4, cudaMemcpyHostToDevice, s))) return cuda_fail(h, e, "H2D");
+  }
+  int rc = normpre_step(h, t, lr, h->stage_w.data(), const_cast<const void* const*>(h->stage_g.data()),
+                        h->stage_m.data(), stream);
+  if (rc) return rc;
+  for (int i = 0; i < h->n_mats; ++i) {
+    const MatInfo& m = h->mats[i];
+    const size_t n = static_cast<size_t>(m.rows * m.cols);
+    if ((e = cudaMemcpyAsync(W_host[i], h->stage_w[i], n * dsize(m.w_dtype), cudaMemcpyDeviceToHost, s))) return cuda_fail(h, e, "D2H");
+    if ((e = cudaMemcpyAsync(M_host[i], h->stage_m[i], n * 4, cudaMemcpyDeviceToHost, s))) return cuda_fail(h, e, "D2H");
+  }
+  return normpre_sync_status(h, stream);
+}
+
+int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* rows, int64_t* cols, int* dtype) {
+  normpre_handle* hh = const_cast<normpre_handle*>(h);
+  if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
+  if (mat < 0 || mat >= h->n_mats) return fail(hh, NORMPRE_ERR_ARG, "bad matrix index");
+  if (!h->stepped) return fail(hh, NORMPRE_ERR_ARG, "no step has run yet");
+  const MatInfo& m = h->mats[mat];
+  const bool is_g = h->cfg.variant == NORMPRE_G;
+  const bool rows_active = h->last_k == 0;
+  const int64_t m_a = rows_active ? m.rows : m.cols, n_a = rows_active ? m.cols : m.rows;
+  int64_t r = 0, c = 0;
+  int dt = NORMPRE_F32;
+  switch (what) {
+    case NORMPRE_BUF_PSI:
+      r = m.rows; c = m.cols;
+      dt = (is_g && h->cfg.precision == NORMPRE_PREC_BF16) ? NORMPRE_BF16 : NORMPRE_F32;
+      break;
+    case NORMPRE_BUF_T:
+      if (!is_g) return fail(hh, NORMPRE_ERR_ARG, "T is kept only for NormPre-G");
+      r = m.rows; c = m.cols;
+      dt = h->cfg.precision == NORMPRE_PREC_BF16 ? NORMPRE_BF16 : NORMPRE_F32;
+      break;
+    case NORMPRE_BUF_Q: case NORMPRE_BUF_RITZ: case NORMPRE_BUF_Z: case NORMPRE_BUF_OMEGA: {
+      if (is_g) return fail(hh, NORMPRE_ERR_ARG, "sketch buffers exist only for NormPre-L");
+      const SketchGroup& sk = h->groups[m.group].sk;
+      const int64_t l = rows_active ? sk.ell_rows : sk.ell_cols;
+      if (what == NORMPRE_BUF_Q) { r = m_a; c = l; }
+      if (what == NORMPRE_BUF_RITZ) { r = 1; c = l; }
+      if (what == NORMPRE_BUF_Z) { r = l; c = l; }
+      if (what == NORMPRE_BUF_OMEGA) { r = n_a; c = l; }
+      break;
+    }
+    case NORMPRE_BUF_STATS:
+      r = 1; c = 8;
+      break;
+    default:
+      return fail(hh, NORMPRE_ERR_ARG, "unknown buffer");
+  }
+  if (rows) *rows = r;
+  if (cols) *cols = c;
+  if (dtype) *dtype = dt;
+  return NORMPRE_OK;
+}
+
+int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capacity_bytes) {
+  if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
+  if (!dst) return fail(h, NORMPRE_ERR_ARG, "null destination");
+  int64_t r, c;
+  int dt;
+  int rc = normpre_buffer_info(h, mat, what, &r, &c, &dt);
+  if (rc) return rc;
+  const size_t el = dsize(dt);
+  if (capacity_bytes < static_cast<int64_t>(r * c * el)) return fail(h, NORMPRE_ERR_ARG, "destination too small");
+  cudaSetDevice(h->device);
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e) return cuda_fail(h, e, "cudaDeviceSynchronize");
+  const MatInfo& m = h->mats[mat];
+  const Group& g = h->groups[m.group];
+  const bool is_g = h->cfg.variant == NORMPRE_G;
+  const void* src = nullptr;
+  int64_t src_ld = c;
+  if (what == NORMPRE_BUF_PSI || what == NORMPRE_BUF_T) {
+    if (is_g) {
+      NSGroupBuf& nb = h->ns->groups()[m.group];
+      const int idx = (what == NORMPRE_BUF_PSI) ? 0 : NSPlan::out_index(h->cfg.ns_steps);
+      src = static_cast<char*>(nb.X[idx]) + static_cast<int64_t>(m.slot) * nb.rows_pad * nb.cols_pad * nb.elem;
+      src_ld = nb.cols_pad;
+    } else {
+      src = g.sk.psi + static_cast<int64_t>(m.slot) * g.rows * g.sk.ld;
+      src_ld = g.sk.ld;
+    }
+  } else if (what == NORMPRE_BUF_STATS) {
+    src = is_g ? h->stats + 8 * mat : g.sk.stats + 8 * m.slot;
+  } else {
+    const SketchGroup& sk = g.sk;
+    const int64_t vbs = std::max(sk.rows, sk.cols) * sk.lmax;
+    const int64_t sq = static_cast<int64_t>(sk.lmax) * sk.lmax;
+    if (what == NORMPRE_BUF_Q) src = sk.q + m.slot * vbs;
+    if (what == NORMPRE_BUF_OMEGA) src = sk.omega + m.slot * vbs;
+    if (what == NORMPRE_BUF_RITZ) src = sk.ritz + m.slot * sk.lmax;
+    if (what == NORMPRE_BUF_Z) src = sk.zvec + m.slot * sq;
+  }
+  e = cudaMemcpy2D(dst, c * el, src, src_ld * el, c * el, r, cudaMemcpyDeviceToHost);
+  if (e) return cuda_fail(h, e, "cudaMemcpy2D");
+  return NORMPRE_OK;
+}
+
+int normpre_newton_schulz(const normpre_config* cfg, int batch, int64_t rows, int64_t cols, const void* X, void* T,
+                          void* stream) {
+  if (!cfg || !X || !T) return fail(nullptr, NORMPRE_ERR_ARG, "null argument");
+  if (batch < 1) return fail(nullptr, NORMPRE_ERR_ARG, "batch must be >= 1");
+  if (rows < 1 || cols < 1 || rows > 65536 || cols > 65536) return fail(nullptr, NORMPRE_ERR_SHAPE, "dimensions must be in [1, 65536]");
+  if (cfg->ns_steps < 1 || cfg->ns_steps > 100) return fail(nullptr, NORMPRE_ERR_ARG, "ns_steps must be in [1, 100]");
+  if (cfg->precision != NORMPRE_PREC_BF16 && cfg->precision != NORMPRE_PREC_F32) return fail(nullptr, NORMPRE_ERR_ARG, "bad precision");
+  if (!aligned16(X) || !aligned16(T)) return fail(nullptr, NORMPRE_ERR_ALIGN, "X and T must be 16-byte aligned");
+  const bool bf = cfg->precision == NORMPRE_PREC_BF16;
+  const size_t el = bf ? 2 : 4;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  NSPlan plan;
+  std::string msg;
+  cudaError_t e = plan.init(bf, {NSGroupSpec{batch, rows, cols}}, &msg);
+  if (e) return fail(nullptr, NORMPRE_ERR_CUDA, "Newton-Schulz plan: " + (msg.empty() ? std::string(cudaGetErrorString(e)) : msg));
+  int* flags = nullptr;
+  if ((e = cudaMalloc(&flags, sizeof(int)))) return cuda_fail(nullptr, e, "cudaMalloc");
+  cudaMemsetAsync(flags, 0, sizeof(int), s);
+  NSGroupBuf& g = plan.groups()[0];
+  const int64_t xs = g.rows_pad * g.cols_pad;
+  for (int b = 0; b < batch && !e; ++b)
+    e = cudaMemcpy2DAsync(static_cast<char*>(g.X[0]) + b * xs * el, g.cols_pad * el,
+                          static_cast<const char*>(X) + b * rows * cols * el, cols * el, cols * el, rows,
+                          cudaMemcpyDeviceToDevice, s);
+  if (!e) e = plan.scale_from_norm(cfg->ns_eps, s);
+  if (!e) e = plan.run(cfg->ns_steps, cfg->ns_coef, s, flags);
+  const int oi = NSPlan::out_index(cfg->ns_steps);
+  for (int b = 0; b < batch && !e; ++b)
+    e = cudaMemcpy2DAsync(static_cast<char*>(T) + b * rows * cols * el, cols * el,
+                          static_cast<char*>(g.X[oi]) + b * xs * el, g.cols_pad * el, cols * el, rows,
+                          cudaMemcpyDeviceToDevice, s);
+  if (!e) e = cudaStreamSynchronize(s);
+  int hf = 0;
+  if (!e) e = cudaMemcpy(&hf, flags, sizeof(int), cudaMemcpyDeviceToHost);
+  cudaFree(flags);
+  if (e) return cuda_fail(nullptr, e, "Newton-Schulz");
+  if (hf & kFlagTimeout) return fail(nullptr, NORMPRE_ERR_TIMEOUT, "a bounded device wait gave up");
+  return NORMPRE_OK;
+}
+
+}  // extern "C"

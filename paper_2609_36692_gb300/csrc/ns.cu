@@ -1,0 +1,846 @@
+// Newton-Schulz preconditioner of NormPre-G (Sec. 3.2 and App. B of the paper;
+// the iteration is Muon's: X <- a X + (b A + c A^2) X with A = X X^T, after
+// scaling X to unit Frobenius norm, and with the input transposed when it has
+// more rows than columns so that the Gram matrix is s x s, App. C).
+//
+// GB300 design:
+//   * Every matrix stays in its stored (row-major) layout.  A "wide" matrix
+//     (rows <= cols) has Gram X X^T; a "tall" one X^T X.  Instead of
+//     transposing, the GEMMs read operands either K-major or MN-major straight
+//     from the layout they are in (the tcgen05 instruction descriptor's
+//     transpose bits and the matching shared-memory descriptors).
+//   * Each of the three products of an iteration is one persistent launch over
+//     all shape groups and all matrices of a group (grouped GEMM): one CTA per
+//     SM walks a static list of 128 x BN output tiles.
+//   * bf16 path: TMA (cp.async.bulk.tensor, 128-byte swizzle) feeds a 4-stage
+//     shared-memory ring; one thread issues tcgen05.mma (kind::f16, bf16 in,
+//     fp32 accumulate) into a double-buffered TMEM accumulator; four epilogue
+//     warps read TMEM with tcgen05.ld and fuse the polynomial combine
+//     (b A + c A^2), the a X + B X add, the 1/||Psi||_F prescale of the first
+//     iteration and the ||T||_F^2 partial sums of the last one.
+//   * fp32 path (parity mode): a plain SIMT tiled GEMM with the same epilogues.
+//   * Zero padding (dims rounded up to the tile) is preserved by every product,
+//     so tiles never need bounds checks.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cstring>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace normpre {
+
+// ---------------------------------------------------------------------------
+// Driver entry point for tensor-map encoding (no link-time libcuda dependency).
+// ---------------------------------------------------------------------------
+bool driver_encode_tiled(CUtensorMap* map, CUtensorMapDataType dt, uint32_t rank, void* addr,
+                         const uint64_t* dims, const uint64_t* strides_bytes, const uint32_t* box,
+                         std::string* err) {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                                     cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !p) {
+      if (err) *err = "cuTensorMapEncodeTiled entry point unavailable";
+      return false;
+    }
+    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  cuuint64_t d[5], st[4];
+  cuuint32_t bx[5], es[5];
+  for (uint32_t i = 0; i < rank; ++i) { d[i] = dims[i]; bx[i] = box[i]; es[i] = 1; }
+  for (uint32_t i = 0; i + 1 < rank; ++i) st[i] = strides_bytes[i];
+  CUresult r = fn(map, dt, rank, addr, d, st, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (err) *err = "cuTensorMapEncodeTiled failed with CUresult " + std::to_string((int)r);
+    return false;
+  }
+  return true;
+}
+
+int device_sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+// ---------------------------------------------------------------------------
+// PTX wrappers (sm_100-family: mbarrier, TMA, tcgen05)
+// ---------------------------------------------------------------------------
+namespace tc {
+
+__device__ __forceinline__ uint32_t su32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait: gives up after ~2 s (no tile takes a fraction of that) or as
+// soon as another role of the CTA has given up.
+constexpr uint64_t kWaitNs = 2000000000ull;
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > kWaitNs) return false;
+    }
+  }
+}
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar, int c0,
+                                            int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%3, %4, %5}], [%2];" ::"r"(su32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(su32(bar)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(slot)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (bf16 operands, fp32 accumulator).
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrives on `bar` once every tcgen05 operation issued so far by this thread is done.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   su32(bar))
+               : "memory");
+}
+// 32 TMEM lanes x 32 consecutive 32-bit columns: thread i receives lane (base + i).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor (tcgen05): start address, leading and stride
+// byte offsets (all >> 4), version 1 at bits 46-47, 128-byte swizzle (2) at
+// bits 61-63.  K-major SW128 tiles: SBO = 1024 (8 rows of 128 B), LBO unused;
+// MN-major SW128 tiles: LBO = distance between 64-element MN chunks, SBO =
+// distance between 8-row K groups.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= 1ull << 46;
+  d |= 2ull << 61;
+  return d;
+}
+// Instruction descriptor of kind::f16: D fp32 (bits 4-5 = 1), A and B bf16
+// (bits 7-9 = 1, 10-12 = 1), transpose (MN-major) bits 15 / 16, N >> 3 at
+// bits 17-22, M >> 4 at bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(a_mn) << 15) |
+         (static_cast<uint32_t>(b_mn) << 16) | (static_cast<uint32_t>(N >> 3) << 17) |
+         (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+}  // namespace tc
+
+// ---------------------------------------------------------------------------
+// Grouped GEMM description shared by the tensor-core and SIMT kernels.
+//   C[b](i, j) = sum_k A_b(i, k) B_b(j, k)
+//   A_b(i, k) = a_mn ? Abuf_b[k][i] : Abuf_b[i][k]     (likewise B)
+//   out = s * (ca * aux(i, j) + cb * C(i, j)),  s = inscale[b]^scale_pow
+// ---------------------------------------------------------------------------
+struct GemmGroup {
+  CUtensorMap mapA;            // tensor-core path only (3-D, box 64 x 64 x 1)
+  CUtensorMap mapB;
+  const void* Abuf;            // SIMT path: operand bases
+  const void* Bbuf;
+  int64_t a_ld, a_bs, b_ld, b_bs;
+  int a_mn, b_mn;
+  int M, N, K, BN;
+  int batch, tiles_m, tiles_n, tile_begin;
+  float ca, cb;
+  int scale_pow;
+  void* out;
+  int64_t out_ld, out_bs;
+  const void* aux;
+  int64_t aux_ld, aux_bs;
+  const float* inscale;
+  float* sq_part;              // [batch][tiles_m * tiles_n * parts_per_tile] or null
+};
+struct GemmArgs {
+  GemmGroup g[kMaxGroups];
+  int n_groups;
+  int total_tiles;
+  int* flags;
+};
+
+__device__ __forceinline__ int decode_tile(const GemmArgs& a, int t, int& b, int& tm, int& tn) {
+  int gi = 0;
+  for (; gi < a.n_groups - 1; ++gi) {
+    const GemmGroup& g = a.g[gi];
+    if (t < g.tile_begin + g.batch * g.tiles_m * g.tiles_n) break;
+  }
+  const GemmGroup& g = a.g[gi];
+  const int per = g.tiles_m * g.tiles_n;
+  const int l = t - g.tile_begin;
+  b = l / per;
+  const int r = l - b * per;
+  tm = r / g.tiles_n;
+  tn = r - tm * g.tiles_n;
+  return gi;
+}
+
+// ---------------------------------------------------------------------------
+// tcgen05 grouped GEMM
+// ---------------------------------------------------------------------------
+constexpr int kBM = 128, kBK = 64, kStages = 4;
+constexpr int kStageA = kBM * kBK * 2;   // 16 KB
+constexpr int kStageB = 256 * kBK * 2;   // 32 KB (BN <= 256)
+constexpr int kTcThreads = 192;          // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kTmemCols = 512;           // two 128 x 256 fp32 accumulators
+constexpr size_t kTcSmem = 1024 + kStages * (kStageA + kStageB) + 256;
+
+__global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_constant__ GemmArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kStages * kStageA;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kStages * kStageB);
+  uint64_t* empty = full + kStages;
+  uint64_t* tfull = empty + kStages;   // [2]
+  uint64_t* tempty = tfull + 2;        // [2]
+  uint64_t* drain = tempty + 2;        // [1]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [kStages] last parity + 1
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      tc::mbar_init(&full[s], 1);
+      tc::mbar_init(&empty[s], 1);
+      issued[s] = 0;
+    }
+    for (int a = 0; a < 2; ++a) {
+      tc::mbar_init(&tfull[a], 1);
+      tc::mbar_init(&tempty[a], 4);
+    }
+    tc::mbar_init(drain, 1);
+    *abort_flag = 0;
+    tc::fence_barrier_init();
+    for (int gi = 0; gi < args.n_groups; ++gi) {
+      tc::prefetch_map(&args.g[gi].mapA);
+      tc::prefetch_map(&args.g[gi].mapB);
+    }
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(tmem_slot, kTmemCols);
+    tc::tmem_relinquish();
+    tc::fence_before();
+  }
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------- TMA producer (the warp waits, lane 0 issues) ----------------
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < args.total_tiles && ok; t += gridDim.x) {
+      int b, tm, tn;
+      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn)];
+      const int m0 = tm * kBM, n0 = tn * g.BN, nk = g.K / kBK;
+      const uint32_t bytes = static_cast<uint32_t>((kBM + g.BN) * kBK * 2);
+      for (int kb = 0; kb < nk; ++kb) {
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[stage], phase ^ 1u, abort_flag));
+        if (!ok) break;
+        if (lane == 0) {
+          tc::mbar_expect_tx(&full[stage], bytes);
+          issued[stage] = phase + 1;
+          const int k0 = kb * kBK;
+          uint8_t* dA = sA + stage * kStageA;
+          uint8_t* dB = sB + stage * kStageB;
+#pragma unroll
+          for (int i = 0; i < kBM / 64; ++i) {
+            if (g.a_mn) tc::tma_load_3d(dA + i * 8192, &g.mapA, &full[stage], m0 + 64 * i, k0, b);
+            else        tc::tma_load_3d(dA + i * 8192, &g.mapA, &full[stage], k0, m0 + 64 * i, b);
+          }
+          for (int i = 0; i < g.BN / 64; ++i) {
+            if (g.b_mn) tc::tma_load_3d(dB + i * 8192, &g.mapB, &full[stage], n0 + 64 * i, k0, b);
+            else        tc::tma_load_3d(dB + i * 8192, &g.mapB, &full[stage], k0, n0 + 64 * i, b);
+          }
+        }
+        __syncwarp();
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(args.flags, kFlagTimeout); }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer (the warp waits, lane 0 issues) ----------------
+    int stage = 0, it = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < args.total_tiles && ok; t += gridDim.x, ++it) {
+      int b, tm, tn;
+      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn)];
+      const int nk = g.K / kBK;
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag));
+      if (!ok) break;
+      tc::fence_after();
+      const uint32_t idesc = tc::idesc_bf16(kBM, g.BN, g.a_mn, g.b_mn);
+      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * 256);
+      for (int kb = 0; kb < nk; ++kb) {
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&full[stage], phase, abort_flag));
+        if (!ok) break;
+        tc::fence_after();
+        if (lane == 0) {
+          const uint32_t a_addr = tc::su32(sA + stage * kStageA);
+          const uint32_t b_addr = tc::su32(sB + stage * kStageB);
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = g.a_mn ? tc::sdesc(a_addr + kk * 2048, 8192, 1024)
+                                       : tc::sdesc(a_addr + kk * 32, 16, 1024);
+            const uint64_t bd = g.b_mn ? tc::sdesc(b_addr + kk * 2048, 8192, 1024)
+                                       : tc::sdesc(b_addr + kk * 32, 16, 1024);
+            tc::mma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+          }
+          tc::mma_commit(&empty[stage]);
+        }
+        __syncwarp();
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+      if (!ok) break;
+      if (lane == 0) tc::mma_commit(&tfull[acc]);
+      __syncwarp();
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(args.flags, kFlagTimeout); }
+    // every MMA issued by lane 0 has completed once `drain` fires
+    if (lane == 0) {
+      tc::mma_commit(drain);
+      volatile int never = 0;
+      tc::mbar_wait(drain, 0, &never);
+    }
+    __syncwarp();
+  } else {
+    // ---------------- epilogue: warps 2..5 ----------------
+    const int q = warp & 3;                       // TMEM lane quarter of this warp
+    const int row_in_tile = q * 32 + lane;
+    int it = 0;
+    for (int t = blockIdx.x; t < args.total_tiles; t += gridDim.x, ++it) {
+      int b, tm, tn;
+      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn)];
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      if (!tc::mbar_wait(&tfull[acc], acc_phase, abort_flag)) {
+        *abort_flag = 1;
+        raise_flag(args.flags, kFlagTimeout);
+        break;
+      }
+      tc::fence_after();
+      const int64_t row = static_cast<int64_t>(tm) * kBM + row_in_tile;
+      const int n0 = tn * g.BN;
+      float s = 1.f;
+      if (g.scale_pow) {
+        const float v = g.inscale[b];
+        s = g.scale_pow == 2 ? v * v : v;
+      }
+      const float ca = g.ca * s, cb = g.cb * s;
+      bf16* outp = static_cast<bf16*>(g.out) + b * g.out_bs + row * g.out_ld + n0;
+      const bf16* auxp = g.aux ? static_cast<const bf16*>(g.aux) + b * g.aux_bs + row * g.aux_ld + n0 : nullptr;
+      float sq = 0.f;
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * 256);
+      for (int c = 0; c < g.BN; c += 32) {
+        uint32_t r[32];
+        tc::tmem_ld32(tbase + c, r);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          float x[8];
+          if (auxp) {
+            float a8[8];
+            load8(auxp + c + 8 * v, a8);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[e] = fmaf(ca, a8[e], cb * __uint_as_float(r[8 * v + e]));
+          } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[e] = cb * __uint_as_float(r[8 * v + e]);
+          }
+          uint4 pk;
+          pk.x = pack_bf16x2(x[0], x[1]); pk.y = pack_bf16x2(x[2], x[3]);
+          pk.z = pack_bf16x2(x[4], x[5]); pk.w = pack_bf16x2(x[6], x[7]);
+          *reinterpret_cast<uint4*>(outp + c + 8 * v) = pk;
+          if (g.sq_part) {
+            const float y0 = bf16lo(pk.x), y1 = bf16hi(pk.x), y2 = bf16lo(pk.y), y3 = bf16hi(pk.y);
+            const float y4 = bf16lo(pk.z), y5 = bf16hi(pk.z), y6 = bf16lo(pk.w), y7 = bf16hi(pk.w);
+            sq += y0 * y0 + y1 * y1 + y2 * y2 + y3 * y3 + y4 * y4 + y5 * y5 + y6 * y6 + y7 * y7;
+          }
+        }
+      }
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+      if (g.sq_part) {
+        sq = warp_sum(sq);
+        if (lane == 0)
+          g.sq_part[(static_cast<int64_t>(b) * g.tiles_m * g.tiles_n + tm * g.tiles_n + tn) * 4 + q] = sq;
+      }
+    }
+  }
+
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag) {
+    // let every TMA copy still in flight land before the CTA exits
+    volatile int never = 0;
+    for (int s = 0; s < kStages; ++s)
+      if (issued[s]) tc::mbar_wait(&full[s], issued[s] - 1, &never);
+  }
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::fence_after();
+    tc::tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// SIMT grouped GEMM (fp32 parity mode): 64 x 64 tiles, 16-wide K chunks,
+// 256 threads with 4 x 4 register tiles.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) k_ns_gemm_simt(const __grid_constant__ GemmArgs args) {
+  __shared__ float As[16][64];
+  __shared__ float Bs[16][64];
+  __shared__ float red[8];
+  int b, tm, tn;
+  const GemmGroup& g = args.g[decode_tile(args, blockIdx.x, b, tm, tn)];
+  const int tid = threadIdx.x;
+  const int ty = tid >> 4, tx = tid & 15;
+  const int m0 = tm * 64, n0 = tn * 64;
+  const T* Ab = static_cast<const T*>(g.Abuf) + b * g.a_bs;
+  const T* Bb = static_cast<const T*>(g.Bbuf) + b * g.b_bs;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < g.K; k0 += 16) {
+    // stage A(i, k) for i in [m0, m0+64), k in [k0, k0+16) as As[k][i]
+    for (int e = tid; e < 1024; e += 256) {
+      int i, k;
+      if (g.a_mn) { k = e >> 6; i = e & 63; } else { i = e >> 4; k = e & 15; }
+      const int64_t gi = m0 + i, gk = k0 + k;
+      As[k][i] = to_f32(g.a_mn ? Ab[gk * g.a_ld + gi] : Ab[gi * g.a_ld + gk]);
+    }
+    for (int e = tid; e < 1024; e += 256) {
+      int j, k;
+      if (g.b_mn) { k = e >> 6; j = e & 63; } else { j = e >> 4; k = e & 15; }
+      const int64_t gj = n0 + j, gk = k0 + k;
+      Bs[k][j] = to_f32(g.b_mn ? Bb[gk * g.b_ld + gj] : Bb[gj * g.b_ld + gk]);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      float av[4], bv[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) { av[r] = As[k][ty * 4 + r]; bv[r] = Bs[k][tx * 4 + r]; }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(av[r], bv[c], acc[r][c]);
+    }
+    __syncthreads();
+  }
+  float s = 1.f;
+  if (g.scale_pow) {
+    const float v = g.inscale[b];
+    s = g.scale_pow == 2 ? v * v : v;
+  }
+  const float ca = g.ca * s, cb = g.cb * s;
+  T* out = static_cast<T*>(g.out) + b * g.out_bs;
+  const T* aux = g.aux ? static_cast<const T*>(g.aux) + b * g.aux_bs : nullptr;
+  float sq = 0.f;
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int64_t i = m0 + ty * 4 + r;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int64_t j = n0 + tx * 4 + c;
+      float x = cb * acc[r][c];
+      if (aux) x = fmaf(ca, to_f32(aux[i * g.aux_ld + j]), x);
+      const T y = from_f32<T>(x);
+      out[i * g.out_ld + j] = y;
+      const float yf = to_f32(y);
+      sq += yf * yf;
+    }
+  }
+  if (g.sq_part) {
+    sq = block_sum(sq, red);
+    if (tid == 0) g.sq_part[static_cast<int64_t>(b) * g.tiles_m * g.tiles_n + tm * g.tiles_n + tn] = sq;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Prescale 1/(||Psi||_F + eps)
+// ---------------------------------------------------------------------------
+struct ScaleArgs {
+  float* inscale[kMaxGroups];
+  const int* mat_ids[kMaxGroups];
+  int batch[kMaxGroups];
+  int n_groups;
+  float eps;
+  const int* count;
+};
+__global__ void k_scale_from_count(const ScaleArgs a) {
+  const int gi = blockIdx.x;
+  for (int b = threadIdx.x; b < a.batch[gi]; b += blockDim.x) {
+    const float m = static_cast<float>(a.count[a.mat_ids[gi][b]]);
+    a.inscale[gi][b] = 1.f / (sqrtf(m) + a.eps);
+  }
+}
+
+template <typename T>
+__global__ void k_scale_from_norm(const T* X, int64_t per, float* inscale, float eps) {
+  __shared__ double red[32];
+  const T* x = X + static_cast<int64_t>(blockIdx.x) * per;
+  double s = 0;
+  for (int64_t i = threadIdx.x; i < per; i += blockDim.x) {
+    const double v = to_f32(x[i]);
+    s += v * v;
+  }
+  s = block_sum(s, red);
+  if (threadIdx.x == 0) inscale[blockIdx.x] = static_cast<float>(1.0 / (sqrt(s) + static_cast<double>(eps)));
+}
+
+// ---------------------------------------------------------------------------
+// Host plan
+// ---------------------------------------------------------------------------
+struct NSLaunches {
+  GemmArgs gram, poly, update;    // per-iteration templates (scale / sq fields patched per run)
+  CUtensorMap xmap[kMaxGroups][3];  // tensor maps of the X ping-pong buffers
+};
+
+NSPlan::~NSPlan() { release(); }
+
+void NSPlan::release() {
+  for (void* p : allocs_) cudaFree(p);
+  allocs_.clear();
+  if (tc_args_host_) {
+    delete static_cast<NSLaunches*>(tc_args_host_);
+    tc_args_host_ = nullptr;
+  }
+  groups_.clear();
+}
+
+static bool make_map(CUtensorMap* m, void* base, int64_t rows, int64_t cols, int batch,
+                     std::string* err) {
+  const uint64_t dims[3] = {static_cast<uint64_t>(cols), static_cast<uint64_t>(rows),
+                            static_cast<uint64_t>(batch)};
+  const uint64_t strides[2] = {static_cast<uint64_t>(cols) * 2, static_cast<uint64_t>(rows * cols) * 2};
+  const uint32_t box[3] = {64, 64, 1};
+  return driver_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, err);
+}
+
+cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::string* err) {
+  release();
+  bf16_ = bf16;
+  num_sms_ = device_sm_count();
+  if (static_cast<int>(specs.size()) > kMaxGroups) {
+    if (err) *err = "too many Newton-Schulz shape groups";
+    return cudaErrorInvalidValue;
+  }
+  const int64_t tile_m = bf16 ? 128 : 64;
+  for (const NSGroupSpec& sp : specs) {
+    NSGroupBuf g;
+    g.spec = sp;
+    g.tall = sp.rows > sp.cols;
+    g.s = std::min(sp.rows, sp.cols);
+    g.big = std::max(sp.rows, sp.cols);
+    g.elem = bf16 ? 2 : 4;
+    if (bf16) {
+      g.s_pad = round_up(g.s, 128);
+      g.bn_s = (g.s_pad % 256 == 0) ? 256 : 128;
+      if (g.tall) {
+        g.big_pad = round_up(g.big, 128);
+        g.bn_big = g.bn_s;
+      } else {
+        g.big_pad = round_up(g.big, 256);
+        g.bn_big = 256;
+      }
+    } else {
+      g.s_pad = round_up(g.s, tile_m);
+      g.big_pad = round_up(g.big, tile_m);
+      g.bn_s = g.bn_big = 64;
+    }
+    g.rows_pad = g.tall ? g.big_pad : g.s_pad;
+    g.cols_pad = g.tall ? g.s_pad : g.big_pad;
+    const size_t xbytes = static_cast<size_t>(sp.batch) * g.rows_pad * g.cols_pad * g.elem;
+    const size_t abytes = static_cast<size_t>(sp.batch) * g.s_pad * g.s_pad * g.elem;
+    // tiles of the update GEMM (its epilogue emits the ||T||^2 partials)
+    const int64_t um = g.tall ? g.big_pad : g.s_pad, un = g.tall ? g.s_pad : g.big_pad;
+    const int64_t ubn = g.tall ? g.bn_s : g.bn_big;
+    const int tiles = static_cast<int>((um / tile_m) * (un / (bf16 ? ubn : 64)));
+    g.n_part = tiles * (bf16 ? 4 : 1);
+    void* p;
+    for (int i = 0; i < 3; ++i) {
+      cudaError_t e = cudaMalloc(&p, xbytes);
+      if (e != cudaSuccess) return e;
+      allocs_.push_back(p);
+      g.X[i] = p;
+      cudaMemset(p, 0, xbytes);
+    }
+    for (void** dst : {&g.A, &g.B}) {
+      cudaError_t e = cudaMalloc(&p, abytes);
+      if (e != cudaSuccess) return e;
+      allocs_.push_back(p);
+      *dst = p;
+      cudaMemset(p, 0, abytes);
+    }
+    cudaError_t e = cudaMalloc(&p, sizeof(float) * sp.batch);
+    if (e != cudaSuccess) return e;
+    allocs_.push_back(p);
+    g.inscale = static_cast<float*>(p);
+    e = cudaMalloc(&p, sizeof(float) * sp.batch * g.n_part);
+    if (e != cudaSuccess) return e;
+    allocs_.push_back(p);
+    g.sq_part = static_cast<float*>(p);
+    groups_.push_back(g);
+  }
+
+  // launch descriptors
+  NSLaunches* L = new NSLaunches();
+  std::memset(L, 0, sizeof(NSLaunches));
+  tc_args_host_ = L;
+  GemmArgs* phases[3] = {&L->gram, &L->poly, &L->update};
+  for (int ph = 0; ph < 3; ++ph) {
+    GemmArgs& a = *phases[ph];
+    a.n_groups = static_cast<int>(groups_.size());
+    int tiles = 0;
+    for (size_t gi = 0; gi < groups_.size(); ++gi) {
+      NSGroupBuf& gb = groups_[gi];
+      GemmGroup& g = a.g[gi];
+      const int64_t xs = gb.rows_pad * gb.cols_pad, as = gb.s_pad * gb.s_pad;
+      g.batch = gb.spec.batch;
+      if (ph == 0) {           // A = X X^T (wide) or X^T X (tall)
+        g.M = g.N = static_cast<int>(gb.s_pad);
+        g.K = static_cast<int>(gb.big_pad);
+        g.a_mn = g.b_mn = gb.tall ? 1 : 0;
+        g.BN = bf16 ? gb.bn_s : 64;
+        g.a_ld = g.b_ld = gb.cols_pad;
+        g.a_bs = g.b_bs = xs;
+        g.out_ld = gb.s_pad; g.out_bs = as;
+        g.ca = 0.f; g.cb = 1.f;
+      } else if (ph == 1) {    // B = b A + c A A   (A symmetric: A A = A A^T)
+        g.M = g.N = g.K = static_cast<int>(gb.s_pad);
+        g.a_mn = g.b_mn = 0;
+        g.BN = bf16 ? gb.bn_s : 64;
+        g.Abuf = g.Bbuf = gb.A;
+        g.a_ld = g.b_ld = gb.s_pad;
+        g.a_bs = g.b_bs = as;
+        g.out = gb.B; g.out_ld = gb.s_pad; g.out_bs = as;
+        g.aux = gb.A; g.aux_ld = gb.s_pad; g.aux_bs = as;
+      } else {                 // X' = a X + B X (wide) or a X + X B (tall)
+        g.K = static_cast<int>(gb.s_pad);
+        if (!gb.tall) {
+          g.M = static_cast<int>(gb.s_pad); g.N = static_cast<int>(gb.big_pad);
+          g.a_mn = 0; g.b_mn = 1;
+          g.BN = bf16 ? gb.bn_big : 64;
+          g.Abuf = gb.B; g.a_ld = gb.s_pad; g.a_bs = as;
+          g.b_ld = gb.cols_pad; g.b_bs = xs;          // Bbuf = X_in (set per run)
+        } else {
+          g.M = static_cast<int>(gb.big_pad); g.N = static_cast<int>(gb.s_pad);
+          g.a_mn = 0; g.b_mn = 0;
+          g.BN = bf16 ? gb.bn_s : 64;
+          g.a_ld = gb.cols_pad; g.a_bs = xs;          // Abuf = X_in (set per run)
+          g.Bbuf = gb.B; g.b_ld = gb.s_pad; g.b_bs = as;
+        }
+        g.out_ld = gb.cols_pad; g.out_bs = xs;
+        g.aux_ld = gb.cols_pad; g.aux_bs = xs;
+        g.cb = 1.f;
+      }
+      const int tmM = bf16 ? 128 : 64;
+      g.tiles_m = g.M / tmM;
+      g.tiles_n = g.N / g.BN;
+      g.tile_begin = tiles;
+      tiles += g.batch * g.tiles_m * g.tiles_n;
+      if (bf16) {
+        // tensor maps: Gram reads X (set per run: one map per X buffer is
+        // prepared below); poly reads A; update reads B and X.
+        if (ph == 1) {
+          if (!make_map(&g.mapA, gb.A, gb.s_pad, gb.s_pad, g.batch, err)) return cudaErrorInvalidValue;
+          g.mapB = g.mapA;
+        }
+        if (ph == 2) {
+          CUtensorMap mb;
+          if (!make_map(&mb, gb.B, gb.s_pad, gb.s_pad, g.batch, err)) return cudaErrorInvalidValue;
+          if (!gb.tall) g.mapA = mb; else g.mapB = mb;
+        }
+      }
+    }
+    a.total_tiles = tiles;
+  }
+  if (bf16) {
+    for (size_t gi = 0; gi < groups_.size(); ++gi) {
+      NSGroupBuf& gb = groups_[gi];
+      for (int i = 0; i < 3; ++i)
+        if (!make_map(&L->xmap[gi][i], gb.X[i], gb.rows_pad, gb.cols_pad, gb.spec.batch, err))
+          return cudaErrorInvalidValue;
+    }
+    cudaError_t e = cudaFuncSetAttribute(k_ns_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kTcSmem));
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t NSPlan::run(int steps, const float coef[3], cudaStream_t s, int* flags, ProfileHook* prof) {
+  ProfileHook none;
+  if (!prof) prof = &none;
+  NSLaunches* L = static_cast<NSLaunches*>(tc_args_host_);
+  if (!L) return cudaErrorInvalidValue;
+  const int ng = static_cast<int>(groups_.size());
+  const float a = coef[0], b = coef[1], c = coef[2];
+  for (int it = 0; it < steps; ++it) {
+    const int in = (it == 0) ? 0 : ((it % 2 == 1) ? 1 : 2);
+    const int out = (it % 2 == 0) ? 1 : 2;
+    const bool first = (it == 0), last = (it == steps - 1);
+    GemmArgs gram = L->gram, poly = L->poly, upd = L->update;
+    gram.flags = poly.flags = upd.flags = flags;
+    for (int gi = 0; gi < ng; ++gi) {
+      NSGroupBuf& gb = groups_[gi];
+      GemmGroup& g0 = gram.g[gi];
+      g0.Abuf = g0.Bbuf = gb.X[in];
+      g0.out = gb.A;
+      g0.scale_pow = first ? 2 : 0;
+      g0.inscale = gb.inscale;
+      GemmGroup& g1 = poly.g[gi];
+      g1.ca = b; g1.cb = c;
+      GemmGroup& g2 = upd.g[gi];
+      if (!gb.tall) g2.Bbuf = gb.X[in]; else g2.Abuf = gb.X[in];
+      g2.aux = gb.X[in];
+      g2.out = gb.X[out];
+      g2.ca = a; g2.cb = 1.f;
+      g2.scale_pow = first ? 1 : 0;
+      g2.inscale = gb.inscale;
+      g2.sq_part = last ? gb.sq_part : nullptr;
+      if (bf16_) {
+        g0.mapA = g0.mapB = L->xmap[gi][in];
+        if (!gb.tall) g2.mapB = L->xmap[gi][in]; else g2.mapA = L->xmap[gi][in];
+      }
+    }
+    GemmArgs* ph[3] = {&gram, &poly, &upd};
+    const int cls[3] = {kProfNsGram, kProfNsPoly, kProfNsUpdate};
+    for (int p = 0; p < 3; ++p) {
+      prof->begin(cls[p], s);
+      if (bf16_) {
+        const int grid = std::min(ph[p]->total_tiles, num_sms_);
+        k_ns_gemm_tc<<<grid, kTcThreads, kTcSmem, s>>>(*ph[p]);
+      } else {
+        k_ns_gemm_simt<float><<<ph[p]->total_tiles, 256, 0, s>>>(*ph[p]);
+      }
+      cudaError_t e = cudaGetLastError();
+      if (e != cudaSuccess) return e;
+      prof->end(cls[p], s, 1);
+    }
+  }
+  return cudaSuccess;
+}
+
+cudaError_t NSPlan::scale_from_count(const int* count, const int* const* group_mat_ids, float eps,
+                                     cudaStream_t s, ProfileHook* prof) {
+  ScaleArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.n_groups = static_cast<int>(groups_.size());
+  a.eps = eps;
+  a.count = count;
+  for (int gi = 0; gi < a.n_groups; ++gi) {
+    a.inscale[gi] = groups_[gi].inscale;
+    a.mat_ids[gi] = group_mat_ids[gi];
+    a.batch[gi] = groups_[gi].spec.batch;
+  }
+  if (prof) prof->begin(kProfPrescale, s);
+  k_scale_from_count<<<a.n_groups, 128, 0, s>>>(a);
+  if (prof) prof->end(kProfPrescale, s, 1);
+  return cudaGetLastError();
+}
+
+cudaError_t NSPlan::scale_from_norm(float eps, cudaStream_t s) {
+  for (NSGroupBuf& g : groups_) {
+    const int64_t per = g.rows_pad * g.cols_pad;
+    if (bf16_) k_scale_from_norm<normpre::bf16><<<g.spec.batch, 512, 0, s>>>(static_cast<const normpre::bf16*>(g.X[0]), per, g.inscale, eps);
+    else k_scale_from_norm<float><<<g.spec.batch, 512, 0, s>>>(static_cast<const float*>(g.X[0]), per, g.inscale, eps);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace normpre

@@ -1,0 +1,93 @@
+"""The C ABI library without a GPU: it builds, loads, exports every symbol the
+header declares, and rejects bad arguments on the host before any CUDA call."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "normpre.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_36692_gb300 import build
+    build.build()
+    from paper_2609_36692_gb300 import normpre as C
+    return C
+
+
+def _declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(normpre_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_abi():
+    names = _declared_functions()
+    for n in ("normpre_init", "normpre_step", "normpre_free", "normpre_last_error",
+              "normpre_newton_schulz", "normpre_step_host", "normpre_read"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    so = ctypes.CDLL(lib.LIB_PATH)
+    missing = [n for n in _declared_functions() if not hasattr(so, n)]
+    assert not missing, missing
+
+
+def test_default_config_is_the_papers(lib):
+    cfg = lib.normpre_default_config()
+    assert cfg.variant == lib.NORMPRE_G
+    assert abs(cfg.momentum - 0.95) < 1e-7
+    assert abs(cfg.weight_decay - 0.1) < 1e-7
+    assert abs(cfg.target_rms - 0.2) < 1e-7
+    assert cfg.ns_steps == 5
+    assert [round(x, 4) for x in cfg.ns_coef] == [3.4445, -4.775, 2.0315]
+    assert (cfg.rank, cfg.oversample, cfg.power_iters) == (32, 8, 1)
+    assert cfg.precision == lib.NORMPRE_PREC_BF16 and cfg.orientation == 0
+
+
+def test_host_side_argument_errors(lib):
+    C = lib
+    cfg = C.normpre_default_config()
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(cfg, [], [], [])
+    assert e.value.status == C.NORMPRE_ERR_ARG
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(cfg, [(0, 5)], [0], [0])
+    assert e.value.status == C.NORMPRE_ERR_SHAPE
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(cfg, [(4, 5)], [7], [0])
+    assert e.value.status == C.NORMPRE_ERR_DTYPE
+    bad = C.normpre_default_config(ns_steps=0)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    assert e.value.status == C.NORMPRE_ERR_ARG
+    bad = C.normpre_default_config(variant=C.NORMPRE_L, rank=60, oversample=8)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    assert e.value.status == C.NORMPRE_ERR_ARG
+    assert "rank" in C.normpre_last_error()
+    bad = C.normpre_default_config(orientation=5)
+    with pytest.raises(C.NormPreError):
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    # stand-alone Newton-Schulz: argument checks come before any device work
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_newton_schulz(cfg, 1, 4, 4, 0, 0)
+    assert e.value.status == C.NORMPRE_ERR_ARG
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_newton_schulz(cfg, 1, 0, 4, 16, 16)
+    assert e.value.status == C.NORMPRE_ERR_SHAPE
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_newton_schulz(cfg, 1, 4, 4, 17, 32)
+    assert e.value.status == C.NORMPRE_ERR_ALIGN
+
+
+def test_null_handle_calls(lib):
+    C = lib
+    so = C.load_library()
+    assert so.normpre_step(None, 0, 0.1, None, None, None, None) == C.NORMPRE_ERR_ARG
+    assert so.normpre_sync_status(None, None) == C.NORMPRE_ERR_ARG
+    so.normpre_free(None)

@@ -1,0 +1,279 @@
+"""CUDA path vs the fp64 oracle, element by element, on the same seeded inputs.
+
+Tolerances (stated by the workload and derived where it is silent):
+  * momentum M_t: fp32 fma, one rounding: |dM| <= 2.5e-7 |M|.
+  * normalization (fp32 Psi): max |dPsi_ij| / ||psi_i|| <= 1e-5.
+  * Newton-Schulz T: relative Frobenius <= 2e-2 (bf16 operands, fp32
+    accumulation) and <= 1e-4 in the fp32 parity mode.
+  * NormPre-L: largest principal-angle sine between the selected Ritz
+    subspaces <= 1e-3 (fp32), equal |C| whenever the Ritz values are >= 1e-3
+    away from 1 and from the r-th/(r+1)-th cut.
+  * weight update: the change W_{t+1} - W_t has relative Frobenius error within
+    the tolerance of T (fp32 weights); bf16 weights are compared elementwise to
+    the oracle's result within 1 bf16 ulp plus the T tolerance share.
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+from synth import inputs as S
+
+from helpers import (f32, max_row_rel, oracle_config, principal_sine, rel_fro, ritz_gaps_ok,
+                     to_device, to_host)
+
+pytestmark = pytest.mark.gpu
+
+LR = 0.02
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2609_36692_gb300 import build
+    build.build()
+
+
+def _normpre(shapes, w_dtypes, g_dtypes, **cfg):
+    from paper_2609_36692_gb300.optim import NormPre
+    return NormPre(shapes, w_dtypes, g_dtypes, **cfg)
+
+
+def _run(cfgset: S.ParamSetConfig, t: int, variant: str, precision: int, indices=None,
+         zero_weight=False, extra=None, lr=LR):
+    """Run one library step on the whole set; return (opt, inputs, W_new, M_new)."""
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    mats = [S.make_matrix(cfgset, i, zero_weight=zero_weight) for i in range(cfgset.n_mats)]
+    W, G, M = to_device(mats, cfgset.g_dtype, cfgset.w_dtype)
+    kw = dict(variant=C.NORMPRE_G if variant == "G" else C.NORMPRE_L, precision=precision,
+              rank=cfgset.rank, oversample=cfgset.oversample, power_iters=cfgset.power_iters,
+              seed=1234)
+    kw.update(extra or {})
+    opt = _normpre([(m.rows, m.cols) for m in cfgset.matrices], [cfgset.w_dtype] * cfgset.n_mats,
+                   [cfgset.g_dtype] * cfgset.n_mats, **kw)
+    opt.step(t, lr, W, G, M)
+    torch.cuda.synchronize()
+    opt.status()
+    return opt, mats, [to_host(w) for w in W], [to_host(m) for m in M]
+
+
+def _oracle(mats, i, t, variant, cfgset, lr=LR, **kw):
+    oc = oracle_config(variant, rank=cfgset.rank, oversample=cfgset.oversample,
+                       power_iters=cfgset.power_iters, seed=1234, **kw)
+    m = mats[i]
+    return O.normpre_step(m["W"], m["G"], m["M"], t, f32(lr), oc, matrix_id=i)
+
+
+def _stored(x, k):
+    return x if k == 0 else x.T
+
+
+SMALL = S.custom_config("small_mixed", [(128, 384), (128, 128), (128, 512), (512, 128)],
+                        g_dtype="bf16", w_dtype="f32", row_sigma=1.0, col_sigma=1.0,
+                        rank=8, oversample=8)
+RAGGED = S.custom_config("ragged", [(50, 203), (203, 50), (1, 77), (77, 1), (33, 33)],
+                         g_dtype="f32", w_dtype="f32", row_sigma=1.0, rank=4, oversample=4)
+SINGLE = S.CONFIGS["single_256x1024"]
+
+
+# ---------------------------------------------------------------------------
+# momentum + relaxed tangent + normalization
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("t", [0, 1])
+@pytest.mark.parametrize("w_dtype", ["f32", "bf16"])
+def test_normalize_and_momentum(cfgset, t, w_dtype):
+    import dataclasses
+    cs = dataclasses.replace(cfgset, w_dtype=w_dtype)
+    opt, mats, W1, M1 = _run(cs, t, "L", precision=1)
+    for i in range(cs.n_mats):
+        ref = _oracle(mats, i, t, "L", cs)
+        k = ref["k"]
+        psi = opt.read(i, 0)   # NORMPRE_BUF_PSI
+        assert max_row_rel(psi, _stored(ref["Psi"], k)) <= 1e-5, (cs.name, i)
+        dm = np.abs(M1[i].astype(np.float64) - ref["M"])
+        assert np.all(dm <= 2.5e-7 * np.abs(ref["M"]) + 1e-30), (cs.name, i, dm.max())
+        st = opt.read(i, 6)[0]
+        assert int(st[0]) == k and int(st[1]) == int((ref["d"] > 0).sum())
+
+
+# ---------------------------------------------------------------------------
+# NormPre-G
+# ---------------------------------------------------------------------------
+def _check_g(cs, t, precision, tol_t, indices=None):
+    from paper_2609_36692_gb300 import normpre as C
+    opt, mats, W1, _ = _run(cs, t, "G", precision)
+    idx = range(cs.n_mats) if indices is None else indices
+    for i in idx:
+        ref = _oracle(mats, i, t, "G", cs)
+        T = opt.read(i, C.NORMPRE_BUF_T)
+        err = rel_fro(T, _stored(ref["T"], ref["k"]))
+        assert err <= tol_t, (cs.name, i, err)
+        dW = W1[i].astype(np.float64) - mats[i]["W"]
+        dW_ref = ref["W"] - mats[i]["W"]
+        if cs.w_dtype == "f32":
+            assert rel_fro(dW, dW_ref) <= tol_t, (cs.name, i)
+        else:
+            ulp = np.abs(S.round_to_bf16(ref["W"].astype(np.float32)).astype(np.float64)) * 2.0 ** -8
+            assert np.all(np.abs(W1[i] - ref["W"]) <= ulp + tol_t * np.abs(dW_ref).max()), (cs.name, i)
+        st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
+        assert abs(st[2] - (ref["T"] ** 2).sum()) <= 4 * tol_t * (ref["T"] ** 2).sum()
+
+
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("t", [0, 1])
+def test_g_fp32_mode(cfgset, t):
+    _check_g(cfgset, t, precision=1, tol_t=1e-4)
+
+
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("t", [0, 1])
+def test_g_bf16_tensor_cores(cfgset, t):
+    _check_g(cfgset, t, precision=0, tol_t=2e-2)
+
+
+@pytest.mark.parametrize("t", [0, 1])
+def test_g_bf16_gpt2_full_size_sampled(t):
+    """The full GPT-2 Small set in the launch configuration the bench times;
+    one matrix of each shape is checked against the oracle."""
+    cs = S.CONFIGS["gpt2_small_G"]
+    _check_g(cs, t, precision=0, tol_t=2e-2, indices=[0, 1, 2, 3, 45, 46, 47])
+
+
+# ---------------------------------------------------------------------------
+# stand-alone Newton-Schulz: every GEMM phase in isolation
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("shape", [(2, 256, 1024), (3, 384, 128), (1, 128, 128), (2, 100, 300), (1, 300, 100)])
+@pytest.mark.parametrize("coef,steps", [((0.0, 1.0, 0.0), 1), ((0.0, 0.0, 1.0), 1), ((1.0, 0.0, 0.0), 1),
+                                        ((3.4445, -4.7750, 2.0315), 5)])
+@pytest.mark.parametrize("precision", [0, 1])
+def test_newton_schulz_phases(shape, coef, steps, precision):
+    import torch
+    from paper_2609_36692_gb300.optim import newton_schulz
+    rng = np.random.default_rng(sum(shape) + steps)
+    X = rng.standard_normal(shape).astype(np.float32)
+    if precision == 0:
+        X = S.round_to_bf16(X)
+        xt = torch.from_numpy(X).cuda().to(torch.bfloat16)
+    else:
+        xt = torch.from_numpy(X).cuda()
+    T = to_host(newton_schulz(xt, ns_steps=steps, ns_coef=coef, precision=precision))
+    tol = 2e-2 if precision == 0 else 1e-4
+    for b in range(shape[0]):
+        ref = O.newton_schulz(X[b].astype(np.float64), steps, tuple(f32(c) for c in coef), f32(1e-7))
+        assert rel_fro(T[b], ref) <= tol, (shape, coef, b, rel_fro(T[b], ref))
+
+
+# ---------------------------------------------------------------------------
+# NormPre-L
+# ---------------------------------------------------------------------------
+def _check_l(cs, t, indices=None, w_tol=2e-3):
+    from paper_2609_36692_gb300 import normpre as C
+    opt, mats, W1, _ = _run(cs, t, "L", precision=1)
+    idx = range(cs.n_mats) if indices is None else indices
+    n_checked = 0
+    for i in idx:
+        ref = _oracle(mats, i, t, "L", cs)
+        sk = ref["sketch"]
+        om = opt.read(i, C.NORMPRE_BUF_OMEGA)
+        assert np.max(np.abs(om - ref["Omega"])) <= 1e-5 * (1 + np.abs(ref["Omega"]).max()), (cs.name, i)
+        ritz = opt.read(i, C.NORMPRE_BUF_RITZ)[0]
+        lam = sk["ritz"]
+        assert np.max(np.abs(ritz - lam)) <= 1e-4 * max(1.0, lam[0]), (cs.name, i)
+        st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
+        if ritz_gaps_ok(lam, cs.rank):
+            nc = int(st[3])
+            assert nc == sk["n_active"], (cs.name, i, nc, sk["n_active"])
+            Q = opt.read(i, C.NORMPRE_BUF_Q)
+            Z = opt.read(i, C.NORMPRE_BUF_Z)
+            U = Q.astype(np.float64) @ Z[:, :nc].astype(np.float64)
+            assert principal_sine(U, sk["U_C"]) <= 1e-3, (cs.name, i)
+            n_checked += 1
+        dW = W1[i].astype(np.float64) - mats[i]["W"]
+        dW_ref = ref["W"] - mats[i]["W"]
+        if cs.w_dtype == "f32":
+            assert rel_fro(dW, dW_ref) <= w_tol, (cs.name, i, rel_fro(dW, dW_ref))
+    return n_checked
+
+
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("t", [0, 1])
+def test_l_sketch(cfgset, t):
+    _check_l(cfgset, t)
+
+
+@pytest.mark.parametrize("t", [0, 1])
+def test_l_gpt2_full_size_sampled(t):
+    cs = S.CONFIGS["gpt2_small_L"]
+    _check_l(cs, t, indices=[0, 1, 2, 3, 47])
+
+
+# ---------------------------------------------------------------------------
+# edge cases and device status
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("variant", ["G", "L"])
+def test_zero_rows_and_zero_matrix(variant):
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    cs = S.custom_config("zeros", [(64, 96), (64, 96)], g_dtype="f32", w_dtype="f32", rank=4,
+                         oversample=4, prior_momentum=False)
+    mats = [S.make_matrix(cs, i) for i in range(2)]
+    mats[0]["G"][5] = 0.0
+    mats[0]["G"][17] = 0.0
+    mats[1]["G"][:] = 0.0
+    W, G, M = to_device(mats, "f32", "f32")
+    opt = _normpre([(64, 96)] * 2, ["f32"] * 2, ["f32"] * 2,
+                   variant=C.NORMPRE_G if variant == "G" else C.NORMPRE_L, precision=1, rank=4,
+                   oversample=4, seed=1234)
+    opt.step(0, LR, W, G, M)
+    torch.cuda.synchronize()
+    assert opt.status() == C.NORMPRE_OK
+    psi = opt.read(0, C.NORMPRE_BUF_PSI)
+    assert np.all(psi[5] == 0) and np.all(psi[17] == 0)
+    assert int(opt.read(0, C.NORMPRE_BUF_STATS)[0][1]) == 62
+    ref = _oracle(mats, 0, 0, variant, cs)
+    assert rel_fro(to_host(W[0]) - mats[0]["W"], ref["W"] - mats[0]["W"]) <= 1e-3
+    # an all-zero gradient: only weight decay acts
+    np.testing.assert_allclose(to_host(W[1]), mats[1]["W"] * (1 - f32(LR) * f32(0.1)), rtol=1e-6)
+
+
+def test_nonfinite_momentum_is_reported():
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    cs = S.custom_config("nan", [(32, 64)], g_dtype="f32", w_dtype="f32")
+    mats = [S.make_matrix(cs, 0)]
+    mats[0]["G"][3, 7] = np.nan
+    W, G, M = to_device(mats, "f32", "f32")
+    opt = _normpre([(32, 64)], ["f32"], ["f32"], precision=1)
+    opt.step(0, LR, W, G, M)
+    assert opt.status(raise_on_error=False) == C.NORMPRE_ERR_NONFINITE
+    # the flag is cleared once reported
+    assert opt.status(raise_on_error=False) == C.NORMPRE_OK
+
+
+@pytest.mark.parametrize("variant", ["G", "L"])
+def test_deterministic(variant):
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    cs = SMALL
+    outs = []
+    for _ in range(2):
+        opt, mats, W1, M1 = _run(cs, 1, variant, precision=0 if variant == "G" else 1)
+        outs.append(W1)
+    for a, b in zip(*outs):
+        assert np.array_equal(a, b)
+
+
+def test_host_entry_point_matches_device_step():
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    cs = SMALL
+    opt, mats, W1, M1 = _run(cs, 0, "G", precision=0)
+    opt2 = _normpre([(m.rows, m.cols) for m in cs.matrices], ["f32"] * cs.n_mats, ["bf16"] * cs.n_mats,
+                    precision=0, seed=1234)
+    Wh = [torch.from_numpy(m["W"].copy()).pin_memory() for m in mats]
+    Gh = [torch.from_numpy(m["G"]).to(torch.bfloat16).pin_memory() for m in mats]
+    Mh = [torch.from_numpy(m["M"].copy()).pin_memory() for m in mats]
+    opt2.step_host(0, LR, Wh, Gh, Mh)
+    for i in range(cs.n_mats):
+        assert np.array_equal(Wh[i].numpy(), W1[i])
+        assert np.array_equal(Mh[i].numpy(), M1[i])
