@@ -15,9 +15,15 @@
 //   * bf16 path: TMA (cp.async.bulk.tensor, 128-byte swizzle) feeds a 4-stage
 //     shared-memory ring; one thread issues tcgen05.mma (kind::f16, bf16 in,
 //     fp32 accumulate) into a double-buffered TMEM accumulator; four epilogue
-//     warps read TMEM with tcgen05.ld and fuse the polynomial combine
-//     (b A + c A^2), the a X + B X add, the 1/||Psi||_F prescale of the first
-//     iteration and the ||T||_F^2 partial sums of the last one.
+//     warps read TMEM with tcgen05.ld and fuse the polynomial combine, the
+//     1/||Psi||_F prescale of the first iteration and the ||T||_F^2 partial
+//     sums of the last one.
+//   * The iteration is evaluated as X <- C X with C = a I + b A + c A^2 formed
+//     (in fp32, rounded once) by the epilogue of the A A product.  For singular
+//     values near the quintic's fixed band a X and B X nearly cancel, so adding
+//     them after rounding B to bf16 would amplify B's rounding error; folding
+//     a I into C keeps every stored operand's relative error at one rounding
+//     and spares the update epilogue a read of X.
 //   * fp32 path (parity mode): a plain SIMT tiled GEMM with the same epilogues.
 //   * Zero padding (dims rounded up to the tile) is preserved by every product,
 //     so tiles never need bounds checks.
@@ -217,7 +223,8 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_
 // Grouped GEMM description shared by the tensor-core and SIMT kernels.
 //   C[b](i, j) = sum_k A_b(i, k) B_b(j, k)
 //   A_b(i, k) = a_mn ? Abuf_b[k][i] : Abuf_b[i][k]     (likewise B)
-//   out = s * (ca * aux(i, j) + cb * C(i, j)),  s = inscale[b]^scale_pow
+//   out = s * (ca * aux(i, j) + cb * C(i, j) + (i == j ? diag : 0)),
+//   s = inscale[b]^scale_pow
 // ---------------------------------------------------------------------------
 struct GemmGroup {
   CUtensorMap mapA;            // tensor-core path only (3-D, box 64 x 64 x 1)
@@ -228,7 +235,7 @@ struct GemmGroup {
   int a_mn, b_mn;
   int M, N, K, BN;
   int batch, tiles_m, tiles_n, tile_begin;
-  float ca, cb;
+  float ca, cb, diag;
   int scale_pow;
   void* out;
   int64_t out_ld, out_bs;
@@ -417,7 +424,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
         const float v = g.inscale[b];
         s = g.scale_pow == 2 ? v * v : v;
       }
-      const float ca = g.ca * s, cb = g.cb * s;
+      const float ca = g.ca * s, cb = g.cb * s, dg = g.diag * s;
+      const int64_t diag_col = row - n0;   // column of this thread's diagonal element in the tile
       bf16* outp = static_cast<bf16*>(g.out) + b * g.out_bs + row * g.out_ld + n0;
       const bf16* auxp = g.aux ? static_cast<const bf16*>(g.aux) + b * g.aux_bs + row * g.aux_ld + n0 : nullptr;
       float sq = 0.f;
@@ -437,6 +445,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
           } else {
 #pragma unroll
             for (int e = 0; e < 8; ++e) x[e] = cb * __uint_as_float(r[8 * v + e]);
+          }
+          if (dg != 0.f) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              if (diag_col == c + 8 * v + e) x[e] += dg;
           }
           uint4 pk;
           pk.x = pack_bf16x2(x[0], x[1]); pk.y = pack_bf16x2(x[2], x[3]);
@@ -524,7 +537,7 @@ __global__ void __launch_bounds__(256) k_ns_gemm_simt(const __grid_constant__ Ge
     const float v = g.inscale[b];
     s = g.scale_pow == 2 ? v * v : v;
   }
-  const float ca = g.ca * s, cb = g.cb * s;
+  const float ca = g.ca * s, cb = g.cb * s, dg = g.diag * s;
   T* out = static_cast<T*>(g.out) + b * g.out_bs;
   const T* aux = g.aux ? static_cast<const T*>(g.aux) + b * g.aux_bs : nullptr;
   float sq = 0.f;
@@ -536,6 +549,7 @@ __global__ void __launch_bounds__(256) k_ns_gemm_simt(const __grid_constant__ Ge
       const int64_t j = n0 + tx * 4 + c;
       float x = cb * acc[r][c];
       if (aux) x = fmaf(ca, to_f32(aux[i * g.aux_ld + j]), x);
+      if (i == j) x += dg;
       const T y = from_f32<T>(x);
       out[i * g.out_ld + j] = y;
       const float yf = to_f32(y);
@@ -723,7 +737,6 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
           g.Bbuf = gb.B; g.b_ld = gb.s_pad; g.b_bs = as;
         }
         g.out_ld = gb.cols_pad; g.out_bs = xs;
-        g.aux_ld = gb.cols_pad; g.aux_bs = xs;
         g.cb = 1.f;
       }
       const int tmM = bf16 ? 128 : 64;
@@ -782,12 +795,12 @@ cudaError_t NSPlan::run(int steps, const float coef[3], cudaStream_t s, int* fla
       g0.scale_pow = first ? 2 : 0;
       g0.inscale = gb.inscale;
       GemmGroup& g1 = poly.g[gi];
-      g1.ca = b; g1.cb = c;
+      g1.ca = b; g1.cb = c; g1.diag = a;          // C = a I + b A + c A^2
       GemmGroup& g2 = upd.g[gi];
       if (!gb.tall) g2.Bbuf = gb.X[in]; else g2.Abuf = gb.X[in];
-      g2.aux = gb.X[in];
+      g2.aux = nullptr;
       g2.out = gb.X[out];
-      g2.ca = a; g2.cb = 1.f;
+      g2.ca = 0.f; g2.cb = 1.f;                   // X' = C X (wide) or X C (tall)
       g2.scale_pow = first ? 1 : 0;
       g2.inscale = gb.inscale;
       g2.sq_part = last ? gb.sq_part : nullptr;
