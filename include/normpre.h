@@ -220,6 +220,37 @@ enum normpre_profile_class {
  */
 int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* launches);
 
+/*
+ * Allocation-free column-active normalization of ONE matrix (no counterpart
+ * in the paper: it exists for callers that cannot allocate device memory when
+ * they need this step, such as code running inside a memory-pool or allocator
+ * callback, a framework whose allocator must not be re-entered, or a process
+ * whose device memory is fully reserved in advance).  It computes what a
+ * column-active step (k = 1) of normpre_step computes before the spectral
+ * stage, with the same kernels:
+ *   M <- mu M + G;  x_j = m_j - <m_j, w_j> w_j per column j;  Psi = x_j / ||x_j||
+ * (zero columns give zero columns of Psi).
+ *   rows, cols  stored shape (row-major, contiguous), each in [1, 65536] and
+ *               rows * cols at most about 22 million (see the scratch limit).
+ *   G           device, g_dtype (NORMPRE_F32 or NORMPRE_BF16), read only.
+ *   M           device fp32, M_{t-1} on entry, M_t on return.
+ *   W           device, w_dtype, read only.
+ *   Psi         device fp32 output, rows x cols.
+ * Scratch lives in a fixed 8 MiB array in the library's device memory (held
+ * by every GPU that loads the library until the process exits); the call
+ * performs no cudaMalloc or cudaFree.  Every call shares that array, so calls
+ * whose work overlaps on the GPU (on different streams, or concurrently from
+ * several host threads on one device) race and give wrong results: order
+ * them on one stream.  The first call on each device looks up the array's
+ * device address (cudaGetSymbolAddress) with that device current; make that
+ * first call before any stream capture.  Asynchronous on `stream`; device-side
+ * conditions (non-finite input) are not reported by this entry point.
+ * Errors (message from normpre_last_error(NULL)): ARG, SHAPE (including sizes
+ * beyond the scratch array), DTYPE, ALIGN, CUDA.
+ */
+int normpre_normalize_cols_noalloc(int64_t rows, int64_t cols, float mu, const void* G, int g_dtype,
+                                   float* M, const void* W, int w_dtype, float* Psi, void* stream);
+
 /* Releases the handle and every device buffer it owns.  NULL is ignored. */
 void normpre_free(normpre_handle* h);
 

@@ -108,6 +108,7 @@ struct NormLaunch {
 cudaError_t launch_normalize_rows(const NormLaunch& a, cudaStream_t s);
 cudaError_t launch_normalize_cols(const NormLaunch& a, cudaStream_t s);
 size_t normalize_cols_scratch_bytes(int64_t rows, int64_t cols, int n);
+size_t normalize_cols_part_bytes(int64_t rows, int64_t cols, int n);   // col_part share of it
 
 // ----------------------------------------------------------------------------
 // K7: NormPre-G apply: W <- W - lr (target * sqrt(mn)/||T|| T + wd W) (apply.cu)
@@ -225,6 +226,9 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
 cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* mat_ids,
                              const int* count, void* const* W, int* flags, cudaStream_t s,
                              ProfileHook* prof);
+
+// Records the message returned by normpre_last_error(NULL) on this thread.
+void set_thread_error(const std::string& msg);
 
 // Device properties cached per process.
 int device_sm_count();

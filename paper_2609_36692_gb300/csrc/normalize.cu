@@ -26,6 +26,10 @@ namespace normpre {
 constexpr int kColRB = 64;        // rows per block in the column passes
 constexpr int kColThreads = 256;  // 32 column chunks of 8 x 8 row lanes
 
+size_t normalize_cols_part_bytes(int64_t rows, int64_t cols, int n) {
+  return static_cast<size_t>(n) * cdiv(rows, kColRB) * cols * 3 * sizeof(double);
+}
+
 size_t normalize_cols_scratch_bytes(int64_t rows, int64_t cols, int n) {
   const int64_t nrb = cdiv(rows, kColRB);
   return static_cast<size_t>(n) * nrb * cols * 3 * sizeof(double) +

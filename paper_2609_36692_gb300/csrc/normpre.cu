@@ -38,6 +38,8 @@ struct Group {
 
 }  // namespace
 
+void normpre::set_thread_error(const std::string& msg) { g_thread_error = msg; }
+
 struct normpre_handle {
   normpre_config cfg;
   int device = 0;

@@ -89,6 +89,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.normpre_profile_read.argtypes = [P, ctypes.c_int, ctypes.POINTER(ctypes.c_double),
                                          ctypes.POINTER(i64)]
     lib.normpre_profile_read.restype = ctypes.c_int
+    lib.normpre_normalize_cols_noalloc.argtypes = [i64, i64, ctypes.c_float, P, ctypes.c_int, P, P,
+                                                   ctypes.c_int, P, P]
+    lib.normpre_normalize_cols_noalloc.restype = ctypes.c_int
     lib.normpre_free.argtypes = [P]
     lib.normpre_free.restype = None
     lib.normpre_last_error.argtypes = [P]
@@ -186,6 +189,14 @@ def normpre_profile_read(handle: int):
     cnt = (ctypes.c_int64 * n)()
     _check(load_library().normpre_profile_read(handle, n, ms, cnt), handle)
     return {name: (ms[i], cnt[i]) for i, name in enumerate(PROFILE_CLASSES)}
+
+
+def normpre_normalize_cols_noalloc(rows: int, cols: int, mu: float, G_ptr: int, g_dtype: int,
+                                   M_ptr: int, W_ptr: int, w_dtype: int, Psi_ptr: int,
+                                   stream: int = 0) -> int:
+    return _check(load_library().normpre_normalize_cols_noalloc(
+        int(rows), int(cols), float(mu), G_ptr, int(g_dtype), M_ptr, W_ptr, int(w_dtype), Psi_ptr,
+        stream))
 
 
 def normpre_free(handle: int) -> None:
