@@ -41,7 +41,7 @@ LR = 0.02
 # Traffic of one launch of the dominant kernel class from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum), per workload; None until a
 # capture of the current kernel exists (profiles/ keeps the summaries).
-NCU_TRAFFIC_PER_LAUNCH = {}
+NCU_TRAFFIC_PER_LAUNCH = {"gpt2_small_G": 209.3e6}   # profiles/ns_gemm_tc_gpt2_small_G.md
 
 
 # ---------------------------------------------------------------------------
