@@ -199,7 +199,7 @@ def run_ours(args, cfg, variant, rank, world):
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream()
 
-    mats = [S.make_matrix(cfg, i) for i in range(cfg.n_mats)]
+    mats = S.make_param_set(cfg, workers=min(16, os.cpu_count() or 1))
     tdt = {"f32": torch.float32, "bf16": torch.bfloat16}
     W = [torch.from_numpy(m["W"]).to(tdt[cfg.w_dtype]).cuda() for m in mats]
     G = [torch.from_numpy(m["G"]).to(tdt[cfg.g_dtype]).cuda() for m in mats]

@@ -235,6 +235,8 @@ struct GemmGroup {
   int a_mn, b_mn;
   int M, N, K, BN;
   int batch, tiles_m, tiles_n, tile_begin;
+  int sym;                     // symmetric output: only tiles reaching the diagonal, mirrored
+  int per;                     // tiles per matrix
   float ca, cb, diag;
   int scale_pow;
   void* out;
@@ -251,19 +253,41 @@ struct GemmArgs {
   int* flags;
 };
 
+// Tiles of one matrix: the whole tiles_m x tiles_n grid, or for a symmetric
+// product only the tiles that reach the diagonal or lie above it
+// (tm <= (BN / 128)(tn + 1) - 1), enumerated column by column.
+__host__ __device__ inline int tiles_per_matrix(int tiles_m, int tiles_n, int bn, int sym) {
+  if (!sym) return tiles_m * tiles_n;
+  const int rr = bn / 128;
+  int n = 0;
+  for (int tn = 0; tn < tiles_n; ++tn) n += (rr * (tn + 1) < tiles_m) ? rr * (tn + 1) : tiles_m;
+  return n;
+}
+
 __device__ __forceinline__ int decode_tile(const GemmArgs& a, int t, int& b, int& tm, int& tn) {
   int gi = 0;
   for (; gi < a.n_groups - 1; ++gi) {
     const GemmGroup& g = a.g[gi];
-    if (t < g.tile_begin + g.batch * g.tiles_m * g.tiles_n) break;
+    if (t < g.tile_begin + g.batch * g.per) break;
   }
   const GemmGroup& g = a.g[gi];
-  const int per = g.tiles_m * g.tiles_n;
   const int l = t - g.tile_begin;
-  b = l / per;
-  const int r = l - b * per;
-  tm = r / g.tiles_n;
-  tn = r - tm * g.tiles_n;
+  b = l / g.per;
+  int r = l - b * g.per;
+  if (!g.sym) {
+    tm = r / g.tiles_n;
+    tn = r - tm * g.tiles_n;
+  } else {
+    const int rr = g.BN / 128;
+    int c = 0;
+    for (;; ++c) {
+      const int cnt = (rr * (c + 1) < g.tiles_m) ? rr * (c + 1) : g.tiles_m;
+      if (r < cnt) break;
+      r -= cnt;
+    }
+    tm = r;
+    tn = c;
+  }
   return gi;
 }
 
@@ -275,7 +299,9 @@ constexpr int kStageA = kBM * kBK * 2;   // 16 KB
 constexpr int kStageB = 256 * kBK * 2;   // 32 KB (BN <= 256)
 constexpr int kTcThreads = 192;          // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr int kTmemCols = 512;           // two 128 x 256 fp32 accumulators
-constexpr size_t kTcSmem = 1024 + kStages * (kStageA + kStageB) + 256;
+constexpr int kMirrorLd = 40;            // row stride (bf16) of the per-warp transpose buffer
+constexpr size_t kMirrorBytes = 4 * 32 * kMirrorLd * 2;
+constexpr size_t kTcSmem = 1024 + kStages * (kStageA + kStageB) + 256 + kMirrorBytes;
 
 __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_constant__ GemmArgs args) {
   extern __shared__ uint8_t smem_raw[];
@@ -290,6 +316,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [kStages] last parity + 1
+  uint16_t* mirror = reinterpret_cast<uint16_t*>(sB + kStages * kStageB + 256);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -404,21 +431,42 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
   } else {
     // ---------------- epilogue: warps 2..5 ----------------
     const int q = warp & 3;                       // TMEM lane quarter of this warp
-    const int row_in_tile = q * 32 + lane;
+    uint16_t* tbuf = mirror + q * 32 * kMirrorLd; // this warp's transpose buffer
     int it = 0;
     for (int t = blockIdx.x; t < args.total_tiles; t += gridDim.x, ++it) {
       int b, tm, tn;
       const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn)];
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
+      const int64_t r0 = static_cast<int64_t>(tm) * kBM + q * 32;   // first row of this warp
+      const int64_t row = r0 + lane;
+      const int64_t n0 = static_cast<int64_t>(tn) * g.BN;
+      bf16* outb = static_cast<bf16*>(g.out) + b * g.out_bs;
+      const bf16* auxp = g.aux ? static_cast<const bf16*>(g.aux) + b * g.aux_bs + row * g.aux_ld + n0 : nullptr;
+      // 32-column chunk kinds (rows r0.. and columns n0 + c.. are both 32-aligned):
+      // 0 = store as is (and mirror when symmetric: strictly above the diagonal),
+      // 1 = the diagonal 32 x 32 block, 2 = strictly below (written by mirrors).
+      auto kind = [&](int c) -> int {
+        if (!g.sym) return 0;
+        const int64_t j0 = n0 + c;
+        return r0 < j0 ? 0 : (r0 == j0 ? 1 : 2);
+      };
+      // the aux operand does not depend on the accumulator: fetch the first two
+      // chunks before waiting for it
+      uint4 ax[2][4];
+      if (auxp) {
+#pragma unroll
+        for (int k = 0; k < 2; ++k)
+          if (k * 32 < g.BN && kind(k * 32) != 2)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) ax[k][v] = __ldg(reinterpret_cast<const uint4*>(auxp + k * 32 + 8 * v));
+      }
       if (!tc::mbar_wait(&tfull[acc], acc_phase, abort_flag)) {
         *abort_flag = 1;
         raise_flag(args.flags, kFlagTimeout);
         break;
       }
       tc::fence_after();
-      const int64_t row = static_cast<int64_t>(tm) * kBM + row_in_tile;
-      const int n0 = tn * g.BN;
       float s = 1.f;
       if (g.scale_pow) {
         const float v = g.inscale[b];
@@ -426,41 +474,86 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
       }
       const float ca = g.ca * s, cb = g.cb * s, dg = g.diag * s;
       const int64_t diag_col = row - n0;   // column of this thread's diagonal element in the tile
-      bf16* outp = static_cast<bf16*>(g.out) + b * g.out_bs + row * g.out_ld + n0;
-      const bf16* auxp = g.aux ? static_cast<const bf16*>(g.aux) + b * g.aux_bs + row * g.aux_ld + n0 : nullptr;
       float sq = 0.f;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * 256);
-      for (int c = 0; c < g.BN; c += 32) {
+      // one 32-column chunk; `axs` holds its prefetched aux and receives the
+      // aux of chunk c + 64 (two chunks in flight)
+      auto chunk = [&](const int c, uint4 (&axs)[4]) {
+        const int kd = kind(c);
+        const bool pref = auxp && c + 64 < g.BN && kind(c + 64) != 2;
+        if (kd == 2) {
+          if (pref)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) axs[v] = __ldg(reinterpret_cast<const uint4*>(auxp + c + 64 + 8 * v));
+          return;
+        }
         uint32_t r[32];
         tc::tmem_ld32(tbase + c, r);
         tc::tmem_ld_wait();
+        uint32_t pk[16];
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
           float x[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) x[e] = cb * __uint_as_float(r[8 * v + e]);
           if (auxp) {
-            float a8[8];
-            load8(auxp + c + 8 * v, a8);
+            const uint32_t w4[4] = {axs[v].x, axs[v].y, axs[v].z, axs[v].w};
 #pragma unroll
-            for (int e = 0; e < 8; ++e) x[e] = fmaf(ca, a8[e], cb * __uint_as_float(r[8 * v + e]));
-          } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) x[e] = cb * __uint_as_float(r[8 * v + e]);
+            for (int e = 0; e < 8; ++e)
+              x[e] = fmaf(ca, (e & 1) ? bf16hi(w4[e >> 1]) : bf16lo(w4[e >> 1]), x[e]);
           }
           if (dg != 0.f) {
 #pragma unroll
             for (int e = 0; e < 8; ++e)
               if (diag_col == c + 8 * v + e) x[e] += dg;
           }
-          uint4 pk;
-          pk.x = pack_bf16x2(x[0], x[1]); pk.y = pack_bf16x2(x[2], x[3]);
-          pk.z = pack_bf16x2(x[4], x[5]); pk.w = pack_bf16x2(x[6], x[7]);
-          *reinterpret_cast<uint4*>(outp + c + 8 * v) = pk;
-          if (g.sq_part) {
-            const float y0 = bf16lo(pk.x), y1 = bf16hi(pk.x), y2 = bf16lo(pk.y), y3 = bf16hi(pk.y);
-            const float y4 = bf16lo(pk.z), y5 = bf16hi(pk.z), y6 = bf16lo(pk.w), y7 = bf16hi(pk.w);
-            sq += y0 * y0 + y1 * y1 + y2 * y2 + y3 * y3 + y4 * y4 + y5 * y5 + y6 * y6 + y7 * y7;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) pk[4 * v + e] = pack_bf16x2(x[2 * e], x[2 * e + 1]);
+        }
+        if (pref)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) axs[v] = __ldg(reinterpret_cast<const uint4*>(auxp + c + 64 + 8 * v));
+        bf16* orow = outb + row * g.out_ld + n0 + c;
+        if (kd == 0) {
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            reinterpret_cast<uint4*>(orow)[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        } else {
+          // diagonal block: this row's elements on or above the diagonal
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (e >= lane)
+              reinterpret_cast<uint16_t*>(orow)[e] =
+                  static_cast<uint16_t>((e & 1) ? (pk[e >> 1] >> 16) : (pk[e >> 1] & 0xFFFFu));
+        }
+        if (g.sq_part) {
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const float y0 = bf16lo(pk[e]), y1 = bf16hi(pk[e]);
+            sq += y0 * y0 + y1 * y1;
           }
         }
+        if (g.sym) {
+          // mirror (row, j) -> (j, row) through a 32 x 32 transpose in shared memory
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            tbuf[e * kMirrorLd + lane] = static_cast<uint16_t>((e & 1) ? (pk[e >> 1] >> 16) : (pk[e >> 1] & 0xFFFFu));
+          __syncwarp();
+          const uint16_t* src = tbuf + lane * kMirrorLd;            // column j = n0 + c + lane
+          bf16* dst = outb + (n0 + c + lane) * g.out_ld + r0;       // row j, columns r0 .. r0 + 31
+          if (kd == 0) {
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              reinterpret_cast<uint4*>(dst)[v] = reinterpret_cast<const uint4*>(src)[v];
+          } else {
+            for (int e = 0; e < lane; ++e) reinterpret_cast<uint16_t*>(dst)[e] = src[e];   // rows above j
+          }
+          __syncwarp();
+        }
+      };
+      for (int c = 0; c < g.BN; c += 64) {
+        chunk(c, ax[0]);
+        chunk(c + 32, ax[1]);
       }
       tc::fence_before();
       __syncwarp();
@@ -742,8 +835,12 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
       const int tmM = bf16 ? 128 : 64;
       g.tiles_m = g.M / tmM;
       g.tiles_n = g.N / g.BN;
+      // the Gram and polynomial products are symmetric: the tensor-core path
+      // computes the tiles on or above the diagonal and mirrors them
+      g.sym = (bf16 && ph < 2) ? 1 : 0;
+      g.per = tiles_per_matrix(g.tiles_m, g.tiles_n, g.BN, g.sym);
       g.tile_begin = tiles;
-      tiles += g.batch * g.tiles_m * g.tiles_n;
+      tiles += g.batch * g.per;
       if (bf16) {
         // tensor maps: Gram reads X (set per run: one map per X buffer is
         // prepared below); poly reads A; update reads B and X.

@@ -213,8 +213,14 @@ def make_matrix(cfg: ParamSetConfig, index: int, seed: Optional[int] = None,
 
 
 def make_param_set(cfg: ParamSetConfig, seed: Optional[int] = None,
-                   indices: Optional[List[int]] = None) -> List[Dict[str, np.ndarray]]:
-    idx = range(cfg.n_mats) if indices is None else indices
+                   indices: Optional[List[int]] = None, workers: int = 0) -> List[Dict[str, np.ndarray]]:
+    """Draw every matrix of the set (in parallel threads when workers > 1; each
+    matrix has its own random streams, so the values do not depend on it)."""
+    idx = list(range(cfg.n_mats) if indices is None else indices)
+    if workers and workers > 1 and len(idx) > 1:
+        from concurrent.futures import ThreadPoolExecutor
+        with ThreadPoolExecutor(max_workers=workers) as ex:
+            return list(ex.map(lambda i: make_matrix(cfg, i, seed), idx))
     return [make_matrix(cfg, i, seed) for i in idx]
 
 
