@@ -204,9 +204,9 @@ struct SketchGroup {
   float* q = nullptr;           // [m_a][l]
   float* bt = nullptr;          // [n_a][l]  B^T = Psi_a^T Q
   float* qk = nullptr;          // [m_a][l]  Q K
-  double* part = nullptr;       // split-K partial Gram sums
-  double* small = nullptr;      // [l][l] Gram / R^{-1} workspace per matrix (fp64)
-  float* kmat = nullptr;        // [l][l] K = Z_C (Lam_C^{-1/2} - I) Z_C^T
+  float* kpart = nullptr;       // split-K partials of the contractions
+  float* part = nullptr;        // partial Gram sums (fp32, folded with compensation)
+  float* kmat = nullptr;        // [l][l] R^{-1} of a CholeskyQR pass, then K = Z_C (Lam_C^{-1/2} - I) Z_C^T
   float* ritz = nullptr;        // [l]
   float* zvec = nullptr;        // [l][l]
   float* stats = nullptr;       // [8] per matrix

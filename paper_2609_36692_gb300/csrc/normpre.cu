@@ -58,6 +58,11 @@ struct normpre_handle {
   // host-buffer entry point staging
   std::vector<void*> stage_w, stage_g, stage_m;
   ProfileHook prof;
+  // NormPre-L: one side stream per shape group so that the groups' sketch
+  // pipelines (many small kernels each) run concurrently; joined by events
+  std::vector<cudaStream_t> side;
+  std::vector<cudaEvent_t> side_done;
+  cudaEvent_t fork_ev = nullptr;
   std::string err;
 };
 
@@ -142,6 +147,9 @@ void normpre_free(normpre_handle* h) {
   cudaSetDevice(h->device);
   cudaDeviceSynchronize();
   h->ns.reset();
+  for (cudaStream_t st : h->side) cudaStreamDestroy(st);
+  for (cudaEvent_t ev : h->side_done) cudaEventDestroy(ev);
+  if (h->fork_ev) cudaEventDestroy(h->fork_ev);
   for (void* p : h->allocs) cudaFree(p);
   for (auto* v : {&h->stage_w, &h->stage_g, &h->stage_m})
     for (void* p : *v) cudaFree(p);
@@ -219,6 +227,17 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
       g.sk.ld = round_up(g.cols, 8);
       e = sketch_group_alloc(g.sk, cfg->rank, cfg->oversample, h->allocs);
       if (e != cudaSuccess) return cuda_fail(nullptr, e, "sketch workspace");
+    }
+    if (h->groups.size() > 1) {
+      if ((e = cudaEventCreateWithFlags(&h->fork_ev, cudaEventDisableTiming))) return cuda_fail(nullptr, e, "cudaEventCreate");
+      for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+        cudaStream_t st;
+        cudaEvent_t ev;
+        if ((e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking))) return cuda_fail(nullptr, e, "cudaStreamCreate");
+        h->side.push_back(st);
+        if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming))) return cuda_fail(nullptr, e, "cudaEventCreate");
+        h->side_done.push_back(ev);
+      }
     }
   }
   e = cudaDeviceSynchronize();
@@ -334,12 +353,24 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
     p.rank = c.rank; p.oversample = c.oversample; p.power_iters = c.power_iters;
     p.seed = c.seed; p.t = t; p.k = k;
     p.lr = lr; p.wd = c.weight_decay; p.target = c.target_rms;
-    for (Group& g : h->groups) {
+    // groups run concurrently on side streams (forked from and joined back
+    // into `s`), except while per-phase profiling is on, whose event pairs
+    // must not overlap
+    const bool fork = !h->side.empty() && !h->prof.on;
+    if (fork && (e = cudaEventRecord(h->fork_ev, s))) return cuda_fail(h, e, "cudaEventRecord");
+    for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+      Group& g = h->groups[gi];
       std::vector<void*> wp;
       for (int mid : g.mats) wp.push_back(W[mid]);
-      e = run_sketch_group(g.sk, p, g.mat_ids_dev, h->count, wp.data(), h->flags, s, &h->prof);
+      cudaStream_t gs = fork ? h->side[gi] : s;
+      if (fork && (e = cudaStreamWaitEvent(gs, h->fork_ev, 0))) return cuda_fail(h, e, "cudaStreamWaitEvent");
+      e = run_sketch_group(g.sk, p, g.mat_ids_dev, h->count, wp.data(), h->flags, gs, &h->prof);
       if (e) return cuda_fail(h, e, "sketch launch");
+      if (fork && (e = cudaEventRecord(h->side_done[gi], gs))) return cuda_fail(h, e, "cudaEventRecord");
     }
+    if (fork)
+      for (size_t gi = 0; gi < h->groups.size(); ++gi)
+        if ((e = cudaStreamWaitEvent(s, h->side_done[gi], 0))) return cuda_fail(h, e, "cudaStreamWaitEvent");
   }
   h->last_k = k;
   h->stepped = true;

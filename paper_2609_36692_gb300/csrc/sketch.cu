@@ -12,12 +12,15 @@
 // contracts over stored columns ("row contract": out = Psi V) and a
 // column-active step over stored rows ("column contract": out = Psi^T U).
 //
-// Kernels: Philox4x32-10 Omega; SIMT skinny contractions (l <= 64 columns);
-// split Gram sums Y^T Y in fp32 chunks folded in fp64; CholeskyQR (three
-// passes, the first shifted when the Gram matrix is numerically singular) with
-// an fp64 Cholesky and triangular inverse; a parallel (round-robin) cyclic
-// Jacobi eigensolver in fp64 with a sweep cap; and a fused apply that forms
-// T = Psi + L R^T tile by tile and updates W in the same pass.
+// GB300 notes.  FP64 runs at a small fraction of the FP32 rate on this part,
+// so every l x l kernel (Gram folds, Cholesky, triangular solve, Jacobi)
+// works in fp32; sums that fold many partial results use compensated
+// (Kahan) addition.  The l <= 64 wide products (contractions with Psi, the
+// projector apply) keep one output row per thread with its l accumulators in
+// registers and read the small operand from shared memory by broadcast, so
+// they are bound by FMA issue rather than by shared-memory bandwidth; K is
+// split (deterministic fixed-order reduce) when a launch would not fill the
+// GPU.
 //
 // ||T||_F^2 comes from the closed form ||Psi||_F^2 - sum_C (lam_i - 1)
 // (= m' - sum_C (lam_i - 1) for unit rows), which holds for any orthonormal Q
@@ -33,6 +36,18 @@ namespace normpre {
 
 constexpr int kLmax = 64;        // largest supported sketch width l
 constexpr int kGramRows = 64;    // rows per fp32 chunk of the split Gram sums
+constexpr int kMaxKSplit = 8;    // split-K factor bound of the contractions
+
+// Kahan-compensated accumulator
+struct Kahan {
+  float s = 0.f, c = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    const float y = x - c;
+    const float t = s + y;
+    c = (t - s) - y;
+    s = t;
+  }
+};
 
 // ---------------------------------------------------------------------------
 // Philox4x32-10 (Salmon et al., SC'11) and the Gaussian test matrix Omega
@@ -85,87 +100,191 @@ __global__ void k_omega(const __grid_constant__ OmegaArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// cp.async helpers (a zero source size fills the destination with zeros)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src), "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* dst, const void* src, bool valid) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(valid ? 4 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// ---------------------------------------------------------------------------
 // Skinny contractions: out[P x l] = op(Psi) V,  op(Psi) = Psi (TRANS = false,
 // P = rows, K = cols) or Psi^T (TRANS = true, P = cols, K = rows).
-// V is [K x l] row-major (stride l), out is [P x l] (stride l).
-// 64 x 64 output tiles, K chunks of 32, 256 threads x (4 x 4).
+// V is [K x l] row-major (stride l).  With ksplit > 1 every split writes a
+// partial [P x l] block and k_split_reduce folds them in a fixed order.
+// Tile: 128 output rows x 8 CPT columns, K chunks of 32, 256 threads; thread
+// (ty, tx) = (tid / 8, tid % 8) owns rows 4 ty .. 4 ty + 3 and columns
+// CPT tx .. CPT tx + CPT - 1.  Two shared-memory stages filled by cp.async;
+// the inner loop reads four K values at a time with 16-byte loads.
 // ---------------------------------------------------------------------------
 struct ContractArgs {
   const float* psi; int64_t psi_bs, psi_ld;
   const float* v; int64_t v_bs;
-  float* out; int64_t out_bs;
+  float* out; int64_t out_bs;      // final [P][l] or partials [ksplit][P][l]
   int64_t rows, cols;
   int l;
+  int ksplit;
+  int64_t kchunk;                  // K range of one split (multiple of 32)
 };
-template <bool TRANS>
+constexpr int kCtP = 128, kCtK = 32;
+constexpr int kCtPsiLd = kCtK + 4;          // non-TRANS: Ps[p][k]
+constexpr int kCtPtLd = kCtP + 4;           // TRANS: Pt[k][p]
+constexpr int kCtVLd = kCtK + 4;            // Vt[c][k]
+constexpr int kCtPsiFloats = (kCtP * kCtPsiLd > kCtK * kCtPtLd) ? kCtP * kCtPsiLd : kCtK * kCtPtLd;
+constexpr int kCtStageFloats = kCtPsiFloats + kLmax * kCtVLd;
+constexpr size_t kCtSmem = 2 * kCtStageFloats * sizeof(float);
+
+template <bool TRANS, int CPT>
 __global__ void __launch_bounds__(256) k_contract(const __grid_constant__ ContractArgs a) {
-  __shared__ float Ps[32][64 + 4];
-  __shared__ float Vs[32][64];
-  const int b = blockIdx.y;
-  const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
+  extern __shared__ float4 ct_smem4[];
+  float* smem = reinterpret_cast<float*>(ct_smem4);
+  const int b = blockIdx.y, split = blockIdx.z;
+  const int tid = threadIdx.x, ty = tid >> 3, tx = tid & 7;
   const int64_t P = TRANS ? a.cols : a.rows, K = TRANS ? a.rows : a.cols;
-  const int64_t p0 = static_cast<int64_t>(blockIdx.x) * 64;
+  const int64_t p0 = static_cast<int64_t>(blockIdx.x) * kCtP;
+  const int64_t kbeg = static_cast<int64_t>(split) * a.kchunk;
+  const int64_t kend = min(K, kbeg + a.kchunk);
   const float* psi = a.psi + b * a.psi_bs;
   const float* v = a.v + b * a.v_bs;
   const int l = a.l;
-  float acc[4][4] = {};
-  for (int64_t k0 = 0; k0 < K; k0 += 32) {
+  const int64_t ld = a.psi_ld;
+
+  auto load_stage = [&](int st, int64_t k0) {
+    float* S = smem + st * kCtStageFloats;
+    float* Vt = S + kCtPsiFloats;
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
+    for (int q = 0; q < 4; ++q) {
       const int e = tid + 256 * q;
-      int i, k;
-      if (TRANS) { k = e >> 6; i = e & 63; } else { i = e >> 5; k = e & 31; }
-      const int64_t gp = p0 + i, gk = k0 + k;
-      float x = 0.f;
-      if (gp < P && gk < K) x = TRANS ? psi[gk * a.psi_ld + gp] : psi[gp * a.psi_ld + gk];
-      Ps[k][i] = x;
+      if (!TRANS) {
+        const int row = e >> 3, k4 = (e & 7) * 4;      // 128 rows x 8 float4
+        const int64_t gp = p0 + row, gk = k0 + k4;
+        const bool ok = gp < P && gk < kend && gk + 4 <= ld;
+        cp_async16(S + row * kCtPsiLd + k4, ok ? psi + gp * ld + gk : psi, ok);
+      } else {
+        const int k = e >> 5, p4 = (e & 31) * 4;       // 32 rows x 32 float4
+        const int64_t gk = k0 + k, gp = p0 + p4;
+        const bool ok = gk < kend && gp + 4 <= ld;
+        cp_async16(S + k * kCtPtLd + p4, ok ? psi + gk * ld + gp : psi, ok);
+      }
     }
+    // V chunk, transposed: Vt[c][k] = V[k0 + k][c]
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
       const int e = tid + 256 * q;
-      const int k = e >> 6, j = e & 63;
+      const int k = e >> 6, c = e & 63;
       const int64_t gk = k0 + k;
-      Vs[k][j] = (j < l && gk < K) ? v[gk * l + j] : 0.f;
+      const bool ok = c < l && gk < kend;
+      cp_async4(Vt + c * kCtVLd + k, ok ? v + gk * l + c : v, ok);
+    }
+    cp_async_commit();
+  };
+
+  float acc[4][CPT];
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) acc[r][c] = 0.f;
+
+  int st = 0;
+  if (kbeg < kend) load_stage(0, kbeg);
+  for (int64_t k0 = kbeg; k0 < kend; k0 += kCtK) {
+    if (k0 + kCtK < kend) {
+      load_stage(st ^ 1, k0 + kCtK);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
     __syncthreads();
-#pragma unroll 8
-    for (int k = 0; k < 32; ++k) {
-      float pv[4], vv[4];
+    const float* S = smem + st * kCtStageFloats;
+    const float* Vt = S + kCtPsiFloats;
 #pragma unroll
-      for (int r = 0; r < 4; ++r) { pv[r] = Ps[k][ty * 4 + r]; vv[r] = Vs[k][tx * 4 + r]; }
+    for (int kk = 0; kk < kCtK; kk += 4) {
+      float4 bv[CPT];
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
+      for (int c = 0; c < CPT; ++c) bv[c] = *reinterpret_cast<const float4*>(Vt + (tx * CPT + c) * kCtVLd + kk);
+      if (!TRANS) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(pv[r], vv[c], acc[r][c]);
+        for (int r = 0; r < 4; ++r) {
+          const float4 av = *reinterpret_cast<const float4*>(S + (ty * 4 + r) * kCtPsiLd + kk);
+#pragma unroll
+          for (int c = 0; c < CPT; ++c) {
+            acc[r][c] = fmaf(av.x, bv[c].x, acc[r][c]);
+            acc[r][c] = fmaf(av.y, bv[c].y, acc[r][c]);
+            acc[r][c] = fmaf(av.z, bv[c].z, acc[r][c]);
+            acc[r][c] = fmaf(av.w, bv[c].w, acc[r][c]);
+          }
+        }
+      } else {
+        float4 a4[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) a4[i] = *reinterpret_cast<const float4*>(S + (kk + i) * kCtPtLd + ty * 4);
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) {
+          const float bb[4] = {bv[c].x, bv[c].y, bv[c].z, bv[c].w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            acc[0][c] = fmaf(a4[i].x, bb[i], acc[0][c]);
+            acc[1][c] = fmaf(a4[i].y, bb[i], acc[1][c]);
+            acc[2][c] = fmaf(a4[i].z, bb[i], acc[2][c]);
+            acc[3][c] = fmaf(a4[i].w, bb[i], acc[3][c]);
+          }
+        }
+      }
     }
     __syncthreads();
+    st ^= 1;
   }
-  float* out = a.out + b * a.out_bs;
+  float* out = a.out + b * a.out_bs + static_cast<int64_t>(split) * P * l;
 #pragma unroll
   for (int r = 0; r < 4; ++r) {
     const int64_t gp = p0 + ty * 4 + r;
     if (gp >= P) continue;
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int j = tx * 4 + c;
+    for (int c = 0; c < CPT; ++c) {
+      const int j = tx * CPT + c;
       if (j < l) out[gp * l + j] = acc[r][c];
     }
   }
 }
 
+struct SplitReduceArgs {
+  const float* part; int64_t part_bs;   // [ksplit][n] per matrix
+  float* out; int64_t out_bs;
+  int64_t n;
+  int ksplit;
+};
+__global__ void k_split_reduce(const __grid_constant__ SplitReduceArgs a) {
+  const int b = blockIdx.y;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= a.n) return;
+  const float* p = a.part + b * a.part_bs + i;
+  float s = 0.f;
+  for (int k = 0; k < a.ksplit; ++k) s += p[k * a.n];
+  a.out[b * a.out_bs + i] = s;
+}
+
 // ---------------------------------------------------------------------------
-// Split Gram sums: part[b][s] = sum over rows of chunk s of y_i y_i^T (fp64),
-// each chunk accumulated in fp32 over kGramRows rows.  Y is [N x l].
+// Split Gram sums: part[b][s] = sum over the rows of chunk s of y_i y_i^T,
+// fp32 over kGramRows rows.  Y is [N x l].
 // ---------------------------------------------------------------------------
 struct GramArgs {
   const float* y; int64_t y_bs;
-  double* part; int64_t part_bs;  // [nsplit][l][l] per matrix
+  float* part; int64_t part_bs;   // [nsplit][l][l] per matrix
   int64_t n;
   int l;
   int nsplit;
 };
 __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramArgs a) {
-  __shared__ float ys[kGramRows][kLmax];
+  __shared__ float ys[kGramRows][kLmax + 1];
   const int b = blockIdx.y, s = blockIdx.x, l = a.l;
   const int64_t i0 = static_cast<int64_t>(s) * kGramRows;
   const float* y = a.y + b * a.y_bs;
@@ -174,106 +293,116 @@ __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramA
     ys[i][j] = (i0 + i < a.n) ? y[(i0 + i) * l + j] : 0.f;
   }
   __syncthreads();
-  double* out = a.part + b * a.part_bs + static_cast<int64_t>(s) * l * l;
+  float* out = a.part + b * a.part_bs + static_cast<int64_t>(s) * l * l;
   for (int e = threadIdx.x; e < l * l; e += blockDim.x) {
     const int p = e / l, q = e - p * l;
     float acc = 0.f;
+#pragma unroll 8
     for (int i = 0; i < kGramRows; ++i) acc = fmaf(ys[i][p], ys[i][q], acc);
-    out[e] = static_cast<double>(acc);
+    out[e] = acc;
+  }
+}
+
+// Folds nsplit partial l x l sums into dst (shared, row stride ld), compensated.
+// Loads are issued eight at a time so their latencies overlap.
+__device__ __forceinline__ void fold_partials(const float* part, int nsplit, int l, float* dst, int ld) {
+  const int64_t stride = static_cast<int64_t>(l) * l;
+  for (int e = threadIdx.x; e < l * l; e += blockDim.x) {
+    Kahan k;
+    int s = 0;
+    for (; s + 8 <= nsplit; s += 8) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldcg(part + (s + u) * stride + e);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) k.add(v[u]);
+    }
+    for (; s < nsplit; ++s) k.add(__ldcg(part + s * stride + e));
+    dst[(e / l) * ld + (e % l)] = k.s;
   }
 }
 
 // ---------------------------------------------------------------------------
-// Small dense helpers on l x l matrices, one CTA per matrix.
+// One CholeskyQR pass, fused: every CTA folds the Gram partials of Y,
+// factors G = R^T R (upper R, fp32; one diagonal shift when a pivot falls
+// below 1e-6 tr(G)) and then solves q R = y for 256 rows of Y, one row per
+// thread (forward substitution, R read by broadcast).  The factorization is
+// repeated by each CTA of a matrix: it is tiny next to the row solves.
 // ---------------------------------------------------------------------------
-struct CholArgs {
-  const double* part; int64_t part_bs; int nsplit;
-  double* work; int64_t work_bs;   // [2][l][l]: G, then R^{-1}
-  float* rinv; int64_t rinv_bs;    // [l][l] fp32 copy of R^{-1}
+struct CholQRArgs {
+  const float* part; int64_t part_bs; int nsplit;
+  const float* y; float* q; int64_t v_bs;    // [n][l] panels
+  int64_t n;
   int l;
-  int allow_shift;
   int* flags;
 };
-// Sums the Gram partials, Cholesky-factors G = R^T R (upper R) with one
-// optional diagonal shift on breakdown, and writes R^{-1}.
-__global__ void __launch_bounds__(256) k_chol_inv(const __grid_constant__ CholArgs a) {
-  extern __shared__ double dsm[];
+template <int LP>
+__global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRArgs a) {
+  __shared__ float Gm[LP][LP + 1];
+  __shared__ float Rm[LP][LP + 1];
   __shared__ int bad;
-  __shared__ double tr;
-  const int b = blockIdx.x, l = a.l, tid = threadIdx.x;
-  const int ld = l + 1;
-  double* Gm = dsm;              // [l][l+1]
-  double* Rm = dsm + l * ld;     // [l][l+1]
-#define G(i, j) Gm[(i) * ld + (j)]
-#define Ri(i, j) Rm[(i) * ld + (j)]
-  const double* part = a.part + b * a.part_bs;
-  for (int e = tid; e < l * l; e += blockDim.x) {
-    double s = 0;
-    for (int k = 0; k < a.nsplit; ++k) s += part[static_cast<int64_t>(k) * l * l + e];
-    G(e / l, e % l) = s;
-  }
+  __shared__ float tr;
+  const int b = blockIdx.y, l = a.l, tid = threadIdx.x;
+  if (tid == 0) bad = 0;
+  fold_partials(a.part + b * a.part_bs, a.nsplit, l, &Gm[0][0], LP + 1);
   __syncthreads();
   if (tid == 0) {
-    double t = 0;
-    for (int i = 0; i < l; ++i) t += G(i, i);
+    float t = 0.f;
+    for (int i = 0; i < l; ++i) t += Gm[i][i];
     tr = t;
   }
   __syncthreads();
-  for (int attempt = 0; attempt < 2; ++attempt) {
-    // working copy in Ri (upper triangle), shifted on the second attempt
-    const double shift = attempt == 0 ? 0.0 : 1e-6 * tr;
-    for (int e = tid; e < l * l; e += blockDim.x) {
-      const int i = e / l, j = e % l;
-      Ri(i, j) = (j >= i) ? G(i, j) + (i == j ? shift : 0.0) : 0.0;
-    }
-    if (tid == 0) bad = 0;
-    __syncthreads();
-    for (int k = 0; k < l; ++k) {
-      if (tid == 0) {
-        const double d = Ri(k, k);
-        if (!(d > 1e-13 * tr) || !isfinite(d)) bad = 1;
-        Ri(k, k) = sqrt(fmax(d, 1e-300));
-      }
-      __syncthreads();
-      const double dk = Ri(k, k);
-      for (int j = k + 1 + tid; j < l; j += blockDim.x) Ri(k, j) /= dk;
-      __syncthreads();
-      for (int e = tid; e < l * l; e += blockDim.x) {
-        const int i = e / l, j = e % l;
-        if (i > k && j >= i) Ri(i, j) -= Ri(k, i) * Ri(k, j);
-      }
-      __syncthreads();
-    }
-    if (!bad || !a.allow_shift) break;
-    __syncthreads();
-  }
-  float* ro = a.rinv + b * a.rinv_bs;
-  if (!(tr > 0)) {
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * 256 + tid;
+  const float* y = a.y + b * a.v_bs + row * l;
+  float* q = a.q + b * a.v_bs + row * l;
+  if (!(tr > 0.f)) {
     // Y = 0 (a zero normalized update): Q = 0, nothing is selected downstream
-    for (int e = tid; e < l * l; e += blockDim.x) ro[e] = 0.f;
+    if (row < a.n)
+      for (int j = 0; j < l; ++j) q[j] = 0.f;
     return;
   }
-  if (tid == 0 && bad) raise_flag(a.flags, kFlagNumeric);
-  // R is in Ri (upper).  Invert column by column: R X = I, X upper.
-  // Store R in G (upper) and build X in Ri.
-  for (int e = tid; e < l * l; e += blockDim.x) {
-    const int i = e / l, j = e % l;
-    G(i, j) = (j >= i) ? Ri(i, j) : 0.0;
-  }
-  __syncthreads();
-  for (int j = tid; j < l; j += blockDim.x) {
-    // back substitution for column j of X (X[i][j] = 0 for i > j)
-    for (int i = l - 1; i >= 0; --i) {
-      if (i > j) { Ri(i, j) = 0.0; continue; }
-      double s = (i == j) ? 1.0 : 0.0;
-      for (int k = i + 1; k <= j; ++k) s -= G(i, k) * Ri(k, j);
-      Ri(i, j) = s / G(i, i);
+  // G = R^T R, row by row in one warp (row j needs rows 0 .. j-1); the whole
+  // CTA then solves its rows of Y against R.
+  if (tid < 32) {
+    for (int attempt = 0; attempt < 2; ++attempt) {
+      const float shift = attempt == 0 ? 0.f : 1e-5f * tr;
+      int bd = 0;
+      for (int j = 0; j < l; ++j) {
+        float d = Gm[j][j] + shift;
+        for (int k = 0; k < j; ++k) d = fmaf(-Rm[k][j], Rm[k][j], d);
+        if (!(d > 1e-6f * tr)) bd = 1;
+        const float rjj = sqrtf(fmaxf(d, 1e-30f * tr));
+        for (int i = j + 1 + tid; i < l; i += 32) {
+          float v = Gm[j][i];
+          for (int k = 0; k < j; ++k) v = fmaf(-Rm[k][j], Rm[k][i], v);
+          Rm[j][i] = v / rjj;
+        }
+        if (tid == 0) Rm[j][j] = rjj;
+        __syncwarp();
+      }
+      if (!bd) break;
+      if (attempt == 1 && tid == 0) bad = 1;
     }
   }
   __syncthreads();
-  for (int e = tid; e < l * l; e += blockDim.x) ro[e] = static_cast<float>(Ri(e / l, e % l));
-#undef G
-#undef Ri
+  if (tid == 0 && bad && blockIdx.x == 0) raise_flag(a.flags, kFlagNumeric);
+  if (row >= a.n) return;
+  float x[LP];
+#pragma unroll
+  for (int j = 0; j < LP; ++j) x[j] = (j < l) ? y[j] : 0.f;
+  // q R = y  =>  q_j = (y_j - sum_{k<j} q_k R_kj) / R_jj
+#pragma unroll
+  for (int j = 0; j < LP; ++j) {
+    if (j < l) {
+      float s = x[j];
+#pragma unroll
+      for (int k = 0; k < j; ++k) s = fmaf(-x[k], Rm[k][j], s);
+      x[j] = s / Rm[j][j];
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < LP; ++j)
+    if (j < l) q[j] = x[j];
 }
 
 // out[N x l] = Y[N x l] * S[l x l] (S fp32 row-major), one thread per output
@@ -301,10 +430,14 @@ __global__ void __launch_bounds__(256) k_rowmul(const __grid_constant__ RowMulAr
 }
 
 // ---------------------------------------------------------------------------
-// Jacobi eigensolver of Gamma_Q (fp64), selection and K.
+// Parallel cyclic Jacobi (round-robin pairing) of Gamma_Q in fp32, then the
+// descending sort, the selection C and K.  One CTA per matrix; each thread
+// owns up to two (pair, row) items of every rotation step, with the item
+// indices computed once, so a step is three barriers and a handful of
+// shared-memory updates per thread.
 // ---------------------------------------------------------------------------
 struct EigArgs {
-  const double* part; int64_t part_bs; int nsplit;   // Gram partials of B^T
+  const float* part; int64_t part_bs; int nsplit;   // Gram partials of B^T
   float* ritz; int64_t ritz_bs;      // [l]
   float* z; int64_t z_bs;            // [l][l]
   float* kmat; int64_t k_bs;         // [l][l]
@@ -315,56 +448,62 @@ struct EigArgs {
   int max_sweeps;
   int* flags;
 };
-__global__ void __launch_bounds__(256) k_jacobi(const __grid_constant__ EigArgs a) {
-  extern __shared__ double dsm[];
-  __shared__ double cs[kLmax / 2], sn[kLmax / 2];
+__global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs a) {
+  extern __shared__ float4 jc_smem4[];
+  float* dsm = reinterpret_cast<float*>(jc_smem4);
+  __shared__ float cs[kLmax / 2], sn[kLmax / 2];
   __shared__ int pp[kLmax / 2], qq[kLmax / 2];
-  __shared__ double red[32];
+  __shared__ float red[32];
   __shared__ int order[kLmax];
-  const int b = blockIdx.x, l = a.l, tid = threadIdx.x;
+  const int b = blockIdx.x, l = a.l, tid = threadIdx.x, nt = blockDim.x;
   const int n = (l + 1) & ~1;          // even number of "players" (one dummy if l is odd)
+  const int npairs = n / 2;
   const int ld = l + 1;
-  double* Am = dsm;              // [l][l+1]
-  double* Vm = dsm + l * ld;     // [l][l+1]
+  float* Am = dsm;              // [l][l+1]
+  float* Vm = dsm + l * ld;     // [l][l+1]
 #define A(i, j) Am[(i) * ld + (j)]
 #define V(i, j) Vm[(i) * ld + (j)]
-  const double* part = a.part + b * a.part_bs;
-  for (int e = tid; e < l * l; e += blockDim.x) {
-    double s = 0;
-    for (int k = 0; k < a.nsplit; ++k) s += part[static_cast<int64_t>(k) * l * l + e];
-    A(e / l, e % l) = s;
-    V(e / l, e % l) = (e / l == e % l) ? 1.0 : 0.0;
-  }
+  fold_partials(a.part + b * a.part_bs, a.nsplit, l, Am, ld);
+  for (int e = tid; e < l * l; e += nt) V(e / l, e % l) = (e / l == e % l) ? 1.f : 0.f;
   __syncthreads();
-  // symmetrize (the two triangles are summed in the same order, but be exact)
-  for (int e = tid; e < l * l; e += blockDim.x) {
+  // exact symmetry
+  for (int e = tid; e < l * l; e += nt) {
     const int i = e / l, j = e % l;
-    if (i < j) { const double v = 0.5 * (A(i, j) + A(j, i)); A(i, j) = v; A(j, i) = v; }
+    if (i < j) { const float v = 0.5f * (A(i, j) + A(j, i)); A(i, j) = v; A(j, i) = v; }
   }
   __syncthreads();
-  double diag2 = 0;
+  float frob2;
   {
-    double s = 0;
-    for (int i = tid; i < l; i += blockDim.x) s += A(i, i) * A(i, i);
-    diag2 = block_sum(s, red);
+    float s = 0.f;
+    for (int e = tid; e < l * l; e += nt) s += A(e / l, e % l) * A(e / l, e % l);
+    frob2 = block_sum(s, red);
+  }
+  // this thread's (pair, row) items: e = tid + nt * it, pair = e / l, row = e % l
+  int ik[2], ir[2];
+#pragma unroll
+  for (int it = 0; it < 2; ++it) {
+    const int e = tid + nt * it;
+    ik[it] = (e < npairs * l) ? e / l : -1;
+    ir[it] = (e < npairs * l) ? e % l : 0;
   }
   int sweep = 0;
-  __syncthreads();
+  float off = frob2, prev = frob2;
   for (; sweep < a.max_sweeps; ++sweep) {
     for (int step = 0; step < n - 1; ++step) {
-      // round-robin pairing: position 0 fixed, the others rotate by `step`
-      for (int k = tid; k < n / 2; k += blockDim.x) {
-        const int pa = k, pb = n - 1 - k;
-        const int p = pa == 0 ? 0 : 1 + (pa - 1 + step) % (n - 1);
-        const int q = 1 + (pb - 1 + step) % (n - 1);
+      if (tid < npairs) {
+        // round-robin pairing: position 0 fixed, the others rotate by `step`
+        const int k = tid, pa = k, pb = n - 1 - k;
+        int p = 0;
+        if (pa != 0) { p = pa - 1 + step; if (p >= n - 1) p -= n - 1; p += 1; }
+        int q = pb - 1 + step; if (q >= n - 1) q -= n - 1; q += 1;
         int i = min(p, q), j = max(p, q);
-        double c = 1.0, s = 0.0;
+        float c = 1.f, s = 0.f;
         if (j < l) {
-          const double apq = A(i, j);
-          if (apq != 0.0) {
-            const double th = (A(j, j) - A(i, i)) / (2.0 * apq);
-            const double t = (th >= 0 ? 1.0 : -1.0) / (fabs(th) + sqrt(th * th + 1.0));
-            c = 1.0 / sqrt(t * t + 1.0);
+          const float apq = A(i, j);
+          if (fabsf(apq) > 1e-30f) {
+            const float th = (A(j, j) - A(i, i)) / (2.f * apq);
+            const float t = copysignf(1.f, th) / (fabsf(th) + sqrtf(fmaf(th, th, 1.f)));
+            c = rsqrtf(fmaf(t, t, 1.f));
             s = t * c;
           }
         } else {
@@ -374,46 +513,54 @@ __global__ void __launch_bounds__(256) k_jacobi(const __grid_constant__ EigArgs 
       }
       __syncthreads();
       // columns: A <- A J, V <- V J
-      for (int e = tid; e < (n / 2) * l; e += blockDim.x) {
-        const int k = e / l, r = e % l;
+#pragma unroll
+      for (int it = 0; it < 2; ++it) {
+        if (ik[it] < 0) continue;
+        const int k = ik[it], r = ir[it];
         const int i = pp[k], j = qq[k];
         if (i < 0) continue;
-        const double c = cs[k], s = sn[k];
-        const double ai = A(r, i), aj = A(r, j);
+        const float c = cs[k], s = sn[k];
+        const float ai = A(r, i), aj = A(r, j);
         A(r, i) = c * ai - s * aj;
         A(r, j) = s * ai + c * aj;
-        const double vi = V(r, i), vj = V(r, j);
+        const float vi = V(r, i), vj = V(r, j);
         V(r, i) = c * vi - s * vj;
         V(r, j) = s * vi + c * vj;
       }
       __syncthreads();
       // rows: A <- J^T A
-      for (int e = tid; e < (n / 2) * l; e += blockDim.x) {
-        const int k = e / l, r = e % l;
+#pragma unroll
+      for (int it = 0; it < 2; ++it) {
+        if (ik[it] < 0) continue;
+        const int k = ik[it], r = ir[it];
         const int i = pp[k], j = qq[k];
         if (i < 0) continue;
-        const double c = cs[k], s = sn[k];
-        const double ai = A(i, r), aj = A(j, r);
+        const float c = cs[k], s = sn[k];
+        const float ai = A(i, r), aj = A(j, r);
         A(i, r) = c * ai - s * aj;
         A(j, r) = s * ai + c * aj;
       }
       __syncthreads();
     }
-    double off = 0;
-    for (int e = tid; e < l * l; e += blockDim.x) {
+    float so = 0.f;
+    for (int e = tid; e < l * l; e += nt) {
       const int i = e / l, j = e % l;
-      if (i != j) off += A(i, j) * A(i, j);
+      if (i != j) so += A(i, j) * A(i, j);
     }
-    off = block_sum(off, red);
-    if (off <= 1e-30 * diag2 || off == 0.0) { ++sweep; break; }
+    prev = off;
+    off = block_sum(so, red);
+    // converged, or stalled at the fp32 rounding floor (~ l^2 (u ||A||)^2):
+    // Jacobi converges quadratically, so a sweep that no longer halves the
+    // off-diagonal mass once it is tiny has reached that floor
+    if (off <= 1e-12f * frob2 || (off <= 1e-9f * frob2 && off > 0.5f * prev)) { ++sweep; break; }
   }
-  if (tid == 0 && sweep >= a.max_sweeps) raise_flag(a.flags, kFlagNumeric);
+  if (tid == 0 && sweep >= a.max_sweeps && off > 1e-8f * frob2) raise_flag(a.flags, kFlagNumeric);
   // sort eigenvalues descending, ties by lower index (stable)
-  for (int i = tid; i < l; i += blockDim.x) {
-    const double li = A(i, i);
+  for (int i = tid; i < l; i += nt) {
+    const float li = A(i, i);
     int pos = 0;
     for (int j = 0; j < l; ++j) {
-      const double lj = A(j, j);
+      const float lj = A(j, j);
       if (lj > li || (lj == li && j < i)) ++pos;
     }
     order[pos] = i;
@@ -422,50 +569,51 @@ __global__ void __launch_bounds__(256) k_jacobi(const __grid_constant__ EigArgs 
   const int rr = min(a.rank, l);
   float* ritz = a.ritz + b * a.ritz_bs;
   float* z = a.z + b * a.z_bs;
-  for (int c = tid; c < l; c += blockDim.x) ritz[c] = static_cast<float>(A(order[c], order[c]));
-  for (int e = tid; e < l * l; e += blockDim.x) {
+  for (int c = tid; c < l; c += nt) ritz[c] = A(order[c], order[c]);
+  for (int e = tid; e < l * l; e += nt) {
     const int r = e / l, c = e % l;
-    z[e] = static_cast<float>(V(r, order[c]));
+    z[e] = V(r, order[c]);
   }
   // K = sum_{c in C} (lam_c^{-1/2} - 1) z_c z_c^T
   float* km = a.kmat + b * a.k_bs;
-  for (int e = tid; e < l * l; e += blockDim.x) {
+  for (int e = tid; e < l * l; e += nt) {
     const int r = e / l, s = e % l;
-    double acc = 0;
+    float acc = 0.f;
     for (int c = 0; c < rr; ++c) {
-      const double lam = A(order[c], order[c]);
-      if (!(lam > 1.0)) break;       // descending: the first lam <= 1 ends C
-      acc += (1.0 / sqrt(lam) - 1.0) * V(r, order[c]) * V(s, order[c]);
+      const float lam = A(order[c], order[c]);
+      if (!(lam > 1.f)) break;       // descending: the first lam <= 1 ends C
+      acc = fmaf(rsqrtf(lam) - 1.f, V(r, order[c]) * V(s, order[c]), acc);
     }
-    km[e] = static_cast<float>(acc);
+    km[e] = acc;
   }
   if (tid == 0) {
     int nc = 0;
-    double excess = 0;
+    float excess = 0.f;
     for (int c = 0; c < rr; ++c) {
-      const double lam = A(order[c], order[c]);
-      if (!(lam > 1.0)) break;
+      const float lam = A(order[c], order[c]);
+      if (!(lam > 1.f)) break;
       ++nc;
-      excess += lam - 1.0;
+      excess += lam - 1.f;
     }
-    const double mprime = static_cast<double>(a.count[a.mat_id[b]]);
+    const float mprime = static_cast<float>(a.count[a.mat_id[b]]);
     float* st = a.stats + b * a.stats_bs;
     st[0] = static_cast<float>(a.k_orient);
-    st[1] = static_cast<float>(mprime);
-    st[2] = static_cast<float>(fmax(mprime - excess, 0.0));
+    st[1] = mprime;
+    st[2] = fmaxf(mprime - excess, 0.f);
     st[3] = static_cast<float>(nc);
     st[4] = static_cast<float>(l);
     st[5] = static_cast<float>(a.n_a);
     st[6] = static_cast<float>(a.m_a);
     st[7] = static_cast<float>(sweep);
   }
-}
 #undef A
 #undef V
+}
 
 // ---------------------------------------------------------------------------
 // Fused apply: T = Psi + Lm R^T (Lm [rows x l], R [cols x l]) and
 // W <- (1 - lr wd) W - lr * target * sqrt(mn) / ||T||_F * T
+// 64 x 64 tiles, thread = 4 x 4 block of consecutive rows / columns.
 // ---------------------------------------------------------------------------
 struct LApplyArgs {
   const float* psi; int64_t psi_bs, psi_ld;
@@ -477,10 +625,10 @@ struct LApplyArgs {
   int l;
   float lr, wd, target;
 };
-template <typename TW>
+template <typename TW, bool VEC>
 __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyArgs a) {
-  __shared__ float Ls[kLmax][64 + 4];   // [p][row]
-  __shared__ float Rs[kLmax][64 + 4];   // [p][col]
+  __shared__ __align__(16) float Ls[kLmax][64 + 4];   // [p][row]
+  __shared__ __align__(16) float Rs[kLmax][64 + 4];   // [p][col]
   const int b = blockIdx.z;
   const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
   const int64_t r0 = static_cast<int64_t>(blockIdx.y) * 64, c0 = static_cast<int64_t>(blockIdx.x) * 64;
@@ -495,32 +643,54 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
   __syncthreads();
   float acc[4][4] = {};
   for (int p = 0; p < l; ++p) {
-    float lv[4], rv[4];
-#pragma unroll
-    for (int r = 0; r < 4; ++r) { lv[r] = Ls[p][ty * 4 + r]; rv[r] = Rs[p][tx * 4 + r]; }
+    const float4 lv = *reinterpret_cast<const float4*>(&Ls[p][ty * 4]);
+    const float4 rv = *reinterpret_cast<const float4*>(&Rs[p][tx * 4]);
+    const float la[4] = {lv.x, lv.y, lv.z, lv.w}, ra[4] = {rv.x, rv.y, rv.z, rv.w};
 #pragma unroll
     for (int r = 0; r < 4; ++r)
 #pragma unroll
-      for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(lv[r], rv[c], acc[r][c]);
+      for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(la[r], ra[c], acc[r][c]);
   }
   const float* st = a.stats + b * a.stats_bs;
-  const double nrm2 = st[2];
+  const float nrm2 = st[2];
   const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
-  const float scale = nrm2 > 0 ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
+  const float scale = nrm2 > 0.f ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
   const float cw = 1.f - a.lr * a.wd, ct = -a.lr * scale;
   const float* psi = a.psi + b * a.psi_bs;
   TW* W = static_cast<TW*>(a.W[b]);
+  const int64_t j0 = c0 + tx * 4;
 #pragma unroll
   for (int r = 0; r < 4; ++r) {
     const int64_t i = r0 + ty * 4 + r;
     if (i >= a.rows) continue;
+    if (VEC && j0 + 4 <= a.cols) {
+      const float4 pv = *reinterpret_cast<const float4*>(psi + i * a.psi_ld + j0);
+      const float ps[4] = {pv.x, pv.y, pv.z, pv.w};
+      float w[4];
+      if (std::is_same<TW, float>::value) {
+        const float4 wv = *reinterpret_cast<const float4*>(reinterpret_cast<float*>(W) + i * a.cols + j0);
+        w[0] = wv.x; w[1] = wv.y; w[2] = wv.z; w[3] = wv.w;
+      } else {
+        const uint2 wv = *reinterpret_cast<const uint2*>(reinterpret_cast<bf16*>(W) + i * a.cols + j0);
+        w[0] = bf16lo(wv.x); w[1] = bf16hi(wv.x); w[2] = bf16lo(wv.y); w[3] = bf16hi(wv.y);
+      }
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int64_t j = c0 + tx * 4 + c;
-      if (j >= a.cols) continue;
-      const float t = psi[i * a.psi_ld + j] + acc[r][c];
-      const float w = to_f32(W[i * a.cols + j]);
-      W[i * a.cols + j] = from_f32<TW>(fmaf(cw, w, ct * t));
+      for (int c = 0; c < 4; ++c) w[c] = fmaf(cw, w[c], ct * (ps[c] + acc[r][c]));
+      if (std::is_same<TW, float>::value) {
+        *reinterpret_cast<float4*>(reinterpret_cast<float*>(W) + i * a.cols + j0) = make_float4(w[0], w[1], w[2], w[3]);
+      } else {
+        *reinterpret_cast<uint2*>(reinterpret_cast<bf16*>(W) + i * a.cols + j0) =
+            make_uint2(pack_bf16x2(w[0], w[1]), pack_bf16x2(w[2], w[3]));
+      }
+    } else {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int64_t j = j0 + c;
+        if (j >= a.cols) continue;
+        const float t = psi[i * a.psi_ld + j] + acc[r][c];
+        const float w = to_f32(W[i * a.cols + j]);
+        W[i * a.cols + j] = from_f32<TW>(fmaf(cw, w, ct * t));
+      }
     }
   }
 }
@@ -528,6 +698,43 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
 // ---------------------------------------------------------------------------
 // host orchestration
 // ---------------------------------------------------------------------------
+#define NP_FOR_LP(X) X(8) X(16) X(24) X(32) X(40) X(48) X(56) X(64)
+
+template <bool TRANS>
+static cudaError_t launch_contract(const ContractArgs& c, int batch, int cpt, cudaStream_t s) {
+  const int64_t P = TRANS ? c.cols : c.rows;
+  const dim3 grid(static_cast<unsigned>(cdiv(P, kCtP)), static_cast<unsigned>(batch),
+                  static_cast<unsigned>(c.ksplit));
+  switch (cpt) {
+#define NP_CT(N) case N: k_contract<TRANS, N><<<grid, 256, kCtSmem, s>>>(c); break;
+    NP_CT(1) NP_CT(2) NP_CT(3) NP_CT(4) NP_CT(5) NP_CT(6) NP_CT(7) NP_CT(8)
+#undef NP_CT
+    default:
+      return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+template <bool TRANS>
+static void contract_attrs() {
+#define NP_CT(N) \
+  cudaFuncSetAttribute(k_contract<TRANS, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kCtSmem));
+  NP_CT(1) NP_CT(2) NP_CT(3) NP_CT(4) NP_CT(5) NP_CT(6) NP_CT(7) NP_CT(8)
+#undef NP_CT
+}
+
+static cudaError_t launch_cholqr(const CholQRArgs& c, int batch, int lp, cudaStream_t s) {
+  const dim3 grid(static_cast<unsigned>(cdiv(c.n, 256)), static_cast<unsigned>(batch));
+  switch (lp) {
+#define NP_CQ(N) case N: k_cholqr<N><<<grid, 256, 0, s>>>(c); break;
+    NP_FOR_LP(NP_CQ)
+#undef NP_CQ
+    default:
+      return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
 cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::vector<void*>& allocs) {
   g.ell_rows = static_cast<int>(std::min<int64_t>(g.rows, rank + oversample));
   g.ell_cols = static_cast<int>(std::min<int64_t>(g.cols, rank + oversample));
@@ -546,13 +753,17 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
   float** vbufs[] = {&g.omega, &g.y0, &g.zt, &g.y, &g.q, &g.bt, &g.qk};
   for (float** v : vbufs)
     if ((e = alloc((void**)v, vec))) return e;
-  if ((e = alloc((void**)&g.part, static_cast<size_t>(g.batch) * g.max_part * g.lmax * g.lmax * sizeof(double)))) return e;
-  if ((e = alloc((void**)&g.small, sq * 2 * sizeof(double)))) return e;
+  if ((e = alloc((void**)&g.kpart, vec * kMaxKSplit))) return e;
+  if ((e = alloc((void**)&g.part, static_cast<size_t>(g.batch) * g.max_part * g.lmax * g.lmax * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.kmat, sq * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.ritz, static_cast<size_t>(g.batch) * g.lmax * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.zvec, sq * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.stats, static_cast<size_t>(g.batch) * 8 * sizeof(float)))) return e;
-  return cudaSuccess;
+  contract_attrs<false>();
+  contract_attrs<true>();
+  const int smem = 2 * g.lmax * (g.lmax + 1) * static_cast<int>(sizeof(float));
+  cudaFuncSetAttribute(k_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  return cudaGetLastError();
 }
 
 cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* mat_ids,
@@ -567,6 +778,10 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   const int64_t vbs = big * g.lmax;            // per-matrix stride of the l-wide buffers
   const int64_t psi_bs = g.rows * g.ld;
   const int B = g.batch;
+  const int lp = static_cast<int>(round_up(l, 8));   // register width of the QR solves
+  const int cpt = (l + 7) / 8;                         // columns per thread of the contractions
+  const int64_t sq = static_cast<int64_t>(g.lmax) * g.lmax;
+  const size_t small_smem = 2 * static_cast<size_t>(l) * (l + 1) * sizeof(float);
   cudaError_t e;
 #define NP_CHECK() do { e = cudaGetLastError(); if (e != cudaSuccess) return e; } while (0)
 
@@ -583,94 +798,104 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     NP_CHECK();
     prof->end(kProfOmega, s, 1);
   }
-  // out = Psi_a V  (contract over the active row length n_a) or Psi_a^T U
-  auto contract_a = [&](const float* v, float* out) -> cudaError_t {
+  // out = op(Psi) V; op = Psi contracts over stored columns, Psi^T over stored
+  // rows.  K is split when the tiles alone would leave SMs idle (fixed-order reduce).
+  auto contract = [&](bool trans, const float* v, float* out) -> cudaError_t {
     prof->begin(kProfContract, s);
+    const int64_t P = trans ? g.cols : g.rows, K = trans ? g.rows : g.cols;
+    const int64_t tiles = cdiv(P, kCtP) * B;
+    int ks = 1;
+    const int64_t want = 2 * static_cast<int64_t>(device_sm_count());
+    while (ks < kMaxKSplit && tiles * ks < want && K / (2 * ks) >= 256) ks *= 2;
     ContractArgs c;
     c.psi = g.psi; c.psi_bs = psi_bs; c.psi_ld = g.ld;
-    c.v = v; c.v_bs = vbs; c.out = out; c.out_bs = vbs;
+    c.v = v; c.v_bs = vbs;
     c.rows = g.rows; c.cols = g.cols; c.l = l;
-    if (rows_active) k_contract<false><<<dim3(static_cast<unsigned>(cdiv(g.rows, 64)), B), 256, 0, s>>>(c);
-    else k_contract<true><<<dim3(static_cast<unsigned>(cdiv(g.cols, 64)), B), 256, 0, s>>>(c);
-    prof->end(kProfContract, s, 1);
-    return cudaGetLastError();
+    c.ksplit = ks;
+    c.kchunk = round_up(cdiv(K, ks), kCtK);
+    if (ks == 1) {
+      c.out = out; c.out_bs = vbs;
+    } else {
+      c.out = g.kpart; c.out_bs = vbs * kMaxKSplit;
+    }
+    cudaError_t err = trans ? launch_contract<true>(c, B, cpt, s) : launch_contract<false>(c, B, cpt, s);
+    if (err) return err;
+    int n_l = 1;
+    if (ks > 1) {
+      SplitReduceArgs r;
+      r.part = g.kpart; r.part_bs = vbs * kMaxKSplit;
+      r.out = out; r.out_bs = vbs;
+      r.n = P * l; r.ksplit = ks;
+      k_split_reduce<<<dim3(static_cast<unsigned>(cdiv(r.n, 256)), B), 256, 0, s>>>(r);
+      err = cudaGetLastError();
+      if (err) return err;
+      n_l = 2;
+    }
+    prof->end(kProfContract, s, n_l);
+    return cudaSuccess;
   };
-  auto contract_at = [&](const float* u, float* out) -> cudaError_t {
-    prof->begin(kProfContract, s);
-    ContractArgs c;
-    c.psi = g.psi; c.psi_bs = psi_bs; c.psi_ld = g.ld;
-    c.v = u; c.v_bs = vbs; c.out = out; c.out_bs = vbs;
-    c.rows = g.rows; c.cols = g.cols; c.l = l;
-    if (rows_active) k_contract<true><<<dim3(static_cast<unsigned>(cdiv(g.cols, 64)), B), 256, 0, s>>>(c);
-    else k_contract<false><<<dim3(static_cast<unsigned>(cdiv(g.rows, 64)), B), 256, 0, s>>>(c);
-    prof->end(kProfContract, s, 1);
-    return cudaGetLastError();
-  };
+  const bool ta = !rows_active;     // Psi_a V:   row contract (k = 0) or column contract (k = 1)
+  const bool tb = rows_active;      // Psi_a^T U: the other one
   auto gram = [&](const float* y, int64_t n) -> int {
     GramArgs ga;
     ga.y = y; ga.y_bs = vbs; ga.part = g.part;
-    ga.part_bs = static_cast<int64_t>(g.max_part) * g.lmax * g.lmax;
+    ga.part_bs = static_cast<int64_t>(g.max_part) * sq;
     ga.n = n; ga.l = l;
     ga.nsplit = static_cast<int>(cdiv(n, kGramRows));
     k_gram_part<<<dim3(ga.nsplit, B), 256, 0, s>>>(ga);
     return ga.nsplit;
   };
   // Y0 = Psi_a Omega; p times Y <- Psi_a (Psi_a^T Y)
-  if ((e = contract_a(g.omega, g.y0))) return e;
+  if ((e = contract(ta, g.omega, g.y0))) return e;
   float* ycur = g.y0;
   for (int it = 0; it < p.power_iters; ++it) {
-    if ((e = contract_at(ycur, g.zt))) return e;
-    if ((e = contract_a(g.zt, g.y))) return e;
+    if ((e = contract(tb, ycur, g.zt))) return e;
+    if ((e = contract(ta, g.zt, g.y))) return e;
     ycur = g.y;
   }
-  // Q = qr(Y): three CholeskyQR passes (the first may shift)
+  // Q = qr(Y): three CholeskyQR passes (a pass shifts when its Gram matrix is
+  // numerically singular): y -> q -> zt -> q
   prof->begin(kProfQR, s);
   {
     const float* src = ycur;
     for (int pass = 0; pass < 3; ++pass) {
       const int ns = gram(src, m_a);
       NP_CHECK();
-      CholArgs ca;
-      ca.part = g.part; ca.part_bs = static_cast<int64_t>(g.max_part) * g.lmax * g.lmax; ca.nsplit = ns;
-      ca.work = g.small; ca.work_bs = 2 * static_cast<int64_t>(g.lmax) * g.lmax;
-      ca.rinv = g.kmat; ca.rinv_bs = static_cast<int64_t>(g.lmax) * g.lmax;
-      ca.l = l; ca.allow_shift = 1; ca.flags = flags;
-      k_chol_inv<<<B, 256, 2 * l * (l + 1) * sizeof(double), s>>>(ca);
-      NP_CHECK();
-      float* dst = (pass == 1) ? g.zt : g.q;   // y -> q -> zt -> q
-      RowMulArgs rm;
-      rm.y = src; rm.y_bs = vbs; rm.s = g.kmat; rm.s_bs = static_cast<int64_t>(g.lmax) * g.lmax;
-      rm.out = dst; rm.out_bs = vbs; rm.n = m_a; rm.l = l;
-      k_rowmul<<<dim3(static_cast<unsigned>(cdiv(m_a * l, 256)), B), 256, 0, s>>>(rm);
-      NP_CHECK();
+      float* dst = (pass == 1) ? g.zt : g.q;
+      CholQRArgs cq;
+      cq.part = g.part; cq.part_bs = static_cast<int64_t>(g.max_part) * sq; cq.nsplit = ns;
+      cq.y = src; cq.q = dst; cq.v_bs = vbs;
+      cq.n = m_a; cq.l = l; cq.flags = flags;
+      if ((e = launch_cholqr(cq, B, lp, s))) return e;
       src = dst;
     }
   }
-  prof->end(kProfQR, s, 9);
+  prof->end(kProfQR, s, 6);
   // B^T = Psi_a^T Q  [n_a x l];  Gamma_Q = B B^T
-  if ((e = contract_at(g.q, g.bt))) return e;
+  if ((e = contract(tb, g.q, g.bt))) return e;
   prof->begin(kProfEig, s);
   {
     const int ns = gram(g.bt, n_a);
     NP_CHECK();
     EigArgs ea;
-    ea.part = g.part; ea.part_bs = static_cast<int64_t>(g.max_part) * g.lmax * g.lmax; ea.nsplit = ns;
+    ea.part = g.part; ea.part_bs = static_cast<int64_t>(g.max_part) * sq; ea.nsplit = ns;
     ea.ritz = g.ritz; ea.ritz_bs = g.lmax;
-    ea.z = g.zvec; ea.z_bs = static_cast<int64_t>(g.lmax) * g.lmax;
-    ea.kmat = g.kmat; ea.k_bs = static_cast<int64_t>(g.lmax) * g.lmax;
+    ea.z = g.zvec; ea.z_bs = sq;
+    ea.kmat = g.kmat; ea.k_bs = sq;
     ea.stats = g.stats; ea.stats_bs = 8;
     ea.count = count; ea.mat_id = mat_ids;
     ea.l = l; ea.rank = p.rank; ea.k_orient = p.k;
     ea.m_a = m_a; ea.n_a = n_a;
-    ea.max_sweeps = 40;
+    ea.max_sweeps = 30;
     ea.flags = flags;
-    k_jacobi<<<B, 256, 2 * l * (l + 1) * sizeof(double), s>>>(ea);
+    const int jthreads = static_cast<int>(std::min<int64_t>(1024, round_up(static_cast<int64_t>((l + 1) / 2) * l, 32)));
+    k_jacobi<<<B, std::max(jthreads, 32), small_smem, s>>>(ea);
     NP_CHECK();
   }
   // QK = Q K  [m_a x l]
   {
     RowMulArgs rm;
-    rm.y = g.q; rm.y_bs = vbs; rm.s = g.kmat; rm.s_bs = static_cast<int64_t>(g.lmax) * g.lmax;
+    rm.y = g.q; rm.y_bs = vbs; rm.s = g.kmat; rm.s_bs = sq;
     rm.out = g.qk; rm.out_bs = vbs; rm.n = m_a; rm.l = l;
     k_rowmul<<<dim3(static_cast<unsigned>(cdiv(m_a * l, 256)), B), 256, 0, s>>>(rm);
     NP_CHECK();
@@ -680,6 +905,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   // in launches of at most kMaxBatch matrices (W pointers travel as kernel arguments)
   prof->begin(kProfApplyL, s);
   int n_apply = 0;
+  const bool vec = (g.cols % 4 == 0) && (g.ld % 4 == 0);
   for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
     const int nb = std::min(kMaxBatch, B - c0);
     ++n_apply;
@@ -692,8 +918,13 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     la.rows = g.rows; la.cols = g.cols; la.l = l;
     la.lr = p.lr; la.wd = p.wd; la.target = p.target;
     const dim3 grid(static_cast<unsigned>(cdiv(g.cols, 64)), static_cast<unsigned>(cdiv(g.rows, 64)), nb);
-    if (g.w_dtype == 0) k_apply_l<float><<<grid, 256, 0, s>>>(la);
-    else k_apply_l<bf16><<<grid, 256, 0, s>>>(la);
+    if (g.w_dtype == 0) {
+      if (vec) k_apply_l<float, true><<<grid, 256, 0, s>>>(la);
+      else k_apply_l<float, false><<<grid, 256, 0, s>>>(la);
+    } else {
+      if (vec) k_apply_l<bf16, true><<<grid, 256, 0, s>>>(la);
+      else k_apply_l<bf16, false><<<grid, 256, 0, s>>>(la);
+    }
     NP_CHECK();
   }
   prof->end(kProfApplyL, s, n_apply);
