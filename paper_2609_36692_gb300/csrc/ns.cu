@@ -299,9 +299,28 @@ constexpr int kStageA = kBM * kBK * 2;   // 16 KB
 constexpr int kStageB = 256 * kBK * 2;   // 32 KB (BN <= 256)
 constexpr int kTcThreads = 192;          // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr int kTmemCols = 512;           // two 128 x 256 fp32 accumulators
-constexpr int kMirrorLd = 40;            // row stride (bf16) of the per-warp transpose buffer
-constexpr size_t kMirrorBytes = 4 * 32 * kMirrorLd * 2;
-constexpr size_t kTcSmem = 1024 + kStages * (kStageA + kStageB) + 256 + kMirrorBytes;
+// Per epilogue warp: two 32 x 32 bf16 staging blocks (the chunk as computed
+// and its transpose), 64-byte rows whose 16-byte pieces are XOR-swizzled by
+// (row >> 1) & 3 so that both row-per-lane and 8-rows-per-instruction
+// accesses are free of bank conflicts.
+constexpr size_t kStageBlockBytes = 32 * 32 * 2;
+constexpr size_t kEpiBytes = 4 * 2 * kStageBlockBytes;
+constexpr size_t kTcSmem = 1024 + kStages * (kStageA + kStageB) + 256 + kEpiBytes;
+
+// Staging block accessors: row r (0..31), 16-byte piece p (0..3) of a 32 x 32
+// bf16 block with 64-byte rows; the piece is stored at p ^ ((r >> 1) & 3).
+__device__ __forceinline__ uint32_t stage_off(int r, int p) {
+  return static_cast<uint32_t>(r * 64 + ((p ^ ((r >> 1) & 3)) << 4));
+}
+__device__ __forceinline__ void stage_st(uint8_t* blk, int r, int p, uint4 v) {
+  *reinterpret_cast<uint4*>(blk + stage_off(r, p)) = v;
+}
+__device__ __forceinline__ uint4 stage_ld(const uint8_t* blk, int r, int p) {
+  return *reinterpret_cast<const uint4*>(blk + stage_off(r, p));
+}
+__device__ __forceinline__ void stage_st16(uint8_t* blk, int r, int col, uint16_t v) {
+  *reinterpret_cast<uint16_t*>(blk + stage_off(r, col >> 3) + 2 * (col & 7)) = v;
+}
 
 __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_constant__ GemmArgs args) {
   extern __shared__ uint8_t smem_raw[];
@@ -316,7 +335,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [kStages] last parity + 1
-  uint16_t* mirror = reinterpret_cast<uint16_t*>(sB + kStages * kStageB + 256);
+  uint8_t* epi = sB + kStages * kStageB + 256;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -431,7 +450,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
   } else {
     // ---------------- epilogue: warps 2..5 ----------------
     const int q = warp & 3;                       // TMEM lane quarter of this warp
-    uint16_t* tbuf = mirror + q * 32 * kMirrorLd; // this warp's transpose buffer
+    uint8_t* stg = epi + q * 2 * kStageBlockBytes;   // this warp's chunk, as computed
+    uint8_t* tbuf = stg + kStageBlockBytes;          // and transposed
+    const int crow = lane >> 2, cpiece = lane & 3;   // coalesced access: rows crow + 8 i, piece cpiece
     int it = 0;
     for (int t = blockIdx.x; t < args.total_tiles; t += gridDim.x, ++it) {
       int b, tm, tn;
@@ -442,7 +463,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
       const int64_t row = r0 + lane;
       const int64_t n0 = static_cast<int64_t>(tn) * g.BN;
       bf16* outb = static_cast<bf16*>(g.out) + b * g.out_bs;
-      const bf16* auxp = g.aux ? static_cast<const bf16*>(g.aux) + b * g.aux_bs + row * g.aux_ld + n0 : nullptr;
+      // aux rows are read 8 per instruction: lane -> rows r0 + crow + 8 i, columns n0 + 8 cpiece
+      const bf16* auxp = g.aux ? static_cast<const bf16*>(g.aux) + b * g.aux_bs + (r0 + crow) * g.aux_ld + n0 + 8 * cpiece
+                               : nullptr;
       // 32-column chunk kinds (rows r0.. and columns n0 + c.. are both 32-aligned):
       // 0 = store as is (and mirror when symmetric: strictly above the diagonal),
       // 1 = the diagonal 32 x 32 block, 2 = strictly below (written by mirrors).
@@ -454,12 +477,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
       // the aux operand does not depend on the accumulator: fetch the first two
       // chunks before waiting for it
       uint4 ax[2][4];
+      const int64_t aux8 = 8 * g.aux_ld;
       if (auxp) {
 #pragma unroll
         for (int k = 0; k < 2; ++k)
           if (k * 32 < g.BN && kind(k * 32) != 2)
 #pragma unroll
-            for (int v = 0; v < 4; ++v) ax[k][v] = __ldg(reinterpret_cast<const uint4*>(auxp + k * 32 + 8 * v));
+            for (int i = 0; i < 4; ++i) ax[k][i] = __ldg(reinterpret_cast<const uint4*>(auxp + i * aux8 + k * 32));
       }
       if (!tc::mbar_wait(&tfull[acc], acc_phase, abort_flag)) {
         *abort_flag = 1;
@@ -484,11 +508,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
         if (kd == 2) {
           if (pref)
 #pragma unroll
-            for (int v = 0; v < 4; ++v) axs[v] = __ldg(reinterpret_cast<const uint4*>(auxp + c + 64 + 8 * v));
+            for (int i = 0; i < 4; ++i) axs[i] = __ldg(reinterpret_cast<const uint4*>(auxp + i * aux8 + c + 64));
           return;
         }
         uint32_t r[32];
         tc::tmem_ld32(tbase + c, r);
+        uint4 w[4];
+        if (auxp) {
+          // regroup the aux block from 8-rows-per-instruction to row-per-lane
+#pragma unroll
+          for (int i = 0; i < 4; ++i) stage_st(stg, crow + 8 * i, cpiece, axs[i]);
+          __syncwarp();
+#pragma unroll
+          for (int v = 0; v < 4; ++v) w[v] = stage_ld(stg, lane, v);
+          if (pref)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) axs[i] = __ldg(reinterpret_cast<const uint4*>(auxp + i * aux8 + c + 64));
+        }
         tc::tmem_ld_wait();
         uint32_t pk[16];
 #pragma unroll
@@ -497,7 +533,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
 #pragma unroll
           for (int e = 0; e < 8; ++e) x[e] = cb * __uint_as_float(r[8 * v + e]);
           if (auxp) {
-            const uint32_t w4[4] = {axs[v].x, axs[v].y, axs[v].z, axs[v].w};
+            const uint32_t w4[4] = {w[v].x, w[v].y, w[v].z, w[v].w};
 #pragma unroll
             for (int e = 0; e < 8; ++e)
               x[e] = fmaf(ca, (e & 1) ? bf16hi(w4[e >> 1]) : bf16lo(w4[e >> 1]), x[e]);
@@ -510,22 +546,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
 #pragma unroll
           for (int e = 0; e < 4; ++e) pk[4 * v + e] = pack_bf16x2(x[2 * e], x[2 * e + 1]);
         }
-        if (pref)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) axs[v] = __ldg(reinterpret_cast<const uint4*>(auxp + c + 64 + 8 * v));
-        bf16* orow = outb + row * g.out_ld + n0 + c;
-        if (kd == 0) {
-#pragma unroll
-          for (int v = 0; v < 4; ++v)
-            reinterpret_cast<uint4*>(orow)[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
-        } else {
-          // diagonal block: this row's elements on or above the diagonal
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (e >= lane)
-              reinterpret_cast<uint16_t*>(orow)[e] =
-                  static_cast<uint16_t>((e & 1) ? (pk[e >> 1] >> 16) : (pk[e >> 1] & 0xFFFFu));
-        }
         if (g.sq_part) {
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
@@ -533,23 +553,54 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
             sq += y0 * y0 + y1 * y1;
           }
         }
+        // each lane owns one row of stg: the aux it read there is replaced by
+        // its results without crossing lanes
+#pragma unroll
+        for (int v = 0; v < 4; ++v) stage_st(stg, lane, v, make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]));
         if (g.sym) {
-          // mirror (row, j) -> (j, row) through a 32 x 32 transpose in shared memory
+          // transposed copy: element (lane, e) -> (e, lane)
 #pragma unroll
           for (int e = 0; e < 32; ++e)
-            tbuf[e * kMirrorLd + lane] = static_cast<uint16_t>((e & 1) ? (pk[e >> 1] >> 16) : (pk[e >> 1] & 0xFFFFu));
-          __syncwarp();
-          const uint16_t* src = tbuf + lane * kMirrorLd;            // column j = n0 + c + lane
-          bf16* dst = outb + (n0 + c + lane) * g.out_ld + r0;       // row j, columns r0 .. r0 + 31
-          if (kd == 0) {
-#pragma unroll
-            for (int v = 0; v < 4; ++v)
-              reinterpret_cast<uint4*>(dst)[v] = reinterpret_cast<const uint4*>(src)[v];
-          } else {
-            for (int e = 0; e < lane; ++e) reinterpret_cast<uint16_t*>(dst)[e] = src[e];   // rows above j
-          }
-          __syncwarp();
+            stage_st16(tbuf, e, lane, static_cast<uint16_t>((e & 1) ? (pk[e >> 1] >> 16) : (pk[e >> 1] & 0xFFFFu)));
         }
+        __syncwarp();
+        // rows r0 + crow + 8 i, columns n0 + c + 8 cpiece .. + 7
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int rr = crow + 8 * i;
+          const uint4 v = stage_ld(stg, rr, cpiece);
+          bf16* o = outb + (r0 + rr) * g.out_ld + n0 + c + 8 * cpiece;
+          if (kd == 0) {
+            *reinterpret_cast<uint4*>(o) = v;
+          } else {
+            // diagonal block: elements on or above the diagonal (column >= row)
+            const uint32_t v4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              if (8 * cpiece + e >= rr)
+                reinterpret_cast<uint16_t*>(o)[e] = static_cast<uint16_t>((e & 1) ? (v4[e >> 1] >> 16) : (v4[e >> 1] & 0xFFFFu));
+          }
+        }
+        if (g.sym) {
+          // mirror: row n0 + c + jj of the output receives column jj of the chunk
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int jj = crow + 8 * i;
+            const uint4 v = stage_ld(tbuf, jj, cpiece);
+            bf16* o = outb + (n0 + c + jj) * g.out_ld + r0 + 8 * cpiece;
+            if (kd == 0) {
+              *reinterpret_cast<uint4*>(o) = v;
+            } else {
+              // diagonal block: only the elements strictly below it (row index < jj)
+              const uint32_t v4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+              for (int e = 0; e < 8; ++e)
+                if (8 * cpiece + e < jj)
+                  reinterpret_cast<uint16_t*>(o)[e] = static_cast<uint16_t>((e & 1) ? (v4[e >> 1] >> 16) : (v4[e >> 1] & 0xFFFFu));
+            }
+          }
+        }
+        __syncwarp();   // stg / tbuf are rewritten by the next chunk
       };
       for (int c = 0; c < g.BN; c += 64) {
         chunk(c, ax[0]);
