@@ -182,6 +182,7 @@ class NSPlan {
   std::vector<void*> allocs_;
   void* tc_args_host_ = nullptr;   // prepared kernel arguments (opaque)
   int num_sms_ = 0;
+  int max_pairs_ = 0;           // co-resident two-CTA clusters of the tensor-core GEMM
   int* mat_ids_dev_ = nullptr;
 };
 

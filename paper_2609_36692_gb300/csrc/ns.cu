@@ -177,6 +177,33 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
                    su32(bar))
                : "memory");
 }
+// Like mma_commit, but the arrival lands on the barrier at the same offset in
+// every CTA of the cluster named in `mask`.
+__device__ __forceinline__ void mma_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+                   su32(bar)),
+               "h"(mask)
+               : "memory");
+}
+// TMA load multicast to the CTAs of the cluster named in `mask`: the box lands
+// at offset `dst` of each one's shared memory and completes on the barrier at
+// offset `bar` there.
+__device__ __forceinline__ void tma_load_3d_mc(void* dst, const CUtensorMap* map, uint64_t* bar, int c0, int c1,
+                                               int c2, uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster "
+      "[%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(su32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(su32(bar)), "r"(c0), "r"(c1), "r"(c2), "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
 // 32 TMEM lanes x 32 consecutive 32-bit columns: thread i receives lane (base + i).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* r) {
   asm volatile(
@@ -264,28 +291,35 @@ __host__ __device__ inline int tiles_per_matrix(int tiles_m, int tiles_n, int bn
   return n;
 }
 
-__device__ __forceinline__ int decode_tile(const GemmArgs& a, int t, int& b, int& tm, int& tn) {
+// Work unit t -> (group, matrix b, row tile tm, column tile tn).  With
+// pairs = 1 a unit is two vertically adjacent tiles (2p, tn) and (2p + 1, tn)
+// that share their B operand, one per CTA of a cluster (`sub` = 0 or 1); every
+// group then has an even number of row tiles.
+__device__ __forceinline__ int decode_tile(const GemmArgs& a, int t, int& b, int& tm, int& tn, int pairs = 0,
+                                           int sub = 0) {
   int gi = 0;
   for (; gi < a.n_groups - 1; ++gi) {
     const GemmGroup& g = a.g[gi];
-    if (t < g.tile_begin + g.batch * g.per) break;
+    if (t < ((g.tile_begin + g.batch * g.per) >> pairs)) break;
   }
   const GemmGroup& g = a.g[gi];
-  const int l = t - g.tile_begin;
-  b = l / g.per;
-  int r = l - b * g.per;
+  const int per = g.per >> pairs;
+  const int l = t - (g.tile_begin >> pairs);
+  b = l / per;
+  int r = l - b * per;
   if (!g.sym) {
-    tm = r / g.tiles_n;
-    tn = r - tm * g.tiles_n;
+    const int tmu = r / g.tiles_n;
+    tn = r - tmu * g.tiles_n;
+    tm = (tmu << pairs) + sub;
   } else {
     const int rr = g.BN / 128;
     int c = 0;
     for (;; ++c) {
-      const int cnt = (rr * (c + 1) < g.tiles_m) ? rr * (c + 1) : g.tiles_m;
+      const int cnt = ((rr * (c + 1) < g.tiles_m) ? rr * (c + 1) : g.tiles_m) >> pairs;
       if (r < cnt) break;
       r -= cnt;
     }
-    tm = r;
+    tm = (r << pairs) + sub;
     tn = c;
   }
   return gi;
@@ -322,6 +356,13 @@ __device__ __forceinline__ void stage_st16(uint8_t* blk, int r, int col, uint16_
   *reinterpret_cast<uint16_t*>(blk + stage_off(r, col >> 3) + 2 * (col & 7)) = v;
 }
 
+// MC = false: each CTA computes its own 128 x BN tiles.
+// MC = true: clusters of two CTAs take units of two vertically adjacent tiles
+// with the same B operand; each CTA loads its own A rows and half of B,
+// multicasting that half into both CTAs, so a CTA reads 16 + BN/128 * 16 KB
+// per 64-deep K block from L2 instead of 16 + BN/64 * 16 KB.  A stage is
+// refilled only after the MMAs of both CTAs released it.
+template <bool MC>
 __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_constant__ GemmArgs args) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -338,10 +379,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
   uint8_t* epi = sB + kStages * kStageB + 256;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int sub = MC ? static_cast<int>(tc::cluster_rank()) : 0;
+  const int unit0 = MC ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int nunits = MC ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
+  const int units = MC ? (args.total_tiles >> 1) : args.total_tiles;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       tc::mbar_init(&full[s], 1);
-      tc::mbar_init(&empty[s], 1);
+      tc::mbar_init(&empty[s], MC ? 2 : 1);   // MC: released by the MMAs of both CTAs
       issued[s] = 0;
     }
     for (int a = 0; a < 2; ++a) {
@@ -356,6 +401,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
       tc::prefetch_map(&args.g[gi].mapB);
     }
   }
+  if (MC) tc::cluster_sync();   // both CTAs' barriers exist before any multicast reaches them
   if (warp == 1) {
     tc::tmem_alloc(tmem_slot, kTmemCols);
     tc::tmem_relinquish();
@@ -370,10 +416,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < args.total_tiles && ok; t += gridDim.x) {
+    for (int t = unit0; t < units && ok; t += nunits) {
       int b, tm, tn;
-      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn)];
+      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn, MC, sub)];
       const int m0 = tm * kBM, n0 = tn * g.BN, nk = g.K / kBK;
+      // 64-row boxes of B this CTA fetches (MC: its half, for both CTAs)
+      const int nbox = g.BN / 64, bbox0 = MC ? sub * (nbox >> 1) : 0, bbox1 = MC ? bbox0 + (nbox >> 1) : nbox;
       const uint32_t bytes = static_cast<uint32_t>((kBM + g.BN) * kBK * 2);
       for (int kb = 0; kb < nk; ++kb) {
         ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[stage], phase ^ 1u, abort_flag));
@@ -389,9 +437,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
             if (g.a_mn) tc::tma_load_3d(dA + i * 8192, &g.mapA, &full[stage], m0 + 64 * i, k0, b);
             else        tc::tma_load_3d(dA + i * 8192, &g.mapA, &full[stage], k0, m0 + 64 * i, b);
           }
-          for (int i = 0; i < g.BN / 64; ++i) {
-            if (g.b_mn) tc::tma_load_3d(dB + i * 8192, &g.mapB, &full[stage], n0 + 64 * i, k0, b);
-            else        tc::tma_load_3d(dB + i * 8192, &g.mapB, &full[stage], k0, n0 + 64 * i, b);
+          for (int i = bbox0; i < bbox1; ++i) {
+            const int c0 = g.b_mn ? n0 + 64 * i : k0, c1 = g.b_mn ? k0 : n0 + 64 * i;
+            if (MC) tc::tma_load_3d_mc(dB + i * 8192, &g.mapB, &full[stage], c0, c1, b, 3);
+            else    tc::tma_load_3d(dB + i * 8192, &g.mapB, &full[stage], c0, c1, b);
           }
         }
         __syncwarp();
@@ -404,9 +453,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
     int stage = 0, it = 0;
     uint32_t phase = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < args.total_tiles && ok; t += gridDim.x, ++it) {
+    for (int t = unit0; t < units && ok; t += nunits, ++it) {
       int b, tm, tn;
-      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn)];
+      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn, MC, sub)];
       const int nk = g.K / kBK;
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
@@ -430,7 +479,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
                                        : tc::sdesc(b_addr + kk * 32, 16, 1024);
             tc::mma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
           }
-          tc::mma_commit(&empty[stage]);
+          if (MC) tc::mma_commit_mc(&empty[stage], 3);
+          else tc::mma_commit(&empty[stage]);
         }
         __syncwarp();
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
@@ -454,9 +504,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
     uint8_t* tbuf = stg + kStageBlockBytes;          // and transposed
     const int crow = lane >> 2, cpiece = lane & 3;   // coalesced access: rows crow + 8 i, piece cpiece
     int it = 0;
-    for (int t = blockIdx.x; t < args.total_tiles; t += gridDim.x, ++it) {
+    for (int t = unit0; t < units; t += nunits, ++it) {
       int b, tm, tn;
-      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn)];
+      const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn, MC, sub)];
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       const int64_t r0 = static_cast<int64_t>(tm) * kBM + q * 32;   // first row of this warp
@@ -625,6 +675,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
       if (issued[s]) tc::mbar_wait(&full[s], issued[s] - 1, &never);
   }
   __syncthreads();
+  // MC: neither CTA exits while the other may still multicast into it or
+  // arrive on its barriers
+  if (MC) tc::cluster_sync();
   if (warp == 1) {
     __syncwarp();
     tc::fence_after();
@@ -743,8 +796,23 @@ __global__ void k_scale_from_norm(const T* X, int64_t per, float* inscale, float
 // ---------------------------------------------------------------------------
 struct NSLaunches {
   GemmArgs gram, poly, update;    // per-iteration templates (scale / sq fields patched per run)
+  bool mc[3];                     // phase runs on two-CTA clusters sharing B (every tiles_m even)
   CUtensorMap xmap[kMaxGroups][3];  // tensor maps of the X ping-pong buffers
 };
+
+// Launch configuration of the two-CTA-cluster GEMM.
+static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int grid, cudaStream_t s) {
+  cfg->gridDim = dim3(grid);
+  cfg->blockDim = dim3(kTcThreads);
+  cfg->dynamicSmemBytes = kTcSmem;
+  cfg->stream = s;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg->attrs = attr;
+  cfg->numAttrs = 1;
+}
 
 NSPlan::~NSPlan() { release(); }
 
@@ -787,7 +855,9 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
       g.s_pad = round_up(g.s, 128);
       g.bn_s = (g.s_pad % 256 == 0) ? 256 : 128;
       if (g.tall) {
-        g.big_pad = round_up(g.big, 128);
+        // 256: the update of a tall matrix then has an even number of
+        // 128-row tiles and can run on two-CTA clusters
+        g.big_pad = round_up(g.big, 256);
         g.bn_big = g.bn_s;
       } else {
         g.big_pad = round_up(g.big, 256);
@@ -907,6 +977,10 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
       }
     }
     a.total_tiles = tiles;
+    bool mc = bf16;
+    for (int gi = 0; gi < a.n_groups; ++gi)
+      if (a.g[gi].tiles_m % 2 != 0 || (a.g[gi].BN / 64) % 2 != 0) mc = false;
+    L->mc[ph] = mc;
   }
   if (bf16) {
     for (size_t gi = 0; gi < groups_.size(); ++gi) {
@@ -915,9 +989,22 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
         if (!make_map(&L->xmap[gi][i], gb.X[i], gb.rows_pad, gb.cols_pad, gb.spec.batch, err))
           return cudaErrorInvalidValue;
     }
-    cudaError_t e = cudaFuncSetAttribute(k_ns_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_ns_gemm_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(kTcSmem));
     if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k_ns_gemm_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kTcSmem));
+    if (e != cudaSuccess) return e;
+    // how many two-CTA clusters fit at once (a GPC with an odd number of
+    // usable SMs leaves one of them out); the persistent grid stays within it
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    pair_config(&cfg, attr, 2 * std::max(1, num_sms_ / 2), nullptr);
+    int n = 0;
+    e = cudaOccupancyMaxActiveClusters(&n, k_ns_gemm_tc<true>, &cfg);
+    if (e != cudaSuccess) return e;
+    max_pairs_ = n;
+    if (n < 1) L->mc[0] = L->mc[1] = L->mc[2] = false;
   }
   return cudaSuccess;
 }
@@ -962,8 +1049,16 @@ cudaError_t NSPlan::run(int steps, const float coef[3], cudaStream_t s, int* fla
     for (int p = 0; p < 3; ++p) {
       prof->begin(cls[p], s);
       if (bf16_) {
-        const int grid = std::min(ph[p]->total_tiles, num_sms_);
-        k_ns_gemm_tc<<<grid, kTcThreads, kTcSmem, s>>>(*ph[p]);
+        if (L->mc[p]) {
+          cudaLaunchConfig_t cfg = {};
+          cudaLaunchAttribute attr[1];
+          pair_config(&cfg, attr, 2 * std::min(ph[p]->total_tiles / 2, max_pairs_), s);
+          cudaError_t le = cudaLaunchKernelEx(&cfg, k_ns_gemm_tc<true>, *ph[p]);
+          if (le != cudaSuccess) return le;
+        } else {
+          const int grid = std::min(ph[p]->total_tiles, num_sms_);
+          k_ns_gemm_tc<false><<<grid, kTcThreads, kTcSmem, s>>>(*ph[p]);
+        }
       } else {
         k_ns_gemm_simt<float><<<ph[p]->total_tiles, 256, 0, s>>>(*ph[p]);
       }
