@@ -331,14 +331,15 @@ __device__ __forceinline__ int decode_tile(const GemmArgs& a, int t, int& b, int
 constexpr int kBM = 128, kBK = 64, kStages = 4;
 constexpr int kStageA = kBM * kBK * 2;   // 16 KB
 constexpr int kStageB = 256 * kBK * 2;   // 32 KB (BN <= 256)
-constexpr int kTcThreads = 192;          // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kEpiWarps = 8;             // two per TMEM lane quarter, each with half the columns
+constexpr int kTcThreads = 64 + 32 * kEpiWarps;   // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr int kTmemCols = 512;           // two 128 x 256 fp32 accumulators
 // Per epilogue warp: two 32 x 32 bf16 staging blocks (the chunk as computed
 // and its transpose), 64-byte rows whose 16-byte pieces are XOR-swizzled by
 // (row >> 1) & 3 so that both row-per-lane and 8-rows-per-instruction
 // accesses are free of bank conflicts.
 constexpr size_t kStageBlockBytes = 32 * 32 * 2;
-constexpr size_t kEpiBytes = 4 * 2 * kStageBlockBytes;
+constexpr size_t kEpiBytes = kEpiWarps * 2 * kStageBlockBytes;
 constexpr size_t kTcSmem = 1024 + kStages * (kStageA + kStageB) + 256 + kEpiBytes;
 
 // Staging block accessors: row r (0..31), 16-byte piece p (0..3) of a 32 x 32
@@ -354,6 +355,42 @@ __device__ __forceinline__ uint4 stage_ld(const uint8_t* blk, int r, int p) {
 }
 __device__ __forceinline__ void stage_st16(uint8_t* blk, int r, int col, uint16_t v) {
   *reinterpret_cast<uint16_t*>(blk + stage_off(r, col >> 3) + 2 * (col & 7)) = v;
+}
+
+// Stores the diagonal 32 x 32 block of a symmetric product: from the chunk
+// (stg) the elements on or above the diagonal, from its transpose (tbuf) the
+// ones below it, so the block is exactly symmetric.  Lane -> rows crow + 8 i,
+// columns 8 cpiece .. + 7.  Out of line: it runs for few chunks.
+__device__ __noinline__ void store_diag_block(const uint8_t* stg, const uint8_t* tbuf, bf16* outb, int64_t out_ld,
+                                              int64_t r0, int64_t c0, int crow, int cpiece) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int rr = crow + 8 * i;
+    const uint4 a = stage_ld(stg, rr, cpiece), t = stage_ld(tbuf, rr, cpiece);
+    const uint32_t a4[4] = {a.x, a.y, a.z, a.w}, t4[4] = {t.x, t.y, t.z, t.w};
+    uint32_t o4[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int c = 8 * cpiece + 2 * e;   // columns c, c + 1 of row rr
+      const uint32_t lo = (c >= rr ? a4[e] : t4[e]) & 0xFFFFu;
+      const uint32_t hi = (c + 1 >= rr ? a4[e] : t4[e]) & 0xFFFF0000u;
+      o4[e] = lo | hi;
+    }
+    *reinterpret_cast<uint4*>(outb + (r0 + rr) * out_ld + c0 + 8 * cpiece) = make_uint4(o4[0], o4[1], o4[2], o4[3]);
+  }
+}
+
+// Keeps a per-tile parameter in a register: the group descriptors live in the
+// kernel's parameter space and are indexed at run time, and a plain copy may
+// be re-read from there after every asm statement that clobbers memory.
+__device__ __forceinline__ int pin(int v) { asm volatile("" : "+r"(v)); return v; }
+__device__ __forceinline__ int64_t pin(int64_t v) { asm volatile("" : "+l"(v)); return v; }
+__device__ __forceinline__ float pin(float v) { asm volatile("" : "+f"(v)); return v; }
+template <typename T>
+__device__ __forceinline__ T* pin(T* v) {
+  uint64_t u = reinterpret_cast<uint64_t>(v);
+  asm volatile("" : "+l"(u));
+  return reinterpret_cast<T*>(u);
 }
 
 // MC = false: each CTA computes its own 128 x BN tiles.
@@ -391,7 +428,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(&tfull[a], 1);
-      tc::mbar_init(&tempty[a], 4);
+      tc::mbar_init(&tempty[a], kEpiWarps);
     }
     tc::mbar_init(drain, 1);
     *abort_flag = 0;
@@ -419,10 +456,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
     for (int t = unit0; t < units && ok; t += nunits) {
       int b, tm, tn;
       const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn, MC, sub)];
-      const int m0 = tm * kBM, n0 = tn * g.BN, nk = g.K / kBK;
+      const int BN = pin(g.BN), a_mn = pin(g.a_mn), b_mn = pin(g.b_mn);
+      const CUtensorMap* mapA = pin(&g.mapA);
+      const CUtensorMap* mapB = pin(&g.mapB);
+      const int m0 = tm * kBM, n0 = tn * BN, nk = pin(g.K) / kBK;
       // 64-row boxes of B this CTA fetches (MC: its half, for both CTAs)
-      const int nbox = g.BN / 64, bbox0 = MC ? sub * (nbox >> 1) : 0, bbox1 = MC ? bbox0 + (nbox >> 1) : nbox;
-      const uint32_t bytes = static_cast<uint32_t>((kBM + g.BN) * kBK * 2);
+      const int nbox = BN / 64, bbox0 = MC ? sub * (nbox >> 1) : 0, bbox1 = MC ? bbox0 + (nbox >> 1) : nbox;
+      const uint32_t bytes = static_cast<uint32_t>((kBM + BN) * kBK * 2);
       for (int kb = 0; kb < nk; ++kb) {
         ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[stage], phase ^ 1u, abort_flag));
         if (!ok) break;
@@ -434,13 +474,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
           uint8_t* dB = sB + stage * kStageB;
 #pragma unroll
           for (int i = 0; i < kBM / 64; ++i) {
-            if (g.a_mn) tc::tma_load_3d(dA + i * 8192, &g.mapA, &full[stage], m0 + 64 * i, k0, b);
-            else        tc::tma_load_3d(dA + i * 8192, &g.mapA, &full[stage], k0, m0 + 64 * i, b);
+            const int c0 = a_mn ? m0 + 64 * i : k0, c1 = a_mn ? k0 : m0 + 64 * i;
+            tc::tma_load_3d(dA + i * 8192, mapA, &full[stage], c0, c1, b);
           }
           for (int i = bbox0; i < bbox1; ++i) {
-            const int c0 = g.b_mn ? n0 + 64 * i : k0, c1 = g.b_mn ? k0 : n0 + 64 * i;
-            if (MC) tc::tma_load_3d_mc(dB + i * 8192, &g.mapB, &full[stage], c0, c1, b, 3);
-            else    tc::tma_load_3d(dB + i * 8192, &g.mapB, &full[stage], c0, c1, b);
+            const int c0 = b_mn ? n0 + 64 * i : k0, c1 = b_mn ? k0 : n0 + 64 * i;
+            if (MC) tc::tma_load_3d_mc(dB + i * 8192, mapB, &full[stage], c0, c1, b, 3);
+            else    tc::tma_load_3d(dB + i * 8192, mapB, &full[stage], c0, c1, b);
           }
         }
         __syncwarp();
@@ -456,13 +496,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
     for (int t = unit0; t < units && ok; t += nunits, ++it) {
       int b, tm, tn;
       const GemmGroup& g = args.g[decode_tile(args, t, b, tm, tn, MC, sub)];
-      const int nk = g.K / kBK;
+      const int nk = pin(g.K) / kBK, a_mn = pin(g.a_mn), b_mn = pin(g.b_mn), BN = pin(g.BN);
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       ok = __all_sync(0xffffffffu, tc::mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag));
       if (!ok) break;
       tc::fence_after();
-      const uint32_t idesc = tc::idesc_bf16(kBM, g.BN, g.a_mn, g.b_mn);
+      const uint32_t idesc = tc::idesc_bf16(kBM, BN, a_mn, b_mn);
+      // descriptor steps per 16-deep K slice: K-major +32 B, MN-major +2048 B
+      const uint32_t a_step = a_mn ? 2048u : 32u, b_step = b_mn ? 2048u : 32u;
+      const uint32_t a_lbo = a_mn ? 8192u : 16u, b_lbo = b_mn ? 8192u : 16u;
       const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * 256);
       for (int kb = 0; kb < nk; ++kb) {
         ok = __all_sync(0xffffffffu, tc::mbar_wait(&full[stage], phase, abort_flag));
@@ -473,10 +516,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
           const uint32_t b_addr = tc::su32(sB + stage * kStageB);
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t ad = g.a_mn ? tc::sdesc(a_addr + kk * 2048, 8192, 1024)
-                                       : tc::sdesc(a_addr + kk * 32, 16, 1024);
-            const uint64_t bd = g.b_mn ? tc::sdesc(b_addr + kk * 2048, 8192, 1024)
-                                       : tc::sdesc(b_addr + kk * 32, 16, 1024);
+            const uint64_t ad = tc::sdesc(a_addr + kk * a_step, a_lbo, 1024);
+            const uint64_t bd = tc::sdesc(b_addr + kk * b_step, b_lbo, 1024);
             tc::mma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
           }
           if (MC) tc::mma_commit_mc(&empty[stage], 3);
@@ -499,8 +540,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
     __syncwarp();
   } else {
     // ---------------- epilogue: warps 2..5 ----------------
-    const int q = warp & 3;                       // TMEM lane quarter of this warp
-    uint8_t* stg = epi + q * 2 * kStageBlockBytes;   // this warp's chunk, as computed
+    const int q = warp & 3;                          // TMEM lane quarter this warp may read
+    const int ew = warp - 2;                         // epilogue warp 0 .. kEpiWarps - 1
+    const int half = ew >> 2;                        // which half of the tile's columns
+    uint8_t* stg = epi + ew * 2 * kStageBlockBytes;  // this warp's chunk, as computed
     uint8_t* tbuf = stg + kStageBlockBytes;          // and transposed
     const int crow = lane >> 2, cpiece = lane & 3;   // coalesced access: rows crow + 8 i, piece cpiece
     int it = 0;
@@ -511,30 +554,35 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
       const uint32_t acc_phase = (it >> 1) & 1;
       const int64_t r0 = static_cast<int64_t>(tm) * kBM + q * 32;   // first row of this warp
       const int64_t row = r0 + lane;
-      const int64_t n0 = static_cast<int64_t>(tn) * g.BN;
-      bf16* outb = static_cast<bf16*>(g.out) + b * g.out_bs;
+      const int BN = pin(g.BN), sym = pin(g.sym);
+      const int64_t out_ld = pin(g.out_ld);
+      float* const sq_part = pin(g.sq_part);
+      const int64_t n0 = static_cast<int64_t>(tn) * BN;
+      bf16* outb = pin(static_cast<bf16*>(g.out) + b * g.out_bs);
       // aux rows are read 8 per instruction: lane -> rows r0 + crow + 8 i, columns n0 + 8 cpiece
       const bf16* auxp = g.aux ? static_cast<const bf16*>(g.aux) + b * g.aux_bs + (r0 + crow) * g.aux_ld + n0 + 8 * cpiece
                                : nullptr;
+      auxp = pin(auxp);
       // 32-column chunk kinds (rows r0.. and columns n0 + c.. are both 32-aligned):
       // 0 = store as is (and mirror when symmetric: strictly above the diagonal),
       // 1 = the diagonal 32 x 32 block, 2 = strictly below (written by mirrors).
       auto kind = [&](int c) -> int {
-        if (!g.sym) return 0;
+        if (!sym) return 0;
         const int64_t j0 = n0 + c;
         return r0 < j0 ? 0 : (r0 == j0 ? 1 : 2);
       };
       // the aux operand does not depend on the accumulator: fetch the first two
       // chunks before waiting for it
-      uint4 ax[2][4];
-      const int64_t aux8 = 8 * g.aux_ld;
-      if (auxp) {
+      uint4 ax0[4], ax1[4];   // aux of the next two chunks
+      const int64_t aux8 = pin(8 * g.aux_ld);
+      const int c_lo = half * (BN >> 1), c_hi = c_lo + (BN >> 1);   // this warp's columns
+      auto fetch_aux = [&](int c, uint4 (&dst)[4]) {
+        if (auxp && c < c_hi && kind(c) != 2)
 #pragma unroll
-        for (int k = 0; k < 2; ++k)
-          if (k * 32 < g.BN && kind(k * 32) != 2)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) ax[k][i] = __ldg(reinterpret_cast<const uint4*>(auxp + i * aux8 + k * 32));
-      }
+          for (int i = 0; i < 4; ++i) dst[i] = __ldg(reinterpret_cast<const uint4*>(auxp + i * aux8 + c));
+      };
+      fetch_aux(c_lo, ax0);
+      fetch_aux(c_lo + 32, ax1);
       if (!tc::mbar_wait(&tfull[acc], acc_phase, abort_flag)) {
         *abort_flag = 1;
         raise_flag(args.flags, kFlagTimeout);
@@ -546,34 +594,28 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
         const float v = g.inscale[b];
         s = g.scale_pow == 2 ? v * v : v;
       }
-      const float ca = g.ca * s, cb = g.cb * s, dg = g.diag * s;
+      const float ca = pin(g.ca * s), cb = pin(g.cb * s), dg = pin(g.diag * s);
       const int64_t diag_col = row - n0;   // column of this thread's diagonal element in the tile
       float sq = 0.f;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * 256);
-      // one 32-column chunk; `axs` holds its prefetched aux and receives the
-      // aux of chunk c + 64 (two chunks in flight)
-      auto chunk = [&](const int c, uint4 (&axs)[4]) {
+      // one copy of the chunk code (a small loop body stays in the instruction cache)
+#pragma unroll 1
+      for (int c = c_lo; c < c_hi; c += 32) {
         const int kd = kind(c);
-        const bool pref = auxp && c + 64 < g.BN && kind(c + 64) != 2;
-        if (kd == 2) {
-          if (pref)
+        uint4 w[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) axs[i] = __ldg(reinterpret_cast<const uint4*>(auxp + i * aux8 + c + 64));
-          return;
-        }
+        for (int i = 0; i < 4; ++i) { w[i] = ax0[i]; ax0[i] = ax1[i]; }
+        fetch_aux(c + 64, ax1);
+        if (kd == 2) continue;
         uint32_t r[32];
         tc::tmem_ld32(tbase + c, r);
-        uint4 w[4];
         if (auxp) {
           // regroup the aux block from 8-rows-per-instruction to row-per-lane
 #pragma unroll
-          for (int i = 0; i < 4; ++i) stage_st(stg, crow + 8 * i, cpiece, axs[i]);
+          for (int i = 0; i < 4; ++i) stage_st(stg, crow + 8 * i, cpiece, w[i]);
           __syncwarp();
 #pragma unroll
           for (int v = 0; v < 4; ++v) w[v] = stage_ld(stg, lane, v);
-          if (pref)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) axs[i] = __ldg(reinterpret_cast<const uint4*>(auxp + i * aux8 + c + 64));
         }
         tc::tmem_ld_wait();
         uint32_t pk[16];
@@ -588,7 +630,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
             for (int e = 0; e < 8; ++e)
               x[e] = fmaf(ca, (e & 1) ? bf16hi(w4[e >> 1]) : bf16lo(w4[e >> 1]), x[e]);
           }
-          if (dg != 0.f) {
+          if (kd == 1 && dg != 0.f) {
 #pragma unroll
             for (int e = 0; e < 8; ++e)
               if (diag_col == c + 8 * v + e) x[e] += dg;
@@ -596,7 +638,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
 #pragma unroll
           for (int e = 0; e < 4; ++e) pk[4 * v + e] = pack_bf16x2(x[2 * e], x[2 * e + 1]);
         }
-        if (g.sq_part) {
+        if (sq_part) {
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
             const float y0 = bf16lo(pk[e]), y1 = bf16hi(pk[e]);
@@ -607,62 +649,40 @@ __global__ void __launch_bounds__(kTcThreads, 1) k_ns_gemm_tc(const __grid_const
         // its results without crossing lanes
 #pragma unroll
         for (int v = 0; v < 4; ++v) stage_st(stg, lane, v, make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]));
-        if (g.sym) {
+        if (sym) {
           // transposed copy: element (lane, e) -> (e, lane)
 #pragma unroll
           for (int e = 0; e < 32; ++e)
             stage_st16(tbuf, e, lane, static_cast<uint16_t>((e & 1) ? (pk[e >> 1] >> 16) : (pk[e >> 1] & 0xFFFFu)));
         }
         __syncwarp();
-        // rows r0 + crow + 8 i, columns n0 + c + 8 cpiece .. + 7
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int rr = crow + 8 * i;
-          const uint4 v = stage_ld(stg, rr, cpiece);
-          bf16* o = outb + (r0 + rr) * g.out_ld + n0 + c + 8 * cpiece;
-          if (kd == 0) {
-            *reinterpret_cast<uint4*>(o) = v;
-          } else {
-            // diagonal block: elements on or above the diagonal (column >= row)
-            const uint32_t v4[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-            for (int e = 0; e < 8; ++e)
-              if (8 * cpiece + e >= rr)
-                reinterpret_cast<uint16_t*>(o)[e] = static_cast<uint16_t>((e & 1) ? (v4[e >> 1] >> 16) : (v4[e >> 1] & 0xFFFFu));
-          }
-        }
-        if (g.sym) {
-          // mirror: row n0 + c + jj of the output receives column jj of the chunk
+        if (kd == 1) {
+          store_diag_block(stg, tbuf, outb, out_ld, r0, n0 + c, crow, cpiece);
+        } else {
+          // rows r0 + crow + 8 i, columns n0 + c + 8 cpiece .. + 7
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            const int jj = crow + 8 * i;
-            const uint4 v = stage_ld(tbuf, jj, cpiece);
-            bf16* o = outb + (n0 + c + jj) * g.out_ld + r0 + 8 * cpiece;
-            if (kd == 0) {
-              *reinterpret_cast<uint4*>(o) = v;
-            } else {
-              // diagonal block: only the elements strictly below it (row index < jj)
-              const uint32_t v4[4] = {v.x, v.y, v.z, v.w};
+            const int rr = crow + 8 * i;
+            *reinterpret_cast<uint4*>(outb + (r0 + rr) * out_ld + n0 + c + 8 * cpiece) = stage_ld(stg, rr, cpiece);
+          }
+          if (sym) {
+            // mirror: row n0 + c + jj of the output receives column jj of the chunk
 #pragma unroll
-              for (int e = 0; e < 8; ++e)
-                if (8 * cpiece + e < jj)
-                  reinterpret_cast<uint16_t*>(o)[e] = static_cast<uint16_t>((e & 1) ? (v4[e >> 1] >> 16) : (v4[e >> 1] & 0xFFFFu));
+            for (int i = 0; i < 4; ++i) {
+              const int jj = crow + 8 * i;
+              *reinterpret_cast<uint4*>(outb + (n0 + c + jj) * out_ld + r0 + 8 * cpiece) = stage_ld(tbuf, jj, cpiece);
             }
           }
         }
         __syncwarp();   // stg / tbuf are rewritten by the next chunk
-      };
-      for (int c = 0; c < g.BN; c += 64) {
-        chunk(c, ax[0]);
-        chunk(c + 32, ax[1]);
       }
       tc::fence_before();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&tempty[acc]);
-      if (g.sq_part) {
+      if (sq_part) {
         sq = warp_sum(sq);
         if (lane == 0)
-          g.sq_part[(static_cast<int64_t>(b) * g.tiles_m * g.tiles_n + tm * g.tiles_n + tn) * 4 + q] = sq;
+          sq_part[(static_cast<int64_t>(b) * g.tiles_m * g.tiles_n + tm * g.tiles_n + tn) * kEpiWarps + ew] = sq;
       }
     }
   }
@@ -876,7 +896,7 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
     const int64_t um = g.tall ? g.big_pad : g.s_pad, un = g.tall ? g.s_pad : g.big_pad;
     const int64_t ubn = g.tall ? g.bn_s : g.bn_big;
     const int tiles = static_cast<int>((um / tile_m) * (un / (bf16 ? ubn : 64)));
-    g.n_part = tiles * (bf16 ? 4 : 1);
+    g.n_part = tiles * (bf16 ? kEpiWarps : 1);
     void* p;
     for (int i = 0; i < 3; ++i) {
       cudaError_t e = cudaMalloc(&p, xbytes);
@@ -977,10 +997,10 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
       }
     }
     a.total_tiles = tiles;
-    bool mc = bf16;
+    bool cl = bf16;
     for (int gi = 0; gi < a.n_groups; ++gi)
-      if (a.g[gi].tiles_m % 2 != 0 || (a.g[gi].BN / 64) % 2 != 0) mc = false;
-    L->mc[ph] = mc;
+      if (a.g[gi].tiles_m % 2 != 0 || (a.g[gi].BN / 64) % 2 != 0) cl = false;
+    L->mc[ph] = cl;
   }
   if (bf16) {
     for (size_t gi = 0; gi < groups_.size(); ++gi) {
@@ -989,12 +1009,11 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
         if (!make_map(&L->xmap[gi][i], gb.X[i], gb.rows_pad, gb.cols_pad, gb.spec.batch, err))
           return cudaErrorInvalidValue;
     }
-    cudaError_t e = cudaFuncSetAttribute(k_ns_gemm_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(kTcSmem));
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(k_ns_gemm_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kTcSmem));
-    if (e != cudaSuccess) return e;
+    cudaError_t e = cudaSuccess;
+    for (auto fn : {k_ns_gemm_tc<false>, k_ns_gemm_tc<true>}) {
+      e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kTcSmem));
+      if (e != cudaSuccess) return e;
+    }
     // how many two-CTA clusters fit at once (a GPC with an odd number of
     // usable SMs leaves one of them out); the persistent grid stays within it
     cudaLaunchConfig_t cfg = {};
