@@ -41,7 +41,10 @@ LR = 0.02
 # Traffic of one launch of the dominant kernel class from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum), per workload; None until a
 # capture of the current kernel exists (profiles/ keeps the summaries).
-NCU_TRAFFIC_PER_LAUNCH = {"gpt2_small_G": 209.3e6}   # profiles/ns_gemm_tc_gpt2_small_G.md
+NCU_TRAFFIC_PER_LAUNCH = {
+    "gpt2_small_G": 211.1e6,   # mean of the Gram, poly and update launches of one NS iteration
+    "gpt2_small_L": 108.5e6,   # mean of six k_contract launches (both operand orientations)
+}
 
 
 # ---------------------------------------------------------------------------
@@ -62,6 +65,27 @@ def ns_flops(cfg: S.ParamSetConfig, steps: int) -> float:
     for m in cfg.matrices:
         s, big = min(m.rows, m.cols), max(m.rows, m.cols)
         tot += steps * (4.0 * s * s * big + 2.0 * s ** 3)
+    return tot
+
+
+def ns_executed_flops(cfg: S.ParamSetConfig, steps: int) -> float:
+    """Flops the tensor-core path executes in one step.  Dimensions are padded
+    (the short side s to 128, the long side to 256), the Gram and polynomial
+    products compute only the 128 x BN tiles that reach the diagonal (BN = 256
+    when the padded s is a multiple of 256, else 128) and mirror the rest."""
+    def up(x, m):
+        return (x + m - 1) // m * m
+    tot = 0.0
+    for m in cfg.matrices:
+        s, big = min(m.rows, m.cols), max(m.rows, m.cols)
+        sp, bp = up(s, 128), up(big, 256)
+        bn = 256 if sp % 256 == 0 else 128
+        tiles_m, tiles_n, rr = sp // 128, sp // bn, bn // 128
+        sym_tiles = sum(min(rr * (c + 1), tiles_m) for c in range(tiles_n))
+        gram = 2.0 * sym_tiles * 128 * bn * bp
+        poly = 2.0 * sym_tiles * 128 * bn * sp
+        update = 2.0 * sp * bp * sp
+        tot += steps * (gram + poly + update)
     return tot
 
 
@@ -281,24 +305,37 @@ def run_ours(args, cfg, variant, rank, world):
               for k, v in prof.items() if v[1] > 0}
     if variant == "G":
         fl = ns_flops(cfg, cfg.ns_steps)
+        fl_exec = ns_executed_flops(cfg, cfg.ns_steps)
         ns_ms = sum(prof[k][0] for k in ("ns_gram", "ns_poly", "ns_update")) / args.steps
         ns_launches = sum(prof[k][1] for k in ("ns_gram", "ns_poly", "ns_update")) / args.steps
         achieved = fl / (ns_ms * 1e-3) / 1e12
+        # a step that ran into the power cap is held to the sustained matmul rate
+        capped = "sw_power_cap" in clocks.get("reasons", [])
+        peak = bf16_sust if capped else bf16_burst
         roof = {"bound": "tensor", "kernel": "k_ns_gemm_tc (Newton-Schulz Gram / poly / update)",
-                "achieved": achieved, "peak": bf16_burst, "unit": "TFLOP/s",
-                "frac": achieved / bf16_burst,
-                "peak_source": "%s bf16 burst (kernel timed inside a ms-scale step)" % peak_src,
+                "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak,
+                "peak_source": "%s bf16 %s" % (peak_src, "sustained (sw_power_cap seen in the timed region)"
+                                                if capped else "burst"),
                 "flops_per_launch": fl / ns_launches, "ms_per_launch": ns_ms / ns_launches,
+                "flops_note": "nominal dense flops (full Gram); the kernel computes only the "
+                              "tiles on or above the diagonal of the two symmetric products",
+                "executed_flops_per_launch": fl_exec / ns_launches,
+                "achieved_executed": fl_exec / (ns_ms * 1e-3) / 1e12,
+                "frac_executed": fl_exec / (ns_ms * 1e-3) / 1e12 / peak,
                 "traffic": NCU_TRAFFIC_PER_LAUNCH.get(cfg.name)}
     else:
-        ap_ms = prof["apply_l"][0] / args.steps
         con_ms = prof["contract"][0] / args.steps
-        nbytes = n_el * 4.0
-        achieved = nbytes * (2 + 2 * cfg.power_iters) / (con_ms * 1e-3) / 1e9
+        con_launches = prof["contract"][1] / args.steps
+        # each contraction streams the fp32 Psi of its group once: Y0 = Psi Omega,
+        # Psi^T Y and Psi Z per power iteration, B = Q^T Psi
+        nbytes = n_el * 4.0 * (2 + 2 * cfg.power_iters)
+        achieved = nbytes / (con_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "kernel": "k_contract (sketch streams of Psi)",
                 "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                 "peak_source": "%s HBM copy bandwidth" % peak_src,
-                "bytes_per_launch": nbytes, "traffic": NCU_TRAFFIC_PER_LAUNCH.get(cfg.name)}
+                "bytes_per_launch": nbytes / con_launches, "ms_per_launch": con_ms / con_launches,
+                "traffic": NCU_TRAFFIC_PER_LAUNCH.get(cfg.name)}
     norm_gbs = n_el * b_norm / (norm_ms * 1e-3) / 1e9 if norm_ms > 0 else None
 
     # ---- end to end through the C ABI on pinned host buffers ----
