@@ -23,15 +23,16 @@
 
 namespace normpre {
 
-constexpr int kColRB = 64;        // rows per block in the column passes
+constexpr int kColStatsRB = 256;  // rows per block of pass A (one partial sum per block and column)
+constexpr int kColApplyRB = 64;   // rows per block of pass B
 constexpr int kColThreads = 256;  // 32 column chunks of 8 x 8 row lanes
 
 size_t normalize_cols_part_bytes(int64_t rows, int64_t cols, int n) {
-  return static_cast<size_t>(n) * cdiv(rows, kColRB) * cols * 3 * sizeof(double);
+  return static_cast<size_t>(n) * cdiv(rows, kColStatsRB) * cols * 3 * sizeof(double);
 }
 
 size_t normalize_cols_scratch_bytes(int64_t rows, int64_t cols, int n) {
-  const int64_t nrb = cdiv(rows, kColRB);
+  const int64_t nrb = cdiv(rows, kColStatsRB);
   return static_cast<size_t>(n) * nrb * cols * 3 * sizeof(double) +
          static_cast<size_t>(n) * cols * sizeof(float2) + 256;
 }
@@ -140,8 +141,8 @@ __global__ void __launch_bounds__(kColThreads) k_norm_cols_stats(const __grid_co
   const int b = blockIdx.z, rb = blockIdx.y;
   const int cc = threadIdx.x & 31, rl = threadIdx.x >> 5;
   const int64_t rows = a.rows, cols = a.cols;
-  const int64_t r0 = static_cast<int64_t>(rb) * kColRB;
-  const int64_t r1 = min(r0 + kColRB, rows);
+  const int64_t r0 = static_cast<int64_t>(rb) * kColStatsRB;
+  const int64_t r1 = min(r0 + kColStatsRB, rows);
   const TG* g = static_cast<const TG*>(a.G[b]);
   float* M = a.M[b];
   const TW* w = static_cast<const TW*>(a.W[b]);
@@ -151,6 +152,7 @@ __global__ void __launch_bounds__(kColThreads) k_norm_cols_stats(const __grid_co
   if (VEC) {
     const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 256 + cc * 8;
     if (j0 < cols) {
+#pragma unroll 4
       for (int64_t r = r0 + rl; r < r1; r += 8) {
         float gv[8], mp[8], wv[8];
         load8(g + r * cols + j0, gv);
@@ -243,8 +245,8 @@ __global__ void __launch_bounds__(kColThreads) k_norm_cols_apply(const __grid_co
   const int b = blockIdx.z, rb = blockIdx.y;
   const int cc = threadIdx.x & 31, rl = threadIdx.x >> 5;
   const int64_t rows = a.rows, cols = a.cols;
-  const int64_t r0 = static_cast<int64_t>(rb) * kColRB;
-  const int64_t r1 = min(r0 + kColRB, rows);
+  const int64_t r0 = static_cast<int64_t>(rb) * kColApplyRB;
+  const int64_t r1 = min(r0 + kColApplyRB, rows);
   const float* M = a.M[b];
   const TW* w = static_cast<const TW*>(a.W[b]);
   TP* psi = static_cast<TP*>(a.psi[b]);
@@ -312,9 +314,10 @@ cudaError_t launch_normalize_rows(const NormLaunch& a, cudaStream_t s) {
 cudaError_t launch_normalize_cols(const NormLaunch& a, cudaStream_t s) {
   if (a.n <= 0 || a.rows <= 0 || a.cols <= 0) return cudaSuccess;
   const bool vec = (a.cols % 8 == 0) && (a.psi_ld % 8 == 0);
-  const int nrb = static_cast<int>(cdiv(a.rows, kColRB));
+  const int nrb = static_cast<int>(cdiv(a.rows, kColStatsRB));
   const dim3 grid(static_cast<unsigned>(cdiv(a.cols, 256)), static_cast<unsigned>(nrb),
                   static_cast<unsigned>(a.n));
+  const dim3 grid_b(grid.x, static_cast<unsigned>(cdiv(a.rows, kColApplyRB)), static_cast<unsigned>(a.n));
   return dispatch3(a.g_dtype, a.w_dtype, a.psi_dtype, [&](auto* tg, auto* tw, auto* tp) {
     using TG = std::remove_pointer_t<decltype(tg)>;
     using TW = std::remove_pointer_t<decltype(tw)>;
@@ -326,8 +329,8 @@ cudaError_t launch_normalize_cols(const NormLaunch& a, cudaStream_t s) {
     k_norm_cols_final<<<dim3(grid.x, a.n), 256, 0, s>>>(a, nrb);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    if (vec) k_norm_cols_apply<TW, TP, true><<<grid, kColThreads, 0, s>>>(a);
-    else k_norm_cols_apply<TW, TP, false><<<grid, kColThreads, 0, s>>>(a);
+    if (vec) k_norm_cols_apply<TW, TP, true><<<grid_b, kColThreads, 0, s>>>(a);
+    else k_norm_cols_apply<TW, TP, false><<<grid_b, kColThreads, 0, s>>>(a);
     return cudaGetLastError();
   });
 }

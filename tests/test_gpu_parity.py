@@ -84,12 +84,17 @@ SMALL = S.custom_config("small_mixed", [(128, 384), (128, 128), (128, 512), (512
 RAGGED = S.custom_config("ragged", [(50, 203), (203, 50), (1, 77), (77, 1), (33, 33)],
                          g_dtype="f32", w_dtype="f32", row_sigma=1.0, rank=4, oversample=4)
 SINGLE = S.CONFIGS["single_256x1024"]
+# tall column-active strips: clusters of 4, 8 and 12 CTAs (the last with a
+# partial row block) and one matrix whose column count is not a multiple of 32
+TALL = S.custom_config("tall_cols", [(1000, 40), (4100, 64), (6144, 32), (2056, 24)],
+                       g_dtype="bf16", w_dtype="f32", row_sigma=1.0, col_sigma=1.0,
+                       rank=4, oversample=4)
 
 
 # ---------------------------------------------------------------------------
 # momentum + relaxed tangent + normalization
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED, TALL], ids=lambda c: c.name)
 @pytest.mark.parametrize("t", [0, 1])
 @pytest.mark.parametrize("w_dtype", ["f32", "bf16"])
 def test_normalize_and_momentum(cfgset, t, w_dtype):
