@@ -231,7 +231,7 @@ int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* 
  *   M <- mu M + G;  x_j = m_j - <m_j, w_j> w_j per column j;  Psi = x_j / ||x_j||
  * (zero columns give zero columns of Psi).
  *   rows, cols  stored shape (row-major, contiguous), each in [1, 65536] and
- *               rows * cols at most about 22 million (see the scratch limit).
+ *               rows * cols at most about 87 million (see the scratch limit).
  *   G           device, g_dtype (NORMPRE_F32 or NORMPRE_BF16), read only.
  *   M           device fp32, M_{t-1} on entry, M_t on return.
  *   W           device, w_dtype, read only.

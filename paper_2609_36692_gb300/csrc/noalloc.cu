@@ -63,7 +63,7 @@ extern "C" int normpre_normalize_cols_noalloc(int64_t rows, int64_t cols, float 
     return noalloc_fail(NORMPRE_ERR_SHAPE,
                         "rows x cols needs " + std::to_string(need) + " bytes of scratch; the fixed "
                         "array holds " + std::to_string(kNoAllocScratchBytes) +
-                        " (at most about 22 million elements)");
+                        " (at most about 87 million elements)");
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return noalloc_fail(NORMPRE_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));

@@ -27,7 +27,7 @@ def _lib():
 def test_noalloc_rejects_oversized_and_bad_arguments():
     C = _lib()
     with pytest.raises(C.NormPreError) as e:
-        C.normpre_normalize_cols_noalloc(8192, 8192, 0.95, 16, C.NORMPRE_F32, 16, 16, C.NORMPRE_F32, 16)
+        C.normpre_normalize_cols_noalloc(16384, 16384, 0.95, 16, C.NORMPRE_F32, 16, 16, C.NORMPRE_F32, 16)
     assert e.value.status == C.NORMPRE_ERR_SHAPE
     assert "scratch" in C.normpre_last_error()
     with pytest.raises(C.NormPreError) as e:
