@@ -213,6 +213,10 @@ struct SketchGroup {
   float* stats = nullptr;       // [8] per matrix
   int lmax = 0;
   int max_part = 0;
+  // tensor-core contractions: TMA maps of Psi as the K-major (box 32 x 128)
+  // and MN-major (box 32 x 32) A operand; tc = false keeps the SIMT kernel
+  CUtensorMap psi_map_k, psi_map_mn;
+  bool tc = false;
 };
 
 struct SketchParams {

@@ -27,10 +27,13 @@
 // and exact Ritz pairs of Gamma_Q (Lemma 2 of the paper gives the exact-case
 // version), so W can be written in the same pass that forms T.
 #include <algorithm>
+#include <cstring>
+#include <string>
 #include <type_traits>
 
 #include "common.cuh"
 #include "internal.h"
+#include "tc.cuh"
 
 namespace normpre {
 
@@ -121,10 +124,15 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 // P = rows, K = cols) or Psi^T (TRANS = true, P = cols, K = rows).
 // V is [K x l] row-major (stride l).  With ksplit > 1 every split writes a
 // partial [P x l] block and k_split_reduce folds them in a fixed order.
-// Tile: 128 output rows x 8 CPT columns, K chunks of 32, 256 threads; thread
-// (ty, tx) = (tid / 8, tid % 8) owns rows 4 ty .. 4 ty + 3 and columns
-// CPT tx .. CPT tx + CPT - 1.  Two shared-memory stages filled by cp.async;
-// the inner loop reads four K values at a time with 16-byte loads.
+//
+// At l = 40 a contraction does 80 flops per 4-byte element of Psi, so it is
+// bound by fp32 FMA issue, not HBM; the tiling aims at an FMA-to-shared-load
+// ratio that keeps the FMA pipe busy.  Tile: 256 output rows x l columns,
+// K chunks of 32 in two cp.async stages, 128 threads.  Lane (rq, ct) =
+// (lane / 4, lane % 4) of warp w owns the 8 rows 64 w + rq + 8 i (interleaved,
+// so a quarter warp's 16-byte reads of a K-major Psi tile hit distinct banks)
+// and the CPT = ceil(l / 4) columns CPT ct .. CPT ct + CPT - 1: 8 x CPT
+// accumulators per thread, about 0.9 bytes of shared memory per FMA.
 // ---------------------------------------------------------------------------
 struct ContractArgs {
   const float* psi; int64_t psi_bs, psi_ld;
@@ -135,20 +143,23 @@ struct ContractArgs {
   int ksplit;
   int64_t kchunk;                  // K range of one split (multiple of 32)
 };
-constexpr int kCtP = 128, kCtK = 32;
+constexpr int kCtP = 256, kCtK = 32, kCtThreads = 128;
 constexpr int kCtPsiLd = kCtK + 4;          // non-TRANS: Ps[p][k]
 constexpr int kCtPtLd = kCtP + 4;           // TRANS: Pt[k][p]
-constexpr int kCtVLd = kCtK + 4;            // Vt[c][k]
+constexpr int kCtVLd = kLmax + 4;           // Vs[k][c]
 constexpr int kCtPsiFloats = (kCtP * kCtPsiLd > kCtK * kCtPtLd) ? kCtP * kCtPsiLd : kCtK * kCtPtLd;
-constexpr int kCtStageFloats = kCtPsiFloats + kLmax * kCtVLd;
+constexpr int kCtStageFloats = kCtPsiFloats + kCtK * kCtVLd;
 constexpr size_t kCtSmem = 2 * kCtStageFloats * sizeof(float);
 
 template <bool TRANS, int CPT>
-__global__ void __launch_bounds__(256) k_contract(const __grid_constant__ ContractArgs a) {
+__global__ void __launch_bounds__(kCtThreads) k_contract(const __grid_constant__ ContractArgs a) {
   extern __shared__ float4 ct_smem4[];
   float* smem = reinterpret_cast<float*>(ct_smem4);
   const int b = blockIdx.y, split = blockIdx.z;
-  const int tid = threadIdx.x, ty = tid >> 3, tx = tid & 7;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rq = lane >> 2, ct = lane & 3;
+  const int rbase = 64 * warp + rq;           // rows rbase + 8 i
+  const int cbase = CPT * ct;                 // columns cbase .. cbase + CPT - 1
   const int64_t P = TRANS ? a.cols : a.rows, K = TRANS ? a.rows : a.cols;
   const int64_t p0 = static_cast<int64_t>(blockIdx.x) * kCtP;
   const int64_t kbeg = static_cast<int64_t>(split) * a.kchunk;
@@ -157,42 +168,51 @@ __global__ void __launch_bounds__(256) k_contract(const __grid_constant__ Contra
   const float* v = a.v + b * a.v_bs;
   const int l = a.l;
   const int64_t ld = a.psi_ld;
+  const bool v16 = (l % 4) == 0;
 
   auto load_stage = [&](int st, int64_t k0) {
     float* S = smem + st * kCtStageFloats;
-    float* Vt = S + kCtPsiFloats;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int e = tid + 256 * q;
+    float* Vs = S + kCtPsiFloats;
+#pragma unroll 4
+    for (int q = 0; q < 16; ++q) {
+      const int e = tid + kCtThreads * q;
       if (!TRANS) {
-        const int row = e >> 3, k4 = (e & 7) * 4;      // 128 rows x 8 float4
+        const int row = e >> 3, k4 = (e & 7) * 4;      // 256 rows x 8 float4
         const int64_t gp = p0 + row, gk = k0 + k4;
         const bool ok = gp < P && gk < kend && gk + 4 <= ld;
         cp_async16(S + row * kCtPsiLd + k4, ok ? psi + gp * ld + gk : psi, ok);
       } else {
-        const int k = e >> 5, p4 = (e & 31) * 4;       // 32 rows x 32 float4
+        const int k = e >> 6, p4 = (e & 63) * 4;       // 32 rows x 64 float4
         const int64_t gk = k0 + k, gp = p0 + p4;
         const bool ok = gk < kend && gp + 4 <= ld;
         cp_async16(S + k * kCtPtLd + p4, ok ? psi + gk * ld + gp : psi, ok);
       }
     }
-    // V chunk, transposed: Vt[c][k] = V[k0 + k][c]
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const int e = tid + 256 * q;
-      const int k = e >> 6, c = e & 63;
-      const int64_t gk = k0 + k;
-      const bool ok = c < l && gk < kend;
-      cp_async4(Vt + c * kCtVLd + k, ok ? v + gk * l + c : v, ok);
+    // V chunk as Vs[k][c]: rows of l floats (columns l .. 4 CPT - 1 zero)
+    if (v16) {
+      const int per = CPT;                              // float4 per padded row
+      for (int e = tid; e < kCtK * per; e += kCtThreads) {
+        const int k = e / per, c4 = (e - k * per) * 4;
+        const int64_t gk = k0 + k;
+        const bool ok = c4 < l && gk < kend;
+        cp_async16(Vs + k * kCtVLd + c4, ok ? v + gk * l + c4 : v, ok);
+      }
+    } else {
+      for (int e = tid; e < kCtK * 4 * CPT; e += kCtThreads) {
+        const int k = e / (4 * CPT), c = e - k * (4 * CPT);
+        const int64_t gk = k0 + k;
+        const bool ok = c < l && gk < kend;
+        cp_async4(Vs + k * kCtVLd + c, ok ? v + gk * l + c : v, ok);
+      }
     }
     cp_async_commit();
   };
 
-  float acc[4][CPT];
+  float acc[8][CPT];
 #pragma unroll
-  for (int r = 0; r < 4; ++r)
+  for (int i = 0; i < 8; ++i)
 #pragma unroll
-    for (int c = 0; c < CPT; ++c) acc[r][c] = 0.f;
+    for (int c = 0; c < CPT; ++c) acc[i][c] = 0.f;
 
   int st = 0;
   if (kbeg < kend) load_stage(0, kbeg);
@@ -205,39 +225,38 @@ __global__ void __launch_bounds__(256) k_contract(const __grid_constant__ Contra
     }
     __syncthreads();
     const float* S = smem + st * kCtStageFloats;
-    const float* Vt = S + kCtPsiFloats;
+    const float* Vs = S + kCtPsiFloats + cbase;
+    if (!TRANS) {
+#pragma unroll 2
+      for (int kk = 0; kk < kCtK; kk += 4) {
+        float4 av[8];
 #pragma unroll
-    for (int kk = 0; kk < kCtK; kk += 4) {
-      float4 bv[CPT];
+        for (int i = 0; i < 8; ++i) av[i] = *reinterpret_cast<const float4*>(S + (rbase + 8 * i) * kCtPsiLd + kk);
 #pragma unroll
-      for (int c = 0; c < CPT; ++c) bv[c] = *reinterpret_cast<const float4*>(Vt + (tx * CPT + c) * kCtVLd + kk);
-      if (!TRANS) {
+        for (int k4 = 0; k4 < 4; ++k4) {
+          float bv[CPT];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-          const float4 av = *reinterpret_cast<const float4*>(S + (ty * 4 + r) * kCtPsiLd + kk);
+          for (int c = 0; c < CPT; ++c) bv[c] = Vs[(kk + k4) * kCtVLd + c];
 #pragma unroll
-          for (int c = 0; c < CPT; ++c) {
-            acc[r][c] = fmaf(av.x, bv[c].x, acc[r][c]);
-            acc[r][c] = fmaf(av.y, bv[c].y, acc[r][c]);
-            acc[r][c] = fmaf(av.z, bv[c].z, acc[r][c]);
-            acc[r][c] = fmaf(av.w, bv[c].w, acc[r][c]);
+          for (int i = 0; i < 8; ++i) {
+            const float x = k4 == 0 ? av[i].x : k4 == 1 ? av[i].y : k4 == 2 ? av[i].z : av[i].w;
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) acc[i][c] = fmaf(x, bv[c], acc[i][c]);
           }
         }
-      } else {
-        float4 a4[4];
+      }
+    } else {
+#pragma unroll 4
+      for (int k = 0; k < kCtK; ++k) {
+        float x[8], bv[CPT];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) a4[i] = *reinterpret_cast<const float4*>(S + (kk + i) * kCtPtLd + ty * 4);
+        for (int i = 0; i < 8; ++i) x[i] = S[k * kCtPtLd + rbase + 8 * i];
 #pragma unroll
-        for (int c = 0; c < CPT; ++c) {
-          const float bb[4] = {bv[c].x, bv[c].y, bv[c].z, bv[c].w};
+        for (int c = 0; c < CPT; ++c) bv[c] = Vs[k * kCtVLd + c];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            acc[0][c] = fmaf(a4[i].x, bb[i], acc[0][c]);
-            acc[1][c] = fmaf(a4[i].y, bb[i], acc[1][c]);
-            acc[2][c] = fmaf(a4[i].z, bb[i], acc[2][c]);
-            acc[3][c] = fmaf(a4[i].w, bb[i], acc[3][c]);
-          }
-        }
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+          for (int c = 0; c < CPT; ++c) acc[i][c] = fmaf(x[i], bv[c], acc[i][c]);
       }
     }
     __syncthreads();
@@ -245,14 +264,281 @@ __global__ void __launch_bounds__(256) k_contract(const __grid_constant__ Contra
   }
   float* out = a.out + b * a.out_bs + static_cast<int64_t>(split) * P * l;
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const int64_t gp = p0 + ty * 4 + r;
+  for (int i = 0; i < 8; ++i) {
+    const int64_t gp = p0 + rbase + 8 * i;
     if (gp >= P) continue;
 #pragma unroll
     for (int c = 0; c < CPT; ++c) {
-      const int j = tx * CPT + c;
-      if (j < l) out[gp * l + j] = acc[r][c];
+      const int j = cbase + c;
+      if (j < l) out[gp * l + j] = acc[i][c];
     }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Tensor-core form of the same contraction (tcgen05, kind::tf32) with fp32
+// accuracy from three products per K step: every fp32 operand x is split into
+// hi = x rounded to TF32 and lo = x - hi (exact in fp32) rounded to TF32, and
+// A V = Ahi Vhi + Ahi Vlo + Alo Vhi up to the dropped Alo Vlo term and the
+// rounding of lo: below 2^-21 relative per product (fp32 FMA: 2^-24).
+//
+// The TF32 MMA takes only K-major operands, while V ([K][l]) and, for Psi^T,
+// Psi arrive MN-major, so the split pass also transposes: TMA copies 32-deep
+// K blocks as they lie (Psi K-major: box 32 x 128; Psi^T and V: boxes of
+// 32 K rows x 32 elements), and four warps write hi and lo tiles in the
+// K-major 128-byte-swizzle layout (row r, 16-byte chunk j at r * 128 +
+// ((j ^ (r & 7)) * 16)).  A quarter warp then reads one swizzled row or
+// writes eight consecutive rows of one chunk: no bank conflicts either way.
+//
+// One CTA computes a 128 x l tile of one matrix over one K split: warp 0
+// issues the TMA copies into a 3-stage ring, warps 2-5 split, warp 1 issues
+// the 12 MMAs of a block (M = 128, N = l rounded up to 16, K = 8) into a TMEM
+// accumulator.  The tensor core's fp32 accumulation is biased toward zero by
+// up to an ulp per addition, which over thousands of K steps reaches 1e-4
+// relative; so every kCtcSeg blocks the MMAs switch to the other of two TMEM
+// accumulators and warps 2-5 drain the finished one into fp32 registers with
+// round-to-nearest additions (bias bounded by ~48 additions, ~3e-6).
+// ---------------------------------------------------------------------------
+struct ContractTcArgs {
+  CUtensorMap psi_map;    // {cols, rows, batch} fp32, 128-byte swizzle
+  CUtensorMap v_map;      // {l, K, batch} fp32, box 32 x 32
+  float* out; int64_t out_bs;
+  int64_t P, K;
+  int l, np;              // np = MMA N = l rounded up to 16 (<= 64)
+  int64_t kchunk;         // K range of one split (multiple of 32)
+  int* flags;
+};
+constexpr int kCtcStages = 3;
+constexpr int kCtcSeg = 4;                           // K blocks per accumulator segment
+constexpr int kCtcA = 128 * 32 * 4;                  // one A tile (128 rows x 32 K): 16 KB
+constexpr int kCtcV = 64 * 32 * 4;                   // one V tile (64 rows x 32 K): 8 KB
+constexpr int kCtcStage = 3 * kCtcA + 3 * kCtcV;     // copy, hi, lo of both: 72 KB
+constexpr int kCtcThreads = 192;
+constexpr size_t kCtcSmem = 1024 + kCtcStages * kCtcStage + 256;
+
+__device__ __forceinline__ float tf32_rna(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return __uint_as_float(r);
+}
+__device__ __forceinline__ void split4(const float4 x, float4& h, float4& l) {
+  h.x = tf32_rna(x.x); l.x = tf32_rna(x.x - h.x);
+  h.y = tf32_rna(x.y); l.y = tf32_rna(x.y - h.y);
+  h.z = tf32_rna(x.z); l.z = tf32_rna(x.z - h.z);
+  h.w = tf32_rna(x.w); l.w = tf32_rna(x.w - h.w);
+}
+// byte offset of 16-byte chunk j of row r in a 128-byte-swizzled tile
+__device__ __forceinline__ uint32_t sw128(int r, int j) { return static_cast<uint32_t>(r * 128 + ((j ^ (r & 7)) << 4)); }
+
+// K-major source (rows r0 .. r0 + nr - 1 of 32 K values, already swizzled):
+// elementwise split; warp w of the 4 takes rows w, w + 4, ...
+__device__ __forceinline__ void split_kmajor(const uint8_t* src, uint8_t* hi, uint8_t* lo, int nr, int w, int lane) {
+  for (int i = w * 32 + lane; i < nr * 8; i += 128) {
+    const float4 x = *reinterpret_cast<const float4*>(src + 16 * i);
+    float4 h, l;
+    split4(x, h, l);
+    *reinterpret_cast<float4*>(hi + 16 * i) = h;
+    *reinterpret_cast<float4*>(lo + 16 * i) = l;
+  }
+}
+// MN-major source box (32 K rows x 32 elements, swizzled, rows = K) ->
+// K-major rows r0 + c (c = lane) of the hi / lo tiles.
+__device__ __forceinline__ void split_transpose(const uint8_t* box, uint8_t* hi, uint8_t* lo, int r0, int lane) {
+  const int c = lane, r = r0 + c;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {            // K chunk j = K rows 4 j .. 4 j + 3
+    float4 x;
+    x.x = *reinterpret_cast<const float*>(box + sw128(4 * j + 0, c >> 2) + 4 * (c & 3));
+    x.y = *reinterpret_cast<const float*>(box + sw128(4 * j + 1, c >> 2) + 4 * (c & 3));
+    x.z = *reinterpret_cast<const float*>(box + sw128(4 * j + 2, c >> 2) + 4 * (c & 3));
+    x.w = *reinterpret_cast<const float*>(box + sw128(4 * j + 3, c >> 2) + 4 * (c & 3));
+    float4 h, l;
+    split4(x, h, l);
+    *reinterpret_cast<float4*>(hi + sw128(r, j)) = h;
+    *reinterpret_cast<float4*>(lo + sw128(r, j)) = l;
+  }
+}
+
+template <bool TRANS>
+__global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_constant__ ContractTcArgs a) {
+  extern __shared__ uint8_t ctc_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(ctc_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kCtcStages * kCtcStage);
+  uint64_t* splitb = full + kCtcStages;
+  uint64_t* empty = splitb + kCtcStages;
+  uint64_t* tfull = empty + kCtcStages;    // [2]
+  uint64_t* tempty = tfull + 2;            // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [kCtcStages] last parity + 1
+  // stage layout: A copy | A hi | A lo | V copy | V hi | V lo
+  auto a_copy = [&](int st) { return smem + st * kCtcStage; };
+  auto v_copy = [&](int st) { return smem + st * kCtcStage + 3 * kCtcA; };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.y;
+  const int64_t p0 = static_cast<int64_t>(blockIdx.x) * 128;
+  const int64_t kbeg = static_cast<int64_t>(blockIdx.z) * a.kchunk;
+  const int64_t kend = min(a.K, kbeg + a.kchunk);
+  const int nk = kend > kbeg ? static_cast<int>((kend - kbeg + 31) / 32) : 0;
+  const int nvb = a.np > 32 ? 2 : 1;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kCtcStages; ++s) {
+      tc::mbar_init(&full[s], 1);
+      tc::mbar_init(&splitb[s], 4);
+      tc::mbar_init(&empty[s], 1);
+      issued[s] = 0;
+    }
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&tfull[i], 1);
+      tc::mbar_init(&tempty[i], 4);
+    }
+    *abort_flag = 0;
+    tc::fence_barrier_init();
+    tc::prefetch_map(&a.psi_map);
+    tc::prefetch_map(&a.v_map);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(tmem_slot, 128);        // two accumulators of 64 columns
+    tc::tmem_relinquish();
+    tc::fence_before();
+  }
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int nseg = (nk + kCtcSeg - 1) / kCtcSeg;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    bool ok = true;
+    for (int kb = 0; kb < nk && ok; ++kb) {
+      const int st = kb % kCtcStages;
+      const uint32_t ph = (kb / kCtcStages) & 1;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[st], ph ^ 1u, abort_flag));
+      if (!ok) break;
+      if (lane == 0) {
+        tc::mbar_expect_tx(&full[st], static_cast<uint32_t>(kCtcA + nvb * 4096));
+        issued[st] = ph + 1;
+        const int k0 = static_cast<int>(kbeg) + 32 * kb, pr = static_cast<int>(p0);
+        if (!TRANS) {
+          tc::tma_load_3d(a_copy(st), &a.psi_map, &full[st], k0, pr, b);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) tc::tma_load_3d(a_copy(st) + j * 4096, &a.psi_map, &full[st], pr + 32 * j, k0, b);
+        }
+        for (int j = 0; j < nvb; ++j) tc::tma_load_3d(v_copy(st) + j * 4096, &a.v_map, &full[st], 32 * j, k0, b);
+      }
+      __syncwarp();
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    const uint32_t idesc = tc::idesc_tf32(128, a.np, 0, 0);
+    bool ok = true;
+    for (int kb = 0; kb < nk && ok; ++kb) {
+      const int st = kb % kCtcStages;
+      const uint32_t ph = (kb / kCtcStages) & 1;
+      const int seg = kb / kCtcSeg, acc = seg & 1;
+      const bool seg_first = (kb % kCtcSeg) == 0;
+      const bool seg_last = (kb % kCtcSeg) == kCtcSeg - 1 || kb == nk - 1;
+      if (seg_first) {
+        // the accumulator's previous segment has been drained
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&tempty[acc], ((seg >> 1) & 1) ^ 1u, abort_flag));
+        if (!ok) break;
+        tc::fence_after();
+      }
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&splitb[st], ph, abort_flag));
+      if (!ok) break;
+      tc::fence_after();
+      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(64 * acc);
+      if (lane == 0) {
+        const uint32_t ahi = tc::su32(a_copy(st) + kCtcA), alo = ahi + kCtcA;
+        const uint32_t vhi = tc::su32(v_copy(st) + kCtcV), vlo = vhi + kCtcV;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {       // K step of 8 fp32 = 32 bytes of a K-major row
+          const uint64_t dah = tc::sdesc(ahi + kk * 32, 16, 1024);
+          const uint64_t dal = tc::sdesc(alo + kk * 32, 16, 1024);
+          const uint64_t dvh = tc::sdesc(vhi + kk * 32, 16, 1024);
+          const uint64_t dvl = tc::sdesc(vlo + kk * 32, 16, 1024);
+          tc::mma_tf32(d_tmem, dah, dvh, idesc, (!seg_first || kk != 0) ? 1u : 0u);
+          tc::mma_tf32(d_tmem, dah, dvl, idesc, 1u);
+          tc::mma_tf32(d_tmem, dal, dvh, idesc, 1u);
+        }
+        tc::mma_commit(&empty[st]);
+        if (seg_last) tc::mma_commit(&tfull[acc]);
+      }
+      __syncwarp();
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
+  } else {
+    // ---------------- split, segment drains, epilogue (warps 2..5) ----------------
+    const int w = warp - 2;
+    const int q = warp & 3;
+    float sum[64];
+#pragma unroll
+    for (int j = 0; j < 64; ++j) sum[j] = 0.f;
+    // adds the accumulator of segment `seg` into sum (round to nearest) and
+    // hands the accumulator back to the MMA warp
+    auto drain = [&](int seg) -> bool {
+      const int acc = seg & 1;
+      if (!__all_sync(0xffffffffu, tc::mbar_wait(&tfull[acc], (seg >> 1) & 1, abort_flag))) return false;
+      tc::fence_after();
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (32 * h < a.np) {
+          uint32_t r[32];
+          tc::tmem_ld32(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(64 * acc + 32 * h), r);
+          tc::tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; ++j) sum[32 * h + j] += __uint_as_float(r[j]);
+        }
+      }
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+      return true;
+    };
+    bool ok = true;
+    for (int kb = 0; kb < nk && ok; ++kb) {
+      const int st = kb % kCtcStages;
+      const uint32_t ph = (kb / kCtcStages) & 1;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&full[st], ph, abort_flag));
+      if (!ok) break;
+      uint8_t* ac = a_copy(st);
+      uint8_t* vc = v_copy(st);
+      if (!TRANS) split_kmajor(ac, ac + kCtcA, ac + 2 * kCtcA, 128, w, lane);
+      else split_transpose(ac + w * 4096, ac + kCtcA, ac + 2 * kCtcA, 32 * w, lane);
+      if (w < nvb) split_transpose(vc + w * 4096, vc + kCtcV, vc + 2 * kCtcV, 32 * w, lane);
+      // the MMAs read these tiles through the async proxy
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&splitb[st]);
+      // the previous segment ends with the block before this one: drain it
+      // while the MMAs of this segment start
+      if (kb % kCtcSeg == 0 && kb > 0) ok = drain(kb / kCtcSeg - 1);
+    }
+    if (ok && nseg > 0) ok = drain(nseg - 1);
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
+    const int64_t row = p0 + 32 * q + lane;
+    float* out = a.out + b * a.out_bs + static_cast<int64_t>(blockIdx.z) * a.P * a.l;
+    if (row < a.P) {
+#pragma unroll
+      for (int j = 0; j < 64; ++j)
+        if (j < a.l) out[row * a.l + j] = ok ? sum[j] : 0.f;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag) {
+    // let every TMA copy still in flight land before the CTA exits
+    volatile int never = 0;
+    for (int s = 0; s < kCtcStages; ++s)
+      if (issued[s]) tc::mbar_wait(&full[s], issued[s] - 1, &never);
+  }
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::fence_after();
+    tc::tmem_dealloc(tmem_base, 128);
   }
 }
 
@@ -706,8 +992,9 @@ static cudaError_t launch_contract(const ContractArgs& c, int batch, int cpt, cu
   const dim3 grid(static_cast<unsigned>(cdiv(P, kCtP)), static_cast<unsigned>(batch),
                   static_cast<unsigned>(c.ksplit));
   switch (cpt) {
-#define NP_CT(N) case N: k_contract<TRANS, N><<<grid, 256, kCtSmem, s>>>(c); break;
+#define NP_CT(N) case N: k_contract<TRANS, N><<<grid, kCtThreads, kCtSmem, s>>>(c); break;
     NP_CT(1) NP_CT(2) NP_CT(3) NP_CT(4) NP_CT(5) NP_CT(6) NP_CT(7) NP_CT(8)
+    NP_CT(9) NP_CT(10) NP_CT(11) NP_CT(12) NP_CT(13) NP_CT(14) NP_CT(15) NP_CT(16)
 #undef NP_CT
     default:
       return cudaErrorInvalidValue;
@@ -720,6 +1007,7 @@ static void contract_attrs() {
 #define NP_CT(N) \
   cudaFuncSetAttribute(k_contract<TRANS, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kCtSmem));
   NP_CT(1) NP_CT(2) NP_CT(3) NP_CT(4) NP_CT(5) NP_CT(6) NP_CT(7) NP_CT(8)
+  NP_CT(9) NP_CT(10) NP_CT(11) NP_CT(12) NP_CT(13) NP_CT(14) NP_CT(15) NP_CT(16)
 #undef NP_CT
 }
 
@@ -761,6 +1049,21 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
   if ((e = alloc((void**)&g.stats, static_cast<size_t>(g.batch) * 8 * sizeof(float)))) return e;
   contract_attrs<false>();
   contract_attrs<true>();
+  // tensor-core contractions: Psi as a 3-D tensor {cols, rows, batch}; the
+  // l-wide operands need 16-byte rows and matrix strides (checked per launch)
+  {
+    const uint64_t dims[3] = {static_cast<uint64_t>(g.cols), static_cast<uint64_t>(g.rows),
+                              static_cast<uint64_t>(g.batch)};
+    const uint64_t strides[2] = {static_cast<uint64_t>(g.ld) * 4, static_cast<uint64_t>(g.rows * g.ld) * 4};
+    const uint32_t box_k[3] = {32, 128, 1}, box_mn[3] = {32, 32, 1};
+    g.tc = (g.ld % 4 == 0) && g.lmax <= 64 &&
+           driver_encode_tiled(&g.psi_map_k, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, g.psi, dims, strides, box_k, nullptr) &&
+           driver_encode_tiled(&g.psi_map_mn, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, g.psi, dims, strides, box_mn, nullptr);
+    if (g.tc) {
+      cudaFuncSetAttribute(k_contract_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kCtcSmem));
+      cudaFuncSetAttribute(k_contract_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kCtcSmem));
+    }
+  }
   const int smem = 2 * g.lmax * (g.lmax + 1) * static_cast<int>(sizeof(float));
   cudaFuncSetAttribute(k_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   return cudaGetLastError();
@@ -779,7 +1082,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   const int64_t psi_bs = g.rows * g.ld;
   const int B = g.batch;
   const int lp = static_cast<int>(round_up(l, 8));   // register width of the QR solves
-  const int cpt = (l + 7) / 8;                         // columns per thread of the contractions
+  const int cpt = (l + 3) / 4;                         // columns per thread of the contractions
   const int64_t sq = static_cast<int64_t>(g.lmax) * g.lmax;
   const size_t small_smem = 2 * static_cast<size_t>(l) * (l + 1) * sizeof(float);
   cudaError_t e;
@@ -800,12 +1103,15 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   }
   // out = op(Psi) V; op = Psi contracts over stored columns, Psi^T over stored
   // rows.  K is split when the tiles alone would leave SMs idle (fixed-order reduce).
+  // the tensor-core form needs 16-byte rows of the l-wide operand and 16-byte
+  // aligned per-matrix strides (TMA)
+  const bool use_tc = g.tc && (l % 4 == 0) && (vbs % 4 == 0) && l <= 64;
   auto contract = [&](bool trans, const float* v, float* out) -> cudaError_t {
     prof->begin(kProfContract, s);
     const int64_t P = trans ? g.cols : g.rows, K = trans ? g.rows : g.cols;
-    const int64_t tiles = cdiv(P, kCtP) * B;
+    const int64_t tiles = cdiv(P, use_tc ? 128 : kCtP) * B;
     int ks = 1;
-    const int64_t want = 2 * static_cast<int64_t>(device_sm_count());
+    const int64_t want = (use_tc ? 1 : 2) * static_cast<int64_t>(device_sm_count());
     while (ks < kMaxKSplit && tiles * ks < want && K / (2 * ks) >= 256) ks *= 2;
     ContractArgs c;
     c.psi = g.psi; c.psi_bs = psi_bs; c.psi_ld = g.ld;
@@ -818,7 +1124,29 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     } else {
       c.out = g.kpart; c.out_bs = vbs * kMaxKSplit;
     }
-    cudaError_t err = trans ? launch_contract<true>(c, B, cpt, s) : launch_contract<false>(c, B, cpt, s);
+    cudaError_t err;
+    if (use_tc) {
+      ContractTcArgs ct;
+      std::memset(static_cast<void*>(&ct), 0, sizeof(ct));
+      ct.psi_map = trans ? g.psi_map_mn : g.psi_map_k;
+      const uint64_t vdims[3] = {static_cast<uint64_t>(l), static_cast<uint64_t>(K), static_cast<uint64_t>(B)};
+      const uint64_t vstr[2] = {static_cast<uint64_t>(l) * 4, static_cast<uint64_t>(vbs) * 4};
+      const uint32_t vbox[3] = {32, 32, 1};
+      std::string why;
+      if (!driver_encode_tiled(&ct.v_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(v), vdims, vstr,
+                               vbox, &why))
+        return cudaErrorInvalidValue;
+      ct.out = c.out; ct.out_bs = c.out_bs;
+      ct.P = P; ct.K = K; ct.l = l; ct.np = static_cast<int>(round_up(l, 16));
+      ct.kchunk = c.kchunk;
+      ct.flags = flags;
+      const dim3 grid(static_cast<unsigned>(cdiv(P, 128)), static_cast<unsigned>(B), static_cast<unsigned>(ks));
+      if (trans) k_contract_tc<true><<<grid, kCtcThreads, kCtcSmem, s>>>(ct);
+      else k_contract_tc<false><<<grid, kCtcThreads, kCtcSmem, s>>>(ct);
+      err = cudaGetLastError();
+    } else {
+      err = trans ? launch_contract<true>(c, B, cpt, s) : launch_contract<false>(c, B, cpt, s);
+    }
     if (err) return err;
     int n_l = 1;
     if (ks > 1) {
