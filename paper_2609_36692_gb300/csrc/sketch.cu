@@ -291,13 +291,14 @@ __global__ void __launch_bounds__(kCtThreads) k_contract(const __grid_constant__
 // writes eight consecutive rows of one chunk: no bank conflicts either way.
 //
 // One CTA computes a 128 x l tile of one matrix over one K split: warp 0
-// issues the TMA copies into a 3-stage ring, warps 2-5 split, warp 1 issues
+// issues the TMA copies into a 3-stage ring, warps 2-9 split, warp 1 issues
 // the 12 MMAs of a block (M = 128, N = l rounded up to 16, K = 8) into a TMEM
 // accumulator.  The tensor core's fp32 accumulation is biased toward zero by
 // up to an ulp per addition, which over thousands of K steps reaches 1e-4
 // relative; so every kCtcSeg blocks the MMAs switch to the other of two TMEM
 // accumulators and warps 2-5 drain the finished one into fp32 registers with
-// round-to-nearest additions (bias bounded by ~48 additions, ~3e-6).
+// round-to-nearest additions (bias bounded by ~48 additions, ~3e-6); warps
+// 2-5 (one per TMEM lane quarter) drain and write the result.
 // ---------------------------------------------------------------------------
 struct ContractTcArgs {
   CUtensorMap psi_map;    // {cols, rows, batch} fp32, 128-byte swizzle
@@ -313,13 +314,16 @@ constexpr int kCtcSeg = 4;                           // K blocks per accumulator
 constexpr int kCtcA = 128 * 32 * 4;                  // one A tile (128 rows x 32 K): 16 KB
 constexpr int kCtcV = 64 * 32 * 4;                   // one V tile (64 rows x 32 K): 8 KB
 constexpr int kCtcStage = 3 * kCtcA + 3 * kCtcV;     // copy, hi, lo of both: 72 KB
-constexpr int kCtcThreads = 192;
+constexpr int kCtcSplitWarps = 8;
+constexpr int kCtcThreads = 64 + 32 * kCtcSplitWarps;
 constexpr size_t kCtcSmem = 1024 + kCtcStages * kCtcStage + 256;
 
+// x rounded to the nearest TF32 value (ties away from zero), as an fp32 bit
+// pattern with the low 13 mantissa bits clear: adding half of the dropped
+// range to the magnitude bits carries into the kept ones exactly when the
+// dropped part is at least half an ulp of TF32.
 __device__ __forceinline__ float tf32_rna(float x) {
-  uint32_t r;
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-  return __uint_as_float(r);
+  return __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
 }
 __device__ __forceinline__ void split4(const float4 x, float4& h, float4& l) {
   h.x = tf32_rna(x.x); l.x = tf32_rna(x.x - h.x);
@@ -330,10 +334,10 @@ __device__ __forceinline__ void split4(const float4 x, float4& h, float4& l) {
 // byte offset of 16-byte chunk j of row r in a 128-byte-swizzled tile
 __device__ __forceinline__ uint32_t sw128(int r, int j) { return static_cast<uint32_t>(r * 128 + ((j ^ (r & 7)) << 4)); }
 
-// K-major source (rows r0 .. r0 + nr - 1 of 32 K values, already swizzled):
-// elementwise split; warp w of the 4 takes rows w, w + 4, ...
+// K-major source (nr rows of 32 K values, already swizzled): elementwise
+// split; the split warps take consecutive 16-byte chunks.
 __device__ __forceinline__ void split_kmajor(const uint8_t* src, uint8_t* hi, uint8_t* lo, int nr, int w, int lane) {
-  for (int i = w * 32 + lane; i < nr * 8; i += 128) {
+  for (int i = w * 32 + lane; i < nr * 8; i += 32 * kCtcSplitWarps) {
     const float4 x = *reinterpret_cast<const float4*>(src + 16 * i);
     float4 h, l;
     split4(x, h, l);
@@ -342,11 +346,13 @@ __device__ __forceinline__ void split_kmajor(const uint8_t* src, uint8_t* hi, ui
   }
 }
 // MN-major source box (32 K rows x 32 elements, swizzled, rows = K) ->
-// K-major rows r0 + c (c = lane) of the hi / lo tiles.
-__device__ __forceinline__ void split_transpose(const uint8_t* box, uint8_t* hi, uint8_t* lo, int r0, int lane) {
+// K-major rows r0 + c (c = lane) of the hi / lo tiles, K chunks j0 .. j0 + NJ - 1.
+template <int NJ>
+__device__ __forceinline__ void split_transpose(const uint8_t* box, uint8_t* hi, uint8_t* lo, int r0, int lane, int j0) {
   const int c = lane, r = r0 + c;
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {            // K chunk j = K rows 4 j .. 4 j + 3
+  for (int jj = 0; jj < NJ; ++jj) {        // K chunk j = K rows 4 j .. 4 j + 3
+    const int j = j0 + jj;
     float4 x;
     x.x = *reinterpret_cast<const float*>(box + sw128(4 * j + 0, c >> 2) + 4 * (c & 3));
     x.y = *reinterpret_cast<const float*>(box + sw128(4 * j + 1, c >> 2) + 4 * (c & 3));
@@ -385,7 +391,7 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
   if (threadIdx.x == 0) {
     for (int s = 0; s < kCtcStages; ++s) {
       tc::mbar_init(&full[s], 1);
-      tc::mbar_init(&splitb[s], 4);
+      tc::mbar_init(&splitb[s], kCtcSplitWarps);
       tc::mbar_init(&empty[s], 1);
       issued[s] = 0;
     }
@@ -471,8 +477,9 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
     }
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
   } else {
-    // ---------------- split, segment drains, epilogue (warps 2..5) ----------------
+    // ---------------- split (warps 2..9), segment drains and epilogue (warps 2..5) ----------------
     const int w = warp - 2;
+    const bool drainer = w < 4;
     const int q = warp & 3;
     float sum[64];
 #pragma unroll
@@ -506,22 +513,25 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
       if (!ok) break;
       uint8_t* ac = a_copy(st);
       uint8_t* vc = v_copy(st);
+      // A: K-major chunks, or box w / 2, chunk half w % 2; V: box w / 4,
+      // chunk pair w % 4 (two boxes) or box 0, chunk w (one box)
       if (!TRANS) split_kmajor(ac, ac + kCtcA, ac + 2 * kCtcA, 128, w, lane);
-      else split_transpose(ac + w * 4096, ac + kCtcA, ac + 2 * kCtcA, 32 * w, lane);
-      if (w < nvb) split_transpose(vc + w * 4096, vc + kCtcV, vc + 2 * kCtcV, 32 * w, lane);
+      else split_transpose<4>(ac + (w >> 1) * 4096, ac + kCtcA, ac + 2 * kCtcA, 32 * (w >> 1), lane, 4 * (w & 1));
+      if (nvb == 2) split_transpose<2>(vc + (w >> 2) * 4096, vc + kCtcV, vc + 2 * kCtcV, 32 * (w >> 2), lane, 2 * (w & 3));
+      else split_transpose<1>(vc, vc + kCtcV, vc + 2 * kCtcV, 0, lane, w);
       // the MMAs read these tiles through the async proxy
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&splitb[st]);
       // the previous segment ends with the block before this one: drain it
       // while the MMAs of this segment start
-      if (kb % kCtcSeg == 0 && kb > 0) ok = drain(kb / kCtcSeg - 1);
+      if (drainer && kb % kCtcSeg == 0 && kb > 0) ok = drain(kb / kCtcSeg - 1);
     }
-    if (ok && nseg > 0) ok = drain(nseg - 1);
+    if (drainer && ok && nseg > 0) ok = drain(nseg - 1);
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
     const int64_t row = p0 + 32 * q + lane;
     float* out = a.out + b * a.out_bs + static_cast<int64_t>(blockIdx.z) * a.P * a.l;
-    if (row < a.P) {
+    if (drainer && row < a.P) {
 #pragma unroll
       for (int j = 0; j < 64; ++j)
         if (j < a.l) out[row * a.l + j] = ok ? sum[j] : 0.f;
