@@ -43,7 +43,7 @@ LR = 0.02
 # capture of the current kernel exists (profiles/ keeps the summaries).
 NCU_TRAFFIC_PER_LAUNCH = {
     "gpt2_small_G": 211.1e6,   # mean of the Gram, poly and update launches of one NS iteration
-    "gpt2_small_L": 108.5e6,   # mean of six k_contract launches (both operand orientations)
+    "gpt2_small_L": 108.1e6,   # mean of six k_contract_tc launches (both operand orientations)
 }
 
 
@@ -331,7 +331,7 @@ def run_ours(args, cfg, variant, rank, world):
         # Psi^T Y and Psi Z per power iteration, B = Q^T Psi
         nbytes = n_el * 4.0 * (2 + 2 * cfg.power_iters)
         achieved = nbytes / (con_ms * 1e-3) / 1e9
-        roof = {"bound": "hbm", "kernel": "k_contract (sketch streams of Psi)",
+        roof = {"bound": "hbm", "kernel": "k_contract_tc (sketch contractions of Psi, tcgen05 TF32 split)",
                 "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                 "peak_source": "%s HBM copy bandwidth" % peak_src,
                 "bytes_per_launch": nbytes / con_launches, "ms_per_launch": con_ms / con_launches,
