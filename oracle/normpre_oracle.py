@@ -42,6 +42,11 @@ Readings taken where the paper is silent:
   fp64); normals by Box-Muller on word pairs (0,1), (2,3).
 * Top-r selection: Ritz values sorted in descending order with a stable sort
   (ties keep the lower index), r' = min(r, l), then C = {i <= r' : lam_i > 1}.
+* Muon baseline (the comparison optimizer of Sec. 4 and App. A): the same
+  momentum, the Newton-Schulz iteration applied to the momentum itself (no
+  orientation, tangent or normalization step, Sec. 2.1), and the update
+  RMS matched to the same target as NormPre (the Muon convention the paper
+  follows in Sec. 3.1).
 """
 from __future__ import annotations
 
@@ -315,9 +320,23 @@ def normpre_step(W: np.ndarray, G: np.ndarray, M_prev: np.ndarray, t: int, lr: f
     return out
 
 
+def muon_step(W: np.ndarray, G: np.ndarray, M_prev: np.ndarray, lr: float,
+              cfg: OracleConfig) -> Dict[str, np.ndarray]:
+    """One step of the Muon baseline for one matrix: M = mu M_prev + G; the
+    update orthogonalizes M itself by the Newton-Schulz iteration (Sec. 2.1:
+    Muon replaces the momentum by its nearest semi-orthogonal matrix); the
+    update RMS is matched to the target (Sec. 3.1); decoupled weight decay as
+    in Algorithm 1."""
+    W = np.asarray(W, dtype=np.float64)
+    M = momentum_update(M_prev, G, cfg.momentum)
+    T = newton_schulz(M, cfg.ns_steps, cfg.ns_coef, cfg.ns_eps)
+    R = rms_matched(T, 0, cfg.target_rms)
+    return {"M": M, "T": T, "R": R, "W": weight_update(W, R, lr, cfg.weight_decay)}
+
+
 __all__ = [
     "MUON_QUINTIC", "OracleConfig", "philox4x32_10", "philox_uniform", "sketch_omega",
     "momentum_update", "orientation_of", "orient", "relaxed_tangent", "diag_gram_normalize",
     "newton_schulz", "ns_scalar_map", "interaction_sketch", "exact_interaction_eigs",
-    "localized_apply", "rms_matched", "weight_update", "normpre_step",
+    "localized_apply", "rms_matched", "weight_update", "normpre_step", "muon_step",
 ]

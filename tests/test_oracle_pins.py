@@ -421,3 +421,43 @@ def test_full_step_shapes_and_rms():
             dW = (W - out["W"]) / 0.1 - 0.1 * W
             assert dW.shape == W.shape
             assert abs(np.sqrt((dW * dW).mean()) - 0.2) < 1e-12
+
+
+# ---------------------------------------------------------------------------
+# Muon baseline (the comparison optimizer of Sec. 4): momentum, Newton-Schulz
+# on the momentum itself, RMS-matched update
+# ---------------------------------------------------------------------------
+def test_muon_reduces_to_normpre_g_on_unit_rows_and_zero_weight():
+    # With W = 0 the relaxed tangent is the momentum itself, and when the
+    # momentum already has unit rows the diagonal-Gram normalization is the
+    # identity, so at a row-active step NormPre-G and Muon coincide.
+    rng = _rng(30)
+    G = rng.standard_normal((12, 40))
+    G /= np.linalg.norm(G, axis=1, keepdims=True)
+    W = np.zeros((12, 40))
+    cfg = O.OracleConfig(variant="G")
+    mu_out = O.muon_step(W, G, np.zeros_like(G), 0.05, cfg)
+    np_out = O.normpre_step(W, G, np.zeros_like(G), 0, 0.05, cfg)
+    np.testing.assert_allclose(mu_out["T"], np_out["T"], rtol=0, atol=1e-13)
+    np.testing.assert_allclose(mu_out["W"], np_out["W"], rtol=0, atol=1e-15)
+
+
+def test_muon_singular_values_follow_the_quintic_map():
+    # T = U p^5(Sigma / ||M||_F) V^T for the momentum's own SVD (no
+    # normalization in between), and the update RMS is the target.
+    rng = _rng(31)
+    G = rng.standard_normal((10, 30)) * np.exp(rng.standard_normal((10, 1)))
+    Mp = rng.standard_normal((10, 30))
+    cfg = O.OracleConfig(variant="G", momentum=0.9)
+    out = O.muon_step(np.zeros((10, 30)), G, Mp, 0.1, cfg)
+    M = 0.9 * Mp + G
+    U, s, Vt = np.linalg.svd(M, full_matrices=False)
+    x = s / (np.linalg.norm(M) + 1e-7)
+    for _ in range(5):
+        x = A_COEF * x + B_COEF * x ** 3 + C_COEF * x ** 5
+    np.testing.assert_allclose(out["T"], (U * x) @ Vt, rtol=0, atol=1e-12)
+    R = out["R"]
+    assert abs(np.sqrt((R * R).mean()) - 0.2) < 1e-15
+    # a tall momentum gives the transpose of its transpose's result
+    out_t = O.muon_step(np.zeros((30, 10)), G.T, Mp.T, 0.1, cfg)
+    np.testing.assert_allclose(out_t["T"], out["T"].T, rtol=0, atol=1e-13)
