@@ -46,7 +46,11 @@ typedef struct normpre_handle normpre_handle;
 /* Variant of the spectral preconditioner (Algorithm 1). */
 enum normpre_variant {
   NORMPRE_G = 0,   /* global: T = msign(Psi) by Newton-Schulz (Sec. 3.2) */
-  NORMPRE_L = 1    /* localized: randomized interaction sketch (Alg. 2) */
+  NORMPRE_L = 1,   /* localized: randomized interaction sketch (Alg. 2) */
+  NORMPRE_MUON = 2 /* not NormPre: the paper's comparison optimizer Muon (Sec. 2.1, Sec. 4),
+                      i.e. Newton-Schulz applied to the momentum itself, with no orientation,
+                      tangent or normalization step, and the same RMS-matched update; it
+                      shares the Newton-Schulz kernels and serves the latency comparison */
 };
 
 /* Storage dtypes of caller tensors. */

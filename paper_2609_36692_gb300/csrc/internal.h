@@ -106,6 +106,14 @@ struct NormLaunch {
   float2* col_coef = nullptr;
 };
 cudaError_t launch_normalize_rows(const NormLaunch& a, cudaStream_t s);
+// Muon baseline (muon.cu): M = mu M + G written back and copied to a.psi,
+// fp64 sums of ||M||^2 of nblk row blocks into part[i * stride + blk] for the
+// launch's matrix i; then the prescale 1 / (||M||_F + eps) of `batch` matrices
+// whose partials start stride apart.
+cudaError_t launch_momentum_copy(const NormLaunch& a, double* part, int nblk, int stride, cudaStream_t s);
+cudaError_t launch_muon_prescale(const double* part, int nblk, int stride, int batch, float* inscale, float eps,
+                                 cudaStream_t s);
+constexpr int kMuonBlocks = 64;   // row blocks per matrix of the Muon momentum pass
 cudaError_t launch_normalize_cols(const NormLaunch& a, cudaStream_t s);
 size_t normalize_cols_scratch_bytes(int64_t rows, int64_t cols, int n);
 size_t normalize_cols_part_bytes(int64_t rows, int64_t cols, int n);   // col_part share of it

@@ -52,7 +52,8 @@ struct normpre_handle {
   float* stats = nullptr;      // [n_mats][8] (NormPre-G)
   double* col_part = nullptr;  // column-active scratch
   float2* col_coef = nullptr;
-  std::unique_ptr<NSPlan> ns;  // NormPre-G
+  double* muon_part = nullptr; // Muon: ||M||^2 partials, [group slot][kMuonBlocks] per group
+  std::unique_ptr<NSPlan> ns;  // NormPre-G and Muon
   int last_k = -1;
   bool stepped = false;
   // host-buffer entry point staging
@@ -79,13 +80,15 @@ size_t dsize(int dt) { return dt == NORMPRE_BF16 ? 2 : 4; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 int check_config(const normpre_config* c, std::string* msg) {
-  if (c->variant != NORMPRE_G && c->variant != NORMPRE_L) { *msg = "variant must be NORMPRE_G or NORMPRE_L"; return NORMPRE_ERR_ARG; }
+  if (c->variant != NORMPRE_G && c->variant != NORMPRE_L && c->variant != NORMPRE_MUON) {
+    *msg = "variant must be NORMPRE_G, NORMPRE_L or NORMPRE_MUON"; return NORMPRE_ERR_ARG;
+  }
   if (!std::isfinite(c->momentum) || !std::isfinite(c->weight_decay) || !std::isfinite(c->target_rms)) {
     *msg = "momentum, weight_decay and target_rms must be finite"; return NORMPRE_ERR_ARG;
   }
   if (c->precision != NORMPRE_PREC_BF16 && c->precision != NORMPRE_PREC_F32) { *msg = "bad precision"; return NORMPRE_ERR_ARG; }
   if (c->orientation < 0 || c->orientation > 2) { *msg = "orientation must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
-  if (c->variant == NORMPRE_G) {
+  if (c->variant != NORMPRE_L) {
     if (c->ns_steps < 1 || c->ns_steps > 100) { *msg = "ns_steps must be in [1, 100]"; return NORMPRE_ERR_ARG; }
     if (!std::isfinite(c->ns_coef[0]) || !std::isfinite(c->ns_coef[1]) || !std::isfinite(c->ns_coef[2]) ||
         !(c->ns_eps >= 0.f)) { *msg = "bad Newton-Schulz coefficients or eps"; return NORMPRE_ERR_ARG; }
@@ -194,8 +197,9 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
     h->mats[i] = MatInfo{rows[i], cols[i], w_dtype[i], g_dtype[i], gi, static_cast<int>(h->groups[gi].mats.size())};
     h->groups[gi].mats.push_back(i);
   }
-  if (cfg->variant == NORMPRE_G && h->groups.size() > static_cast<size_t>(kMaxGroups))
-    return fail(nullptr, NORMPRE_ERR_SHAPE, "NormPre-G supports at most " + std::to_string(kMaxGroups) + " distinct (shape, dtype) groups per handle");
+  if (cfg->variant != NORMPRE_L && h->groups.size() > static_cast<size_t>(kMaxGroups))
+    return fail(nullptr, NORMPRE_ERR_SHAPE, "the Newton-Schulz variants support at most " + std::to_string(kMaxGroups) +
+                " distinct (shape, dtype) groups per handle");
   normpre_handle* hp = h.get();
   if ((e = dalloc(hp, &h->count, sizeof(int) * n_mats))) return cuda_fail(nullptr, e, "cudaMalloc");
   if ((e = dalloc(hp, &h->flags, sizeof(int) * 4))) return cuda_fail(nullptr, e, "cudaMalloc");
@@ -214,7 +218,10 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
     for (Group& g : h->groups) maxc = std::max<int64_t>(maxc, g.cols * std::min<int>(kMaxBatch, static_cast<int>(g.mats.size())));
     if ((e = dalloc(hp, &h->col_coef, sizeof(float2) * maxc))) return cuda_fail(nullptr, e, "cudaMalloc");
   }
-  if (cfg->variant == NORMPRE_G) {
+  if (cfg->variant == NORMPRE_MUON &&
+      (e = dalloc(hp, &h->muon_part, sizeof(double) * kMuonBlocks * n_mats)))
+    return cuda_fail(nullptr, e, "cudaMalloc");
+  if (cfg->variant != NORMPRE_L) {
     std::vector<NSGroupSpec> specs;
     for (Group& g : h->groups) specs.push_back(NSGroupSpec{static_cast<int>(g.mats.size()), g.rows, g.cols});
     h->ns.reset(new NSPlan());
@@ -262,13 +269,42 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
   const int k = orientation_of(c, t);
   cudaError_t e = cudaMemsetAsync(h->count, 0, sizeof(int) * h->n_mats, s);
   if (e) return cuda_fail(h, e, "cudaMemsetAsync");
-  const bool is_g = (c.variant == NORMPRE_G);
+  const bool is_muon = (c.variant == NORMPRE_MUON);
+  const bool is_g = (c.variant == NORMPRE_G) || is_muon;   // Newton-Schulz preconditioning
   const bool psi_bf16 = is_g && c.precision == NORMPRE_PREC_BF16;
 
-  // (1) momentum + relaxed tangent + diagonal-Gram normalization
+  // (1) momentum + relaxed tangent + diagonal-Gram normalization (Muon: the
+  //     momentum alone, copied to the Newton-Schulz input with ||M||^2 sums)
   h->prof.begin(kProfNormalize, s);
   int n_norm = 0;
-  for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+  int64_t mslot = 0;   // first Muon partial slot of the group
+  for (size_t gi = 0; gi < h->groups.size() && is_muon; ++gi) {
+    Group& g = h->groups[gi];
+    NSGroupBuf& nb = h->ns->groups()[gi];
+    const int B = static_cast<int>(g.mats.size());
+    const int64_t psi_bs = nb.rows_pad * nb.cols_pad * static_cast<int64_t>(nb.elem);
+    for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
+      NormLaunch a;
+      a.n = std::min(kMaxBatch, B - c0);
+      a.rows = g.rows; a.cols = g.cols;
+      a.g_dtype = g.g_dtype; a.w_dtype = g.w_dtype; a.psi_dtype = psi_bf16 ? 1 : 0;
+      for (int i = 0; i < a.n; ++i) {
+        const int mid = g.mats[c0 + i];
+        a.G[i] = G[mid]; a.M[i] = static_cast<float*>(M[mid]); a.W[i] = W[mid];
+        a.psi[i] = static_cast<char*>(nb.X[0]) + static_cast<int64_t>(c0 + i) * psi_bs;
+        a.mat_id[i] = mid;
+      }
+      a.psi_ld = nb.cols_pad;
+      a.mu = c.momentum;
+      a.flags = h->flags;
+      const int nblk = static_cast<int>(std::min<int64_t>(kMuonBlocks, g.rows));
+      e = launch_momentum_copy(a, h->muon_part + (mslot + c0) * kMuonBlocks, nblk, kMuonBlocks, s);
+      if (e) return cuda_fail(h, e, "momentum launch");
+      ++n_norm;
+    }
+    mslot += B;
+  }
+  for (size_t gi = 0; gi < h->groups.size() && !is_muon; ++gi) {
     Group& g = h->groups[gi];
     const int B = static_cast<int>(g.mats.size());
     char* psi_base;
@@ -309,10 +345,25 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
 
   if (is_g) {
     // (2) Newton-Schulz on every group, prescaled by 1/(sqrt(m') + eps)
-    std::vector<const int*> ids;
-    for (Group& g : h->groups) ids.push_back(g.mat_ids_dev);
-    e = h->ns->scale_from_count(h->count, ids.data(), c.ns_eps, s, &h->prof);
-    if (e) return cuda_fail(h, e, "prescale launch");
+    //     (NormPre-G: ||Psi||_F^2 = m'), or by 1/(||M||_F + eps) (Muon)
+    if (is_muon) {
+      h->prof.begin(kProfPrescale, s);
+      int64_t slot = 0;
+      for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+        Group& g = h->groups[gi];
+        const int nblk = static_cast<int>(std::min<int64_t>(kMuonBlocks, g.rows));
+        e = launch_muon_prescale(h->muon_part + slot * kMuonBlocks, nblk, kMuonBlocks, static_cast<int>(g.mats.size()),
+                                 h->ns->groups()[gi].inscale, c.ns_eps, s);
+        if (e) return cuda_fail(h, e, "prescale launch");
+        slot += static_cast<int64_t>(g.mats.size());
+      }
+      h->prof.end(kProfPrescale, s, static_cast<int>(h->groups.size()));
+    } else {
+      std::vector<const int*> ids;
+      for (Group& g : h->groups) ids.push_back(g.mat_ids_dev);
+      e = h->ns->scale_from_count(h->count, ids.data(), c.ns_eps, s, &h->prof);
+      if (e) return cuda_fail(h, e, "prescale launch");
+    }
     e = h->ns->run(c.ns_steps, c.ns_coef, s, h->flags, &h->prof);
     if (e) return cuda_fail(h, e, "Newton-Schulz launch");
     // (3) RMS-matched update with weight decay
@@ -461,7 +512,7 @@ int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* row
   if (mat < 0 || mat >= h->n_mats) return fail(hh, NORMPRE_ERR_ARG, "bad matrix index");
   if (!h->stepped) return fail(hh, NORMPRE_ERR_ARG, "no step has run yet");
   const MatInfo& m = h->mats[mat];
-  const bool is_g = h->cfg.variant == NORMPRE_G;
+  const bool is_g = h->cfg.variant != NORMPRE_L;
   const bool rows_active = h->last_k == 0;
   const int64_t m_a = rows_active ? m.rows : m.cols, n_a = rows_active ? m.cols : m.rows;
   int64_t r = 0, c = 0;
@@ -512,7 +563,7 @@ int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capaci
   if (e) return cuda_fail(h, e, "cudaDeviceSynchronize");
   const MatInfo& m = h->mats[mat];
   const Group& g = h->groups[m.group];
-  const bool is_g = h->cfg.variant == NORMPRE_G;
+  const bool is_g = h->cfg.variant != NORMPRE_L;
   const void* src = nullptr;
   int64_t src_ld = c;
   if (what == NORMPRE_BUF_PSI || what == NORMPRE_BUF_T) {

@@ -15,7 +15,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libnormpre.so")
 
 # enums (mirror include/normpre.h)
-NORMPRE_G, NORMPRE_L = 0, 1
+NORMPRE_G, NORMPRE_L, NORMPRE_MUON = 0, 1, 2
 NORMPRE_F32, NORMPRE_BF16 = 0, 1
 NORMPRE_PREC_BF16, NORMPRE_PREC_F32 = 0, 1
 (NORMPRE_OK, NORMPRE_ERR_ARG, NORMPRE_ERR_SHAPE, NORMPRE_ERR_DTYPE, NORMPRE_ERR_ALIGN,

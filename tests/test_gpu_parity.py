@@ -49,7 +49,7 @@ def _run(cfgset: S.ParamSetConfig, t: int, variant: str, precision: int, indices
     else:
         mats = S.make_param_set(cfgset, workers=min(16, os.cpu_count() or 1))
     W, G, M = to_device(mats, cfgset.g_dtype, cfgset.w_dtype)
-    kw = dict(variant=C.NORMPRE_G if variant == "G" else C.NORMPRE_L, precision=precision,
+    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON}[variant], precision=precision,
               rank=cfgset.rank, oversample=cfgset.oversample, power_iters=cfgset.power_iters,
               seed=1234)
     kw.update(extra or {})
@@ -240,6 +240,43 @@ def test_l_large_sets_sampled(name, indices):
     import dataclasses
     cs = dataclasses.replace(S.CONFIGS[name], rank=32, oversample=8)
     _check_l(cs, 0, indices=indices)
+
+
+# ---------------------------------------------------------------------------
+# Muon baseline (the paper's comparison optimizer) on the same kernels
+# ---------------------------------------------------------------------------
+def _check_muon(cs, t, precision, tol, indices=None):
+    from paper_2609_36692_gb300 import normpre as C
+    opt, mats, W1, M1 = _run(cs, t, "muon", precision)
+    idx = range(cs.n_mats) if indices is None else indices
+    for i in idx:
+        m = mats[i]
+        ref = O.muon_step(m["W"], m["G"], m["M"], f32(LR), oracle_config("G"))
+        dm = np.abs(M1[i].astype(np.float64) - ref["M"])
+        assert np.all(dm <= 2.5e-7 * np.abs(ref["M"]) + 1e-30), (cs.name, i, dm.max())
+        T = opt.read(i, C.NORMPRE_BUF_T)
+        assert rel_fro(T, ref["T"]) <= tol, (cs.name, i, rel_fro(T, ref["T"]))
+        dW = W1[i].astype(np.float64) - m["W"]
+        dW_ref = ref["W"] - m["W"]
+        if cs.w_dtype == "f32":
+            assert rel_fro(dW, dW_ref) <= tol, (cs.name, i)
+        else:
+            half_ulp = 0.5 * bf16_ulp(ref["W"])
+            err = np.linalg.norm(W1[i].astype(np.float64) - ref["W"])
+            assert err <= tol * np.linalg.norm(dW_ref) + np.linalg.norm(half_ulp), (cs.name, i)
+        st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
+        assert abs(st[2] - (ref["T"] ** 2).sum()) <= 4 * tol * (ref["T"] ** 2).sum()
+
+
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("t", [0, 1])
+@pytest.mark.parametrize("precision,tol", [(1, 1e-4), (0, 2e-2)], ids=["fp32", "bf16"])
+def test_muon_baseline(cfgset, t, precision, tol):
+    _check_muon(cfgset, t, precision, tol)
+
+
+def test_muon_gpt2_full_size_sampled():
+    _check_muon(S.CONFIGS["gpt2_small_G"], 0, 0, 2e-2, indices=[0, 1, 2, 3, 47])
 
 
 # ---------------------------------------------------------------------------
