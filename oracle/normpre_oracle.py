@@ -75,6 +75,7 @@ class OracleConfig:
     power_iters: int = 1            # p
     seed: int = 0                   # Philox key for Omega
     orientation: int = 0            # 0 alternate (paper), 1 row only, 2 column only
+    tangent: str = "relaxed"        # "relaxed" (paper), "strict" or "none" (Table 5a ablations)
 
 
 # --------------------------------------------------------------------------
@@ -175,6 +176,29 @@ def relaxed_tangent(Mbar: np.ndarray, Wbar: np.ndarray) -> np.ndarray:
     momentum; w_i is NOT normalized)."""
     a = np.einsum("ij,ij->i", Mbar, Wbar)
     return Mbar - a[:, None] * Wbar
+
+
+def strict_tangent(Mbar: np.ndarray, Wbar: np.ndarray) -> np.ndarray:
+    """x_i = m_i - <m_i, w_i> w_i / ||w_i||^2: the exact projection onto the
+    tangent space of the row direction, which Sec. 3.1 says the relaxed form
+    recovers when ||w_i|| = 1 (the "strict tangent" ablation of Table 5a).
+    A zero weight row has no direction: x_i = m_i."""
+    a = np.einsum("ij,ij->i", Mbar, Wbar)
+    ww = np.einsum("ij,ij->i", Wbar, Wbar)
+    coef = np.divide(a, ww, out=np.zeros_like(a), where=ww > 0)
+    return Mbar - coef[:, None] * Wbar
+
+
+def tangent_step(Mbar: np.ndarray, Wbar: np.ndarray, mode: str = "relaxed") -> np.ndarray:
+    """The momentum treatment before normalization: the paper's relaxed tangent,
+    or the "strict tangent" / "no tangent" ablations (Table 5a)."""
+    if mode == "relaxed":
+        return relaxed_tangent(Mbar, Wbar)
+    if mode == "strict":
+        return strict_tangent(Mbar, Wbar)
+    if mode == "none":
+        return np.array(Mbar, dtype=np.float64, copy=True)
+    raise ValueError(mode)
 
 
 def diag_gram_normalize(X: np.ndarray):
@@ -296,7 +320,7 @@ def normpre_step(W: np.ndarray, G: np.ndarray, M_prev: np.ndarray, t: int, lr: f
     M = momentum_update(M_prev, G, cfg.momentum)
     k = orientation_of(t, cfg.orientation)
     Wbar, Mbar = orient(W, k), orient(M, k)
-    X = relaxed_tangent(Mbar, Wbar)
+    X = tangent_step(Mbar, Wbar, cfg.tangent)
     Psi, d = diag_gram_normalize(X)
     out = {"M": M, "k": k, "X": X, "Psi": Psi, "d": d}
     if cfg.variant == "G":
@@ -336,7 +360,8 @@ def muon_step(W: np.ndarray, G: np.ndarray, M_prev: np.ndarray, lr: float,
 
 __all__ = [
     "MUON_QUINTIC", "OracleConfig", "philox4x32_10", "philox_uniform", "sketch_omega",
-    "momentum_update", "orientation_of", "orient", "relaxed_tangent", "diag_gram_normalize",
+    "momentum_update", "orientation_of", "orient", "relaxed_tangent", "strict_tangent", "tangent_step",
+    "diag_gram_normalize",
     "newton_schulz", "ns_scalar_map", "interaction_sketch", "exact_interaction_eigs",
     "localized_apply", "rms_matched", "weight_update", "normpre_step", "muon_step",
 ]

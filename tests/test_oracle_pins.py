@@ -461,3 +461,38 @@ def test_muon_singular_values_follow_the_quintic_map():
     # a tall momentum gives the transpose of its transpose's result
     out_t = O.muon_step(np.zeros((30, 10)), G.T, Mp.T, 0.1, cfg)
     np.testing.assert_allclose(out_t["T"], out["T"].T, rtol=0, atol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# Tangent ablations (Table 5a): strict projection and no tangent step
+# ---------------------------------------------------------------------------
+def test_strict_tangent_rows_are_orthogonal_to_the_weights():
+    rng = _rng(40)
+    M = rng.standard_normal((9, 25))
+    W = rng.standard_normal((9, 25)) * np.exp(rng.standard_normal((9, 1)))
+    W[3] = 0.0
+    X = O.strict_tangent(M, W)
+    # orthogonal to every nonzero weight row, equal to m on the zero row
+    ip = np.einsum("ij,ij->i", X, W) / np.maximum(np.linalg.norm(W, axis=1), 1e-300)
+    assert np.max(np.abs(np.delete(ip, 3))) < 1e-13
+    np.testing.assert_array_equal(X[3], M[3])
+    # m = x + (component along w), Pythagoras
+    for i in (0, 5):
+        u = W[i] / np.linalg.norm(W[i])
+        np.testing.assert_allclose(M[i], X[i] + (M[i] @ u) * u, atol=1e-13)
+        assert abs(M[i] @ M[i] - X[i] @ X[i] - (M[i] @ u) ** 2) < 1e-12
+
+
+def test_tangent_modes_special_cases():
+    rng = _rng(41)
+    M = rng.standard_normal((6, 12))
+    W = rng.standard_normal((6, 12))
+    Wn = W / np.linalg.norm(W, axis=1, keepdims=True)
+    # unit weight rows: strict == relaxed (Sec. 3.1)
+    np.testing.assert_allclose(O.tangent_step(M, Wn, "strict"), O.tangent_step(M, Wn, "relaxed"), atol=1e-14)
+    # no tangent step: the momentum itself
+    np.testing.assert_array_equal(O.tangent_step(M, W, "none"), M)
+    # strict is invariant to rescaling a weight row, relaxed is not
+    S = W * np.arange(1, 7)[:, None]
+    np.testing.assert_allclose(O.tangent_step(M, S, "strict"), O.tangent_step(M, W, "strict"), atol=1e-13)
+    assert np.max(np.abs(O.tangent_step(M, S, "relaxed") - O.tangent_step(M, W, "relaxed"))) > 1e-3
