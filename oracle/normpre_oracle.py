@@ -182,11 +182,19 @@ def strict_tangent(Mbar: np.ndarray, Wbar: np.ndarray) -> np.ndarray:
     """x_i = m_i - <m_i, w_i> w_i / ||w_i||^2: the exact projection onto the
     tangent space of the row direction, which Sec. 3.1 says the relaxed form
     recovers when ||w_i|| = 1 (the "strict tangent" ablation of Table 5a).
-    A zero weight row has no direction: x_i = m_i."""
+    A zero weight row has no direction: x_i = m_i.
+    A momentum row parallel to its weight row has no tangent component; what
+    the subtraction leaves of it is rounding, so a result below 1e-4 of the
+    momentum row's norm is taken as zero (reading; the threshold sits above
+    the fp32 rounding of any row the library accepts and far below a real
+    tangent component)."""
     a = np.einsum("ij,ij->i", Mbar, Wbar)
     ww = np.einsum("ij,ij->i", Wbar, Wbar)
     coef = np.divide(a, ww, out=np.zeros_like(a), where=ww > 0)
-    return Mbar - coef[:, None] * Wbar
+    X = Mbar - coef[:, None] * Wbar
+    tiny = np.linalg.norm(X, axis=1) <= 1e-4 * np.linalg.norm(Mbar, axis=1)
+    X[tiny] = 0.0
+    return X
 
 
 def tangent_step(Mbar: np.ndarray, Wbar: np.ndarray, mode: str = "relaxed") -> np.ndarray:

@@ -496,3 +496,15 @@ def test_tangent_modes_special_cases():
     S = W * np.arange(1, 7)[:, None]
     np.testing.assert_allclose(O.tangent_step(M, S, "strict"), O.tangent_step(M, W, "strict"), atol=1e-13)
     assert np.max(np.abs(O.tangent_step(M, S, "relaxed") - O.tangent_step(M, W, "relaxed"))) > 1e-3
+
+
+def test_strict_tangent_of_a_parallel_row_is_zero():
+    # a momentum row parallel to its weight row has no tangent component
+    rng = _rng(42)
+    W = rng.standard_normal((4, 7))
+    M = W * np.array([[2.0], [-0.5], [0.0], [3.0]])
+    X = O.strict_tangent(M, W)
+    assert np.all(X == 0.0)
+    # one-element rows are always parallel
+    X1 = O.strict_tangent(rng.standard_normal((5, 1)), rng.standard_normal((5, 1)))
+    assert np.all(X1 == 0.0)
