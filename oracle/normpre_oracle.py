@@ -184,15 +184,15 @@ def strict_tangent(Mbar: np.ndarray, Wbar: np.ndarray) -> np.ndarray:
     recovers when ||w_i|| = 1 (the "strict tangent" ablation of Table 5a).
     A zero weight row has no direction: x_i = m_i.
     A momentum row parallel to its weight row has no tangent component; what
-    the subtraction leaves of it is rounding, so a result below 1e-4 of the
+    the subtraction leaves of it is rounding, so a result below 1e-3 of the
     momentum row's norm is taken as zero (reading; the threshold sits above
-    the fp32 rounding of any row the library accepts and far below a real
-    tangent component)."""
+    the fp32 rounding of any row the library accepts, including the
+    cancellation of the column-active closed form ||m||^2 - <m, w>^2 / ||w||^2)."""
     a = np.einsum("ij,ij->i", Mbar, Wbar)
     ww = np.einsum("ij,ij->i", Wbar, Wbar)
     coef = np.divide(a, ww, out=np.zeros_like(a), where=ww > 0)
     X = Mbar - coef[:, None] * Wbar
-    tiny = np.linalg.norm(X, axis=1) <= 1e-4 * np.linalg.norm(Mbar, axis=1)
+    tiny = np.linalg.norm(X, axis=1) <= 1e-3 * np.linalg.norm(Mbar, axis=1)
     X[tiny] = 0.0
     return X
 
