@@ -95,6 +95,9 @@ typedef struct normpre_config {
   uint64_t seed;          /* Philox4x32-10 key of the sketch matrix Omega */
   int precision;          /* normpre_precision */
   int orientation;        /* 0: alternate rows/columns with t (paper); 1: rows only; 2: columns only */
+  int tangent;            /* momentum treatment before normalization: 0 relaxed tangent (paper,
+                             x_i = m_i - <m_i, w_i> w_i); 1 none (x_i = m_i); 2 strict tangent
+                             (x_i = m_i - <m_i, w_i> w_i / ||w_i||^2) -- the Table 5a ablations */
 } normpre_config;
 
 /* Fills `cfg` with the paper's defaults (NormPre-G, bf16 Newton-Schulz). */

@@ -99,6 +99,7 @@ struct NormLaunch {
   int mat_id[kMaxBatch] = {};     // global matrix index (into count[])
   int64_t psi_ld = 0;
   float mu = 0.95f;
+  int tangent = 0;                // 0 relaxed (paper), 1 none, 2 strict (Table 5a ablations)
   int* count = nullptr;           // [n_mats] nonzero active rows, accumulated
   int* flags = nullptr;
   // column-active scratch (see normalize_cols_scratch_bytes)

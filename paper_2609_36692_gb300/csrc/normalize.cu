@@ -16,6 +16,18 @@
 //
 // Zero active rows (undefined in Eq. 3) give zero rows of Psi; count[] gets
 // the number of nonzero rows m' (so ||Psi||_F^2 = m').
+//
+// The tangent step subtracts c_i w_i with c_i = <m_i, w_i> (relaxed, the
+// paper's), <m_i, w_i> / ||w_i||^2 (strict tangent ablation; 0 for a zero
+// weight row) or 0 (no-tangent ablation), Table 5a.  A strict-tangent row
+// below 1e-3 of its momentum row's norm is rounding left by a momentum row
+// parallel to its weight row (or by the cancellation of the column-active
+// closed form), and is taken as zero.
+__device__ __forceinline__ float tangent_coef(int mode, float mw, float ww) {
+  if (mode == 0) return mw;
+  if (mode == 2) return ww > 0.f ? mw / ww : 0.f;
+  return 0.f;
+}
 #include <type_traits>
 
 #include "common.cuh"
@@ -51,7 +63,7 @@ __global__ void __launch_bounds__(1024) k_norm_rows_vec(const __grid_constant__ 
   const TW* w = static_cast<const TW*>(a.W[b]) + row * cols;
   TP* psi = static_cast<TP*>(a.psi[b]) + row * a.psi_ld;
   float m[2][8], wv[2][8];
-  float dot = 0.f;
+  float dot = 0.f, wsq = 0.f;
 #pragma unroll
   for (int c = 0; c < 2; ++c) {
     const int64_t j = (static_cast<int64_t>(c) * blockDim.x + threadIdx.x) * 8;
@@ -64,6 +76,7 @@ __global__ void __launch_bounds__(1024) k_norm_rows_vec(const __grid_constant__ 
       for (int e = 0; e < 8; ++e) {
         m[c][e] = fmaf(a.mu, mp[e], gv[e]);
         dot = fmaf(m[c][e], wv[c][e], dot);
+        wsq = fmaf(wv[c][e], wv[c][e], wsq);
       }
       store8(M + j, m[c]);
     } else {
@@ -72,15 +85,29 @@ __global__ void __launch_bounds__(1024) k_norm_rows_vec(const __grid_constant__ 
     }
   }
   dot = block_sum(dot, red);
+  if (a.tangent == 2) wsq = block_sum(wsq, red);
+  const float coef = tangent_coef(a.tangent, dot, wsq);
   float ss = 0.f;
 #pragma unroll
   for (int c = 0; c < 2; ++c)
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-      m[c][e] = fmaf(-dot, wv[c][e], m[c][e]);
+      m[c][e] = fmaf(-coef, wv[c][e], m[c][e]);
       ss = fmaf(m[c][e], m[c][e], ss);
     }
   ss = block_sum(ss, red);
+  if (a.tangent == 2) {
+    float mm = 0.f;
+#pragma unroll
+    for (int c = 0; c < 2; ++c)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float mo = fmaf(coef, wv[c][e], m[c][e]);   // the momentum entry
+        mm = fmaf(mo, mo, mm);
+      }
+    mm = block_sum(mm, red);
+    if (ss <= 1e-6f * mm) ss = 0.f;
+  }
   const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
 #pragma unroll
   for (int c = 0; c < 2; ++c) {
@@ -109,22 +136,32 @@ __global__ void __launch_bounds__(256) k_norm_rows_scalar(const __grid_constant_
   float* M = a.M[b] + row * cols;
   const TW* w = static_cast<const TW*>(a.W[b]) + row * cols;
   TP* psi = static_cast<TP*>(a.psi[b]) + row * a.psi_ld;
-  float dot = 0.f;
+  float dot = 0.f, wsq = 0.f;
   for (int64_t j = threadIdx.x; j < cols; j += blockDim.x) {
     const float m = fmaf(a.mu, M[j], to_f32(g[j]));
     M[j] = m;
-    dot = fmaf(m, to_f32(w[j]), dot);
+    const float wj = to_f32(w[j]);
+    dot = fmaf(m, wj, dot);
+    wsq = fmaf(wj, wj, wsq);
   }
   dot = block_sum(dot, red);
+  if (a.tangent == 2) wsq = block_sum(wsq, red);
+  const float coef = tangent_coef(a.tangent, dot, wsq);
   float ss = 0.f;
+  float mm = 0.f;
   for (int64_t j = threadIdx.x; j < cols; j += blockDim.x) {
-    const float x = fmaf(-dot, to_f32(w[j]), M[j]);
+    const float x = fmaf(-coef, to_f32(w[j]), M[j]);
     ss = fmaf(x, x, ss);
+    mm = fmaf(M[j], M[j], mm);
   }
   ss = block_sum(ss, red);
+  if (a.tangent == 2) {
+    mm = block_sum(mm, red);
+    if (ss <= 1e-6f * mm) ss = 0.f;
+  }
   const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
   for (int64_t j = threadIdx.x; j < cols; j += blockDim.x)
-    psi[j] = from_f32<TP>(fmaf(-dot, to_f32(w[j]), M[j]) * inv);
+    psi[j] = from_f32<TP>(fmaf(-coef, to_f32(w[j]), M[j]) * inv);
   if (threadIdx.x == 0) {
     if (ss > 0.f) atomicAdd(&a.count[a.mat_id[b]], 1);
     if (!isfinite(ss) || !isfinite(dot)) raise_flag(a.flags, kFlagNonfinite);
@@ -227,8 +264,16 @@ __global__ void __launch_bounds__(256) k_norm_cols_final(const __grid_constant__
       s0 += p[0]; s1 += p[1]; s2 += p[2];
       p += cols * 3;
     }
-    const double aa = s1;
-    double d2 = s0 - aa * aa * (2.0 - s2);
+    // relaxed: a = S_mw, ||x||^2 = S_mm - a^2 (2 - S_ww); strict: a = S_mw / S_ww,
+    // ||x||^2 = S_mm - a S_mw; none: a = 0, ||x||^2 = S_mm
+    double aa, d2;
+    if (a.tangent == 0) { aa = s1; d2 = s0 - aa * aa * (2.0 - s2); }
+    else if (a.tangent == 2) {
+      aa = s2 > 0.0 ? s1 / s2 : 0.0;
+      d2 = s0 - aa * s1;
+      if (d2 <= 1e-6 * s0) d2 = 0.0;     // parallel to the weight column: no tangent part
+    }
+    else { aa = 0.0; d2 = s0; }
     if (!(d2 > 0.0)) d2 = (d2 == d2) ? 0.0 : d2;    // clamp rounding below zero, keep NaN
     const float inv = d2 > 0.0 ? static_cast<float>(1.0 / sqrt(d2)) : 0.f;
     a.col_coef[static_cast<int64_t>(b) * cols + j] = make_float2(static_cast<float>(aa), inv);

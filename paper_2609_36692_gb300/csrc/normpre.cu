@@ -88,6 +88,7 @@ int check_config(const normpre_config* c, std::string* msg) {
   }
   if (c->precision != NORMPRE_PREC_BF16 && c->precision != NORMPRE_PREC_F32) { *msg = "bad precision"; return NORMPRE_ERR_ARG; }
   if (c->orientation < 0 || c->orientation > 2) { *msg = "orientation must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
+  if (c->tangent < 0 || c->tangent > 2) { *msg = "tangent must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
   if (c->variant != NORMPRE_L) {
     if (c->ns_steps < 1 || c->ns_steps > 100) { *msg = "ns_steps must be in [1, 100]"; return NORMPRE_ERR_ARG; }
     if (!std::isfinite(c->ns_coef[0]) || !std::isfinite(c->ns_coef[1]) || !std::isfinite(c->ns_coef[2]) ||
@@ -139,6 +140,7 @@ void normpre_default_config(normpre_config* c) {
   c->seed = 0;
   c->precision = NORMPRE_PREC_BF16;
   c->orientation = 0;
+  c->tangent = 0;
 }
 
 const char* normpre_last_error(const normpre_handle* h) {
@@ -332,6 +334,7 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
       }
       a.psi_ld = psi_ld;
       a.mu = c.momentum;
+      a.tangent = c.tangent;
       a.count = h->count;
       a.flags = h->flags;
       a.col_part = h->col_part;

@@ -42,6 +42,7 @@ class normpre_config(ctypes.Structure):
         ("seed", ctypes.c_uint64),
         ("precision", ctypes.c_int),
         ("orientation", ctypes.c_int),
+        ("tangent", ctypes.c_int),
     ]
 
 

@@ -47,6 +47,7 @@ def test_default_config_is_the_papers(lib):
     assert [round(x, 4) for x in cfg.ns_coef] == [3.4445, -4.775, 2.0315]
     assert (cfg.rank, cfg.oversample, cfg.power_iters) == (32, 8, 1)
     assert cfg.precision == lib.NORMPRE_PREC_BF16 and cfg.orientation == 0
+    assert cfg.tangent == 0      # the paper's relaxed tangent
 
 
 def test_host_side_argument_errors(lib):
@@ -73,6 +74,14 @@ def test_host_side_argument_errors(lib):
     bad = C.normpre_default_config(orientation=5)
     with pytest.raises(C.NormPreError):
         C.normpre_init(bad, [(4, 5)], [0], [0])
+    bad = C.normpre_default_config(tangent=3)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    assert "tangent" in C.normpre_last_error()
+    bad = C.normpre_default_config(variant=3)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    assert e.value.status == C.NORMPRE_ERR_ARG
     # stand-alone Newton-Schulz: argument checks come before any device work
     with pytest.raises(C.NormPreError) as e:
         C.normpre_newton_schulz(cfg, 1, 4, 4, 0, 0)
