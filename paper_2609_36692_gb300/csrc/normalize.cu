@@ -23,11 +23,6 @@
 // below 1e-3 of its momentum row's norm is rounding left by a momentum row
 // parallel to its weight row (or by the cancellation of the column-active
 // closed form), and is taken as zero.
-__device__ __forceinline__ float tangent_coef(int mode, float mw, float ww) {
-  if (mode == 0) return mw;
-  if (mode == 2) return ww > 0.f ? mw / ww : 0.f;
-  return 0.f;
-}
 #include <type_traits>
 
 #include "common.cuh"
@@ -38,6 +33,14 @@ namespace normpre {
 constexpr int kColStatsRB = 256;  // rows per block of pass A (one partial sum per block and column)
 constexpr int kColApplyRB = 64;   // rows per block of pass B
 constexpr int kColThreads = 256;  // 32 column chunks of 8 x 8 row lanes
+
+// c_i of the tangent step for mode 0 relaxed, 1 none, 2 strict (mw = <m_i, w_i>,
+// ww = ||w_i||^2).
+__device__ __forceinline__ float tangent_coef(int mode, float mw, float ww) {
+  if (mode == 0) return mw;
+  if (mode == 2) return ww > 0.f ? mw / ww : 0.f;
+  return 0.f;
+}
 
 size_t normalize_cols_part_bytes(int64_t rows, int64_t cols, int n) {
   return static_cast<size_t>(n) * cdiv(rows, kColStatsRB) * cols * 3 * sizeof(double);
