@@ -140,8 +140,12 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
 /*
  * The same step on HOST buffers: copies W, G and M from host memory to device
  * staging buffers owned by the handle (allocated on the first call), runs
- * normpre_step, copies W and M back, and synchronizes `stream`.  Host buffers
- * should be pinned (cudaHostAlloc / torch pin_memory) for full copy speed.
+ * normpre_step, copies W and M back, and synchronizes `stream`.  The copies
+ * run on two streams of the handle and overlap the step shape group by shape
+ * group: a group's normalization starts once its own inputs are in, its M_t
+ * goes back while the other groups are preconditioned, its W once its update
+ * is done.  Host buffers should be pinned (cudaHostAlloc / torch pin_memory)
+ * for full copy speed; they must not be touched until the call returns.
  * Errors: as normpre_step, plus the device-detected conditions of the step.
  */
 int normpre_step_host(normpre_handle* h, int64_t t, float lr, void* const* W_host,

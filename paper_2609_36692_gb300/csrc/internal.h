@@ -170,14 +170,19 @@ class NSPlan {
   // Allocates the buffers of every group and prepares launch descriptors.
   // bf16 = true: tcgen05 tensor-core path; false: fp32 SIMT path.
   cudaError_t init(bool bf16, const std::vector<NSGroupSpec>& groups, std::string* err);
-  // q iterations of X <- aX + (b A + c A^2) X on X[0] of every group, with
-  // X[0] scaled by inscale[] in the first iteration.  Leaves T in out_index().
+  // q iterations of X <- aX + (b A + c A^2) X on X[0] of groups
+  // [g0, g0 + cnt) (cnt < 0: every group from g0) -- with cnt = 1, of its
+  // matrices [m0, m1) (m1 < 0: to the last) -- with X[0] scaled by inscale[]
+  // in the first iteration.  Leaves T in out_index().
   cudaError_t run(int steps, const float coef[3], cudaStream_t s, int* flags,
-                  ProfileHook* prof = nullptr);
+                  ProfileHook* prof = nullptr, int g0 = 0, int cnt = -1, int m0 = 0, int m1 = -1);
   // Computes inscale[] = 1/(sqrt(count[mat_id]) + eps) for matrices whose Psi
-  // rows are unit or zero (Eq. 3), i.e. ||Psi||_F^2 = number of nonzero rows.
+  // rows are unit or zero (Eq. 3), i.e. ||Psi||_F^2 = number of nonzero rows,
+  // for the same selection as run(); group_mat_ids[i] (all the group's
+  // matrices) belongs to group g0 + i.
   cudaError_t scale_from_count(const int* count, const int* const* group_mat_ids, float eps,
-                               cudaStream_t s, ProfileHook* prof = nullptr);
+                               cudaStream_t s, ProfileHook* prof = nullptr, int g0 = 0, int cnt = -1,
+                               int m0 = 0, int m1 = -1);
   // Computes inscale[] = 1/(||X0||_F + eps) directly from X[0].
   cudaError_t scale_from_norm(float eps, cudaStream_t s);
   static int out_index(int steps) { return (steps % 2 == 1) ? 1 : 2; }

@@ -56,14 +56,18 @@ struct normpre_handle {
   std::unique_ptr<NSPlan> ns;  // NormPre-G and Muon
   int last_k = -1;
   bool stepped = false;
-  // host-buffer entry point staging
+  // host-buffer entry point: device staging per matrix, and the copy streams
+  // and per-group events that overlap the copies with the step
   std::vector<void*> stage_w, stage_g, stage_m;
+  cudaStream_t h2d = nullptr, d2h = nullptr;
+  std::vector<cudaEvent_t> in_ev, norm_ev, upd_ev;   // per unit of work
+  cudaEvent_t start_ev = nullptr, out_ev = nullptr;
   ProfileHook prof;
   // NormPre-L: one side stream per shape group so that the groups' sketch
   // pipelines (many small kernels each) run concurrently; joined by events
   std::vector<cudaStream_t> side;
+  std::vector<cudaEvent_t> side_fork;   // the group's normalization is done
   std::vector<cudaEvent_t> side_done;
-  cudaEvent_t fork_ev = nullptr;
   std::string err;
 };
 
@@ -77,6 +81,29 @@ int cuda_fail(normpre_handle* h, cudaError_t e, const char* what) {
   return fail(h, NORMPRE_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
 size_t dsize(int dt) { return dt == NORMPRE_BF16 ? 2 : 4; }
+
+// A piece of one step's work: matrices [b0, b1) of shape group g.
+struct Unit {
+  int g, b0, b1;
+};
+
+// How one step's work is cut and ordered, and points of it where a caller
+// adds work, called with the unit's index on the stream that runs the unit:
+// before its first normalize launch, after its last one (M_t is final), and
+// after its update (W is final).
+struct StepHooks {
+  // the units in the order they are taken (empty: every group whole, in index
+  // order); NormPre-L takes whole groups only
+  std::vector<Unit> units;
+  // NormPre-G / Muon: each unit through all three stages before the next one
+  // starts, instead of one grouped Newton-Schulz launch over every group
+  // (which needs whole groups)
+  bool per_unit = false;
+  virtual ~StepHooks() = default;
+  virtual cudaError_t before_normalize(int, cudaStream_t) { return cudaSuccess; }
+  virtual cudaError_t after_normalize(int, cudaStream_t) { return cudaSuccess; }
+  virtual cudaError_t after_update(int, cudaStream_t) { return cudaSuccess; }
+};
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 int check_config(const normpre_config* c, std::string* msg) {
@@ -154,10 +181,16 @@ void normpre_free(normpre_handle* h) {
   h->ns.reset();
   for (cudaStream_t st : h->side) cudaStreamDestroy(st);
   for (cudaEvent_t ev : h->side_done) cudaEventDestroy(ev);
-  if (h->fork_ev) cudaEventDestroy(h->fork_ev);
+  for (cudaEvent_t ev : h->side_fork) cudaEventDestroy(ev);
   for (void* p : h->allocs) cudaFree(p);
   for (auto* v : {&h->stage_w, &h->stage_g, &h->stage_m})
     for (void* p : *v) cudaFree(p);
+  for (auto* v : {&h->in_ev, &h->norm_ev, &h->upd_ev})
+    for (cudaEvent_t ev : *v) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : {h->start_ev, h->out_ev})
+    if (ev) cudaEventDestroy(ev);
+  for (cudaStream_t st : {h->h2d, h->d2h})
+    if (st) cudaStreamDestroy(st);
   delete h;
 }
 
@@ -238,14 +271,15 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
       if (e != cudaSuccess) return cuda_fail(nullptr, e, "sketch workspace");
     }
     if (h->groups.size() > 1) {
-      if ((e = cudaEventCreateWithFlags(&h->fork_ev, cudaEventDisableTiming))) return cuda_fail(nullptr, e, "cudaEventCreate");
       for (size_t gi = 0; gi < h->groups.size(); ++gi) {
         cudaStream_t st;
-        cudaEvent_t ev;
+        cudaEvent_t ev, fev;
         if ((e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking))) return cuda_fail(nullptr, e, "cudaStreamCreate");
         h->side.push_back(st);
         if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming))) return cuda_fail(nullptr, e, "cudaEventCreate");
         h->side_done.push_back(ev);
+        if ((e = cudaEventCreateWithFlags(&fev, cudaEventDisableTiming))) return cuda_fail(nullptr, e, "cudaEventCreate");
+        h->side_fork.push_back(fev);
       }
     }
   }
@@ -255,8 +289,10 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
   return NORMPRE_OK;
 }
 
-int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const void* const* G, void* const* M,
-                 void* stream) {
+namespace {
+
+int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void* const* G, void* const* M,
+              void* stream, StepHooks& hk) {
   if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
   if (!W || !G || !M) return fail(h, NORMPRE_ERR_ARG, "null pointer array");
   if (!std::isfinite(lr)) return fail(h, NORMPRE_ERR_ARG, "lr must be finite");
@@ -274,45 +310,33 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
   const bool is_muon = (c.variant == NORMPRE_MUON);
   const bool is_g = (c.variant == NORMPRE_G) || is_muon;   // Newton-Schulz preconditioning
   const bool psi_bf16 = is_g && c.precision == NORMPRE_PREC_BF16;
+  // NormPre-L: each group's sketch pipeline runs on its own side stream, from
+  // the end of the group's normalization (joined back into `s` at the end),
+  // except while per-phase profiling is on, whose event pairs must not overlap
+  const bool fork = !is_g && !h->side.empty() && !h->prof.on;
 
-  // (1) momentum + relaxed tangent + diagonal-Gram normalization (Muon: the
-  //     momentum alone, copied to the Newton-Schulz input with ||M||^2 sums)
-  h->prof.begin(kProfNormalize, s);
-  int n_norm = 0;
-  int64_t mslot = 0;   // first Muon partial slot of the group
-  for (size_t gi = 0; gi < h->groups.size() && is_muon; ++gi) {
-    Group& g = h->groups[gi];
-    NSGroupBuf& nb = h->ns->groups()[gi];
-    const int B = static_cast<int>(g.mats.size());
-    const int64_t psi_bs = nb.rows_pad * nb.cols_pad * static_cast<int64_t>(nb.elem);
-    for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
-      NormLaunch a;
-      a.n = std::min(kMaxBatch, B - c0);
-      a.rows = g.rows; a.cols = g.cols;
-      a.g_dtype = g.g_dtype; a.w_dtype = g.w_dtype; a.psi_dtype = psi_bf16 ? 1 : 0;
-      for (int i = 0; i < a.n; ++i) {
-        const int mid = g.mats[c0 + i];
-        a.G[i] = G[mid]; a.M[i] = static_cast<float*>(M[mid]); a.W[i] = W[mid];
-        a.psi[i] = static_cast<char*>(nb.X[0]) + static_cast<int64_t>(c0 + i) * psi_bs;
-        a.mat_id[i] = mid;
-      }
-      a.psi_ld = nb.cols_pad;
-      a.mu = c.momentum;
-      a.flags = h->flags;
-      const int nblk = static_cast<int>(std::min<int64_t>(kMuonBlocks, g.rows));
-      e = launch_momentum_copy(a, h->muon_part + (mslot + c0) * kMuonBlocks, nblk, kMuonBlocks, s);
-      if (e) return cuda_fail(h, e, "momentum launch");
-      ++n_norm;
-    }
-    mslot += B;
+  const int ng = static_cast<int>(h->groups.size());
+  std::vector<Unit> units = hk.units;
+  if (units.empty())
+    for (int gi = 0; gi < ng; ++gi) units.push_back({gi, 0, static_cast<int>(h->groups[gi].mats.size())});
+  for (const Unit& u : units) {
+    const int B = (u.g >= 0 && u.g < ng) ? static_cast<int>(h->groups[u.g].mats.size()) : 0;
+    const bool whole = u.b0 == 0 && u.b1 == B;
+    if (u.g < 0 || u.g >= ng || u.b0 < 0 || u.b0 >= u.b1 || u.b1 > B || (!whole && !(is_g && hk.per_unit)))
+      return fail(h, NORMPRE_ERR_ARG, "internal: bad unit of work");
   }
-  for (size_t gi = 0; gi < h->groups.size() && !is_muon; ++gi) {
-    Group& g = h->groups[gi];
-    const int B = static_cast<int>(g.mats.size());
+  std::vector<int64_t> mslot(ng, 0);   // first Muon partial slot of each group
+  for (int gi = 1; gi < ng; ++gi) mslot[gi] = mslot[gi - 1] + static_cast<int64_t>(h->groups[gi - 1].mats.size());
+
+  // (1) momentum + tangent + diagonal-Gram normalization of one unit (Muon:
+  //     the momentum alone, copied to the Newton-Schulz input with ||M||^2 sums)
+  auto normalize = [&](int ui) -> int {
+    const Unit& u = units[ui];
+    Group& g = h->groups[u.g];
     char* psi_base;
     int64_t psi_ld, psi_bs;
     if (is_g) {
-      NSGroupBuf& nb = h->ns->groups()[gi];
+      NSGroupBuf& nb = h->ns->groups()[u.g];
       psi_base = static_cast<char*>(nb.X[0]);
       psi_ld = nb.cols_pad;
       psi_bs = nb.rows_pad * nb.cols_pad * static_cast<int64_t>(nb.elem);
@@ -321,9 +345,13 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
       psi_ld = g.sk.ld;
       psi_bs = g.rows * g.sk.ld * static_cast<int64_t>(sizeof(float));
     }
-    for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
+    cudaError_t e;
+    if ((e = hk.before_normalize(ui, s))) return cuda_fail(h, e, "stream wait");
+    h->prof.begin(kProfNormalize, s);
+    int n_norm = 0;
+    for (int c0 = u.b0; c0 < u.b1; c0 += kMaxBatch) {
       NormLaunch a;
-      a.n = std::min(kMaxBatch, B - c0);
+      a.n = std::min(kMaxBatch, u.b1 - c0);
       a.rows = g.rows; a.cols = g.cols;
       a.g_dtype = g.g_dtype; a.w_dtype = g.w_dtype; a.psi_dtype = psi_bf16 ? 1 : 0;
       for (int i = 0; i < a.n; ++i) {
@@ -339,96 +367,131 @@ int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const v
       a.flags = h->flags;
       a.col_part = h->col_part;
       a.col_coef = h->col_coef;
-      e = (k == 0) ? launch_normalize_rows(a, s) : launch_normalize_cols(a, s);
+      if (is_muon) {
+        const int nblk = static_cast<int>(std::min<int64_t>(kMuonBlocks, g.rows));
+        e = launch_momentum_copy(a, h->muon_part + (mslot[u.g] + c0) * kMuonBlocks, nblk, kMuonBlocks, s);
+        n_norm += 1;
+      } else {
+        e = (k == 0) ? launch_normalize_rows(a, s) : launch_normalize_cols(a, s);
+        n_norm += (k == 0) ? 1 : 3;
+      }
       if (e) return cuda_fail(h, e, "normalize launch");
-      n_norm += (k == 0) ? 1 : 3;
     }
-  }
-  h->prof.end(kProfNormalize, s, n_norm);
+    h->prof.end(kProfNormalize, s, n_norm);
+    if (fork && (e = cudaEventRecord(h->side_fork[u.g], s))) return cuda_fail(h, e, "cudaEventRecord");
+    if ((e = hk.after_normalize(ui, s))) return cuda_fail(h, e, "copy out");
+    return NORMPRE_OK;
+  };
 
-  if (is_g) {
-    // (2) Newton-Schulz on every group, prescaled by 1/(sqrt(m') + eps)
-    //     (NormPre-G: ||Psi||_F^2 = m'), or by 1/(||M||_F + eps) (Muon)
+  // (2) Newton-Schulz, prescaled by 1/(sqrt(m') + eps) (NormPre-G:
+  //     ||Psi||_F^2 = m'), or by 1/(||M||_F + eps) (Muon), on one unit
+  //     (ui >= 0) or on every group in one grouped launch per product (ui < 0)
+  auto precondition = [&](int ui) -> int {
+    const int g0 = ui < 0 ? 0 : units[ui].g, cnt = ui < 0 ? ng : 1;
+    const int m0 = ui < 0 ? 0 : units[ui].b0, m1 = ui < 0 ? -1 : units[ui].b1;
+    cudaError_t e;
     if (is_muon) {
       h->prof.begin(kProfPrescale, s);
-      int64_t slot = 0;
-      for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+      for (int gi = g0; gi < g0 + cnt; ++gi) {
         Group& g = h->groups[gi];
+        const int b0 = ui < 0 ? 0 : m0, b1 = ui < 0 ? static_cast<int>(g.mats.size()) : m1;
         const int nblk = static_cast<int>(std::min<int64_t>(kMuonBlocks, g.rows));
-        e = launch_muon_prescale(h->muon_part + slot * kMuonBlocks, nblk, kMuonBlocks, static_cast<int>(g.mats.size()),
-                                 h->ns->groups()[gi].inscale, c.ns_eps, s);
+        e = launch_muon_prescale(h->muon_part + (mslot[gi] + b0) * kMuonBlocks, nblk, kMuonBlocks, b1 - b0,
+                                 h->ns->groups()[gi].inscale + b0, c.ns_eps, s);
         if (e) return cuda_fail(h, e, "prescale launch");
-        slot += static_cast<int64_t>(g.mats.size());
       }
-      h->prof.end(kProfPrescale, s, static_cast<int>(h->groups.size()));
+      h->prof.end(kProfPrescale, s, cnt);
     } else {
       std::vector<const int*> ids;
-      for (Group& g : h->groups) ids.push_back(g.mat_ids_dev);
-      e = h->ns->scale_from_count(h->count, ids.data(), c.ns_eps, s, &h->prof);
+      for (int gi = g0; gi < g0 + cnt; ++gi) ids.push_back(h->groups[gi].mat_ids_dev);
+      e = h->ns->scale_from_count(h->count, ids.data(), c.ns_eps, s, &h->prof, g0, cnt, m0, m1);
       if (e) return cuda_fail(h, e, "prescale launch");
     }
-    e = h->ns->run(c.ns_steps, c.ns_coef, s, h->flags, &h->prof);
+    e = h->ns->run(c.ns_steps, c.ns_coef, s, h->flags, &h->prof, g0, cnt, m0, m1);
     if (e) return cuda_fail(h, e, "Newton-Schulz launch");
-    // (3) RMS-matched update with weight decay
+    return NORMPRE_OK;
+  };
+
+  // (3) RMS-matched update with weight decay of one unit
+  auto apply = [&](int ui) -> int {
+    const Unit& u = units[ui];
     const int oi = NSPlan::out_index(c.ns_steps);
+    Group& g = h->groups[u.g];
+    NSGroupBuf& nb = h->ns->groups()[u.g];
+    const int64_t xs = nb.rows_pad * nb.cols_pad * static_cast<int64_t>(nb.elem);
+    cudaError_t e;
     h->prof.begin(kProfApplyG, s);
     int n_apply = 0;
-    for (size_t gi = 0; gi < h->groups.size(); ++gi) {
-      Group& g = h->groups[gi];
-      NSGroupBuf& nb = h->ns->groups()[gi];
-      const int B = static_cast<int>(g.mats.size());
-      const int64_t xs = nb.rows_pad * nb.cols_pad * static_cast<int64_t>(nb.elem);
-      for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
-        ApplyLaunch a;
-        a.n = std::min(kMaxBatch, B - c0);
-        a.rows = g.rows; a.cols = g.cols;
-        a.w_dtype = g.w_dtype; a.t_dtype = psi_bf16 ? 1 : 0;
-        for (int i = 0; i < a.n; ++i) {
-          const int mid = g.mats[c0 + i];
-          a.W[i] = W[mid];
-          a.T[i] = static_cast<char*>(nb.X[oi]) + static_cast<int64_t>(c0 + i) * xs;
-          a.sq_part[i] = nb.sq_part + static_cast<int64_t>(c0 + i) * nb.n_part;
-          a.stats[i] = h->stats + 8 * mid;
-          a.mat_id[i] = mid;
-        }
-        a.count = h->count;
-        a.k = k;
-        a.t_ld = nb.cols_pad;
-        a.n_part = nb.n_part;
-        a.lr = lr; a.wd = c.weight_decay; a.target = c.target_rms;
-        e = launch_apply_g(a, s);
-        if (e) return cuda_fail(h, e, "apply launch");
-        ++n_apply;
+    for (int c0 = u.b0; c0 < u.b1; c0 += kMaxBatch) {
+      ApplyLaunch a;
+      a.n = std::min(kMaxBatch, u.b1 - c0);
+      a.rows = g.rows; a.cols = g.cols;
+      a.w_dtype = g.w_dtype; a.t_dtype = psi_bf16 ? 1 : 0;
+      for (int i = 0; i < a.n; ++i) {
+        const int mid = g.mats[c0 + i];
+        a.W[i] = W[mid];
+        a.T[i] = static_cast<char*>(nb.X[oi]) + static_cast<int64_t>(c0 + i) * xs;
+        a.sq_part[i] = nb.sq_part + static_cast<int64_t>(c0 + i) * nb.n_part;
+        a.stats[i] = h->stats + 8 * mid;
+        a.mat_id[i] = mid;
       }
+      a.count = h->count;
+      a.k = k;
+      a.t_ld = nb.cols_pad;
+      a.n_part = nb.n_part;
+      a.lr = lr; a.wd = c.weight_decay; a.target = c.target_rms;
+      if ((e = launch_apply_g(a, s))) return cuda_fail(h, e, "apply launch");
+      ++n_apply;
     }
     h->prof.end(kProfApplyG, s, n_apply);
+    if ((e = hk.after_update(ui, s))) return cuda_fail(h, e, "copy out");
+    return NORMPRE_OK;
+  };
+
+  const int nu = static_cast<int>(units.size());
+  int rc;
+  if (is_g && hk.per_unit) {
+    for (int ui = 0; ui < nu; ++ui)
+      if ((rc = normalize(ui)) || (rc = precondition(ui)) || (rc = apply(ui))) return rc;
+  } else if (is_g) {
+    for (int ui = 0; ui < nu; ++ui)
+      if ((rc = normalize(ui))) return rc;
+    if ((rc = precondition(-1))) return rc;
+    for (int ui = 0; ui < nu; ++ui)
+      if ((rc = apply(ui))) return rc;
   } else {
     SketchParams p;
     p.rank = c.rank; p.oversample = c.oversample; p.power_iters = c.power_iters;
     p.seed = c.seed; p.t = t; p.k = k;
     p.lr = lr; p.wd = c.weight_decay; p.target = c.target_rms;
-    // groups run concurrently on side streams (forked from and joined back
-    // into `s`), except while per-phase profiling is on, whose event pairs
-    // must not overlap
-    const bool fork = !h->side.empty() && !h->prof.on;
-    if (fork && (e = cudaEventRecord(h->fork_ev, s))) return cuda_fail(h, e, "cudaEventRecord");
-    for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+    for (int ui = 0; ui < nu; ++ui) {
+      if ((rc = normalize(ui))) return rc;
+      const int gi = units[ui].g;
       Group& g = h->groups[gi];
       std::vector<void*> wp;
       for (int mid : g.mats) wp.push_back(W[mid]);
       cudaStream_t gs = fork ? h->side[gi] : s;
-      if (fork && (e = cudaStreamWaitEvent(gs, h->fork_ev, 0))) return cuda_fail(h, e, "cudaStreamWaitEvent");
+      if (fork && (e = cudaStreamWaitEvent(gs, h->side_fork[gi], 0))) return cuda_fail(h, e, "cudaStreamWaitEvent");
       e = run_sketch_group(g.sk, p, g.mat_ids_dev, h->count, wp.data(), h->flags, gs, &h->prof);
       if (e) return cuda_fail(h, e, "sketch launch");
+      if ((e = hk.after_update(ui, gs))) return cuda_fail(h, e, "copy out");
       if (fork && (e = cudaEventRecord(h->side_done[gi], gs))) return cuda_fail(h, e, "cudaEventRecord");
     }
     if (fork)
-      for (size_t gi = 0; gi < h->groups.size(); ++gi)
+      for (int gi = 0; gi < ng; ++gi)
         if ((e = cudaStreamWaitEvent(s, h->side_done[gi], 0))) return cuda_fail(h, e, "cudaStreamWaitEvent");
   }
   h->last_k = k;
   h->stepped = true;
   return NORMPRE_OK;
+}
+
+}  // namespace
+
+int normpre_step(normpre_handle* h, int64_t t, float lr, void* const* W, const void* const* G, void* const* M,
+                 void* stream) {
+  StepHooks none;
+  return step_impl(h, t, lr, W, G, M, stream, none);
 }
 
 int normpre_profile(normpre_handle* h, int enable) {
@@ -469,43 +532,137 @@ int normpre_sync_status(normpre_handle* h, void* stream) {
   return NORMPRE_OK;
 }
 
+namespace {
+
+// Copies of the host-buffer step, overlapped with it.  The step is cut into
+// units of at most kHostUnitBytes of input (whole groups for NormPre-L),
+// largest groups first; the host-to-device stream brings in each unit's W, G,
+// M (one event per unit, which the unit's normalize waits on), and one
+// device-to-host stream sends each unit's M_t back once its normalize is done
+// and its W once its update is done.  A small unit then starts the outgoing
+// copies early, and the step ends on a small unit's work.
+constexpr int64_t kHostUnitBytes = 256ll << 20;
+
+struct HostPipe : StepHooks {
+  normpre_handle* h;
+  void* const* W_host;
+  void* const* M_host;
+  cudaError_t copy_out(int ui, cudaStream_t s, std::vector<cudaEvent_t>& ev, void* const* host,
+                       const std::vector<void*>& stage, bool weights) {
+    const Unit& u = units[ui];
+    cudaError_t e = cudaEventRecord(ev[ui], s);
+    if (!e) e = cudaStreamWaitEvent(h->d2h, ev[ui], 0);
+    for (int b = u.b0; b < u.b1 && !e; ++b) {
+      const int mid = h->groups[u.g].mats[b];
+      const MatInfo& m = h->mats[mid];
+      const size_t bytes = static_cast<size_t>(m.rows * m.cols) * (weights ? dsize(m.w_dtype) : 4);
+      e = cudaMemcpyAsync(host[mid], stage[mid], bytes, cudaMemcpyDeviceToHost, h->d2h);
+    }
+    return e;
+  }
+  cudaError_t before_normalize(int ui, cudaStream_t s) override { return cudaStreamWaitEvent(s, h->in_ev[ui], 0); }
+  cudaError_t after_normalize(int ui, cudaStream_t s) override {
+    return copy_out(ui, s, h->norm_ev, M_host, h->stage_m, false);
+  }
+  cudaError_t after_update(int ui, cudaStream_t s) override {
+    return copy_out(ui, s, h->upd_ev, W_host, h->stage_w, true);
+  }
+};
+
+cudaError_t host_pipe_alloc(normpre_handle* h) {
+  cudaError_t e;
+  for (int i = 0; i < h->n_mats; ++i) {
+    const MatInfo& m = h->mats[i];
+    const size_t n = static_cast<size_t>(m.rows * m.cols);
+    void *pw = nullptr, *pg = nullptr, *pm = nullptr;
+    if ((e = cudaMalloc(&pw, n * dsize(m.w_dtype)))) return e;
+    h->stage_w.push_back(pw);
+    if ((e = cudaMalloc(&pg, n * dsize(m.g_dtype)))) return e;
+    h->stage_g.push_back(pg);
+    if ((e = cudaMalloc(&pm, n * 4))) return e;
+    h->stage_m.push_back(pm);
+  }
+  if ((e = cudaStreamCreateWithFlags(&h->h2d, cudaStreamNonBlocking))) return e;
+  if ((e = cudaStreamCreateWithFlags(&h->d2h, cudaStreamNonBlocking))) return e;
+  if ((e = cudaEventCreateWithFlags(&h->start_ev, cudaEventDisableTiming))) return e;
+  return cudaEventCreateWithFlags(&h->out_ev, cudaEventDisableTiming);
+}
+
+// The units of a host-buffer step, largest groups first.
+std::vector<Unit> host_units(const normpre_handle* h) {
+  std::vector<std::pair<int64_t, int>> by_size;
+  for (size_t gi = 0; gi < h->groups.size(); ++gi) {
+    const Group& g = h->groups[gi];
+    by_size.push_back({-g.rows * g.cols * static_cast<int64_t>(g.mats.size()), static_cast<int>(gi)});
+  }
+  std::stable_sort(by_size.begin(), by_size.end());
+  std::vector<Unit> units;
+  for (auto& sz : by_size) {
+    const Group& g = h->groups[sz.second];
+    const int B = static_cast<int>(g.mats.size());
+    int pieces = 1;
+    if (h->cfg.variant != NORMPRE_L) {
+      const int64_t bytes = g.rows * g.cols * static_cast<int64_t>(dsize(g.w_dtype) + dsize(g.g_dtype) + 4) * B;
+      pieces = static_cast<int>(std::min<int64_t>(B, cdiv(bytes, kHostUnitBytes)));
+    }
+    for (int p = 0; p < pieces; ++p)
+      units.push_back({sz.second, static_cast<int>(static_cast<int64_t>(B) * p / pieces),
+                       static_cast<int>(static_cast<int64_t>(B) * (p + 1) / pieces)});
+  }
+  return units;
+}
+
+}  // namespace
+
 int normpre_step_host(normpre_handle* h, int64_t t, float lr, void* const* W_host, const void* const* G_host,
                       void* const* M_host, void* stream) {
   if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
   if (!W_host || !G_host || !M_host) return fail(h, NORMPRE_ERR_ARG, "null pointer array");
+  for (int i = 0; i < h->n_mats; ++i)
+    if (!W_host[i] || !G_host[i] || !M_host[i]) return fail(h, NORMPRE_ERR_ARG, "null host tensor pointer");
   cudaSetDevice(h->device);
   cudaError_t e;
-  if (h->stage_w.empty()) {
-    for (int i = 0; i < h->n_mats; ++i) {
-      const MatInfo& m = h->mats[i];
-      const size_t n = static_cast<size_t>(m.rows * m.cols);
-      void *pw, *pg, *pm;
-      if ((e = cudaMalloc(&pw, n * dsize(m.w_dtype)))) return cuda_fail(h, e, "cudaMalloc staging");
-      h->stage_w.push_back(pw);
-      if ((e = cudaMalloc(&pg, n * dsize(m.g_dtype)))) return cuda_fail(h, e, "cudaMalloc staging");
-      h->stage_g.push_back(pg);
-      if ((e = cudaMalloc(&pm, n * 4))) return cuda_fail(h, e, "cudaMalloc staging");
-      h->stage_m.push_back(pm);
-    }
-  }
+  if (!h->h2d && (e = host_pipe_alloc(h))) return cuda_fail(h, e, "host-buffer staging");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  for (int i = 0; i < h->n_mats; ++i) {
-    const MatInfo& m = h->mats[i];
-    const size_t n = static_cast<size_t>(m.rows * m.cols);
-    if (!W_host[i] || !G_host[i] || !M_host[i]) return fail(h, NORMPRE_ERR_ARG, "null host tensor pointer");
-    if ((e = cudaMemcpyAsync(h->stage_w[i], W_host[i], n * dsize(m.w_dtype), cudaMemcpyHostToDevice, s))) return cuda_fail(h, e, "H2D");
-    if ((e = cudaMemcpyAsync(h->stage_g[i], G_host[i], n * dsize(m.g_dtype), cudaMemcpyHostToDevice, s))) return cuda_fail(h, e, "H2D");
-    if ((e = cudaMemcpyAsync(h->stage_m[i], M_host[i], n * 4, cudaMemcpyHostToDevice, s))) return cuda_fail(h, e, "H2D");
+  HostPipe pipe;
+  pipe.h = h;
+  pipe.W_host = W_host;
+  pipe.M_host = M_host;
+  pipe.units = host_units(h);
+  pipe.per_unit = true;
+  for (auto* v : {&h->in_ev, &h->norm_ev, &h->upd_ev})
+    while (v->size() < pipe.units.size()) {
+      cudaEvent_t ev;
+      if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming))) return cuda_fail(h, e, "cudaEventCreate");
+      v->push_back(ev);
+    }
+  // the copies start after the work already queued on `s`
+  if ((e = cudaEventRecord(h->start_ev, s))) return cuda_fail(h, e, "cudaEventRecord");
+  if ((e = cudaStreamWaitEvent(h->h2d, h->start_ev, 0)) || (e = cudaStreamWaitEvent(h->d2h, h->start_ev, 0)))
+    return cuda_fail(h, e, "cudaStreamWaitEvent");
+  for (size_t ui = 0; ui < pipe.units.size(); ++ui) {
+    const Unit& u = pipe.units[ui];
+    for (int b = u.b0; b < u.b1; ++b) {
+      const int mid = h->groups[u.g].mats[b];
+      const MatInfo& m = h->mats[mid];
+      const size_t n = static_cast<size_t>(m.rows * m.cols);
+      if ((e = cudaMemcpyAsync(h->stage_w[mid], W_host[mid], n * dsize(m.w_dtype), cudaMemcpyHostToDevice, h->h2d)) ||
+          (e = cudaMemcpyAsync(h->stage_g[mid], G_host[mid], n * dsize(m.g_dtype), cudaMemcpyHostToDevice, h->h2d)) ||
+          (e = cudaMemcpyAsync(h->stage_m[mid], M_host[mid], n * 4, cudaMemcpyHostToDevice, h->h2d)))
+        return cuda_fail(h, e, "H2D");
+    }
+    if ((e = cudaEventRecord(h->in_ev[ui], h->h2d))) return cuda_fail(h, e, "cudaEventRecord");
   }
-  int rc = normpre_step(h, t, lr, h->stage_w.data(), const_cast<const void* const*>(h->stage_g.data()),
-                        h->stage_m.data(), stream);
-  if (rc) return rc;
-  for (int i = 0; i < h->n_mats; ++i) {
-    const MatInfo& m = h->mats[i];
-    const size_t n = static_cast<size_t>(m.rows * m.cols);
-    if ((e = cudaMemcpyAsync(W_host[i], h->stage_w[i], n * dsize(m.w_dtype), cudaMemcpyDeviceToHost, s))) return cuda_fail(h, e, "D2H");
-    if ((e = cudaMemcpyAsync(M_host[i], h->stage_m[i], n * 4, cudaMemcpyDeviceToHost, s))) return cuda_fail(h, e, "D2H");
+  int rc = step_impl(h, t, lr, h->stage_w.data(), const_cast<const void* const*>(h->stage_g.data()),
+                     h->stage_m.data(), stream, pipe);
+  if (rc) {
+    cudaStreamSynchronize(h->h2d);
+    cudaStreamSynchronize(h->d2h);
+    return rc;
   }
+  // `s` (and the caller) sees the step complete once the last copy is back
+  if ((e = cudaEventRecord(h->out_ev, h->d2h)) || (e = cudaStreamWaitEvent(s, h->out_ev, 0)))
+    return cuda_fail(h, e, "cudaEventRecord");
   return normpre_sync_status(h, stream);
 }
 

@@ -98,6 +98,7 @@ struct GemmGroup {
   int a_mn, b_mn;
   int M, N, K, BN;
   int batch, tiles_m, tiles_n, tile_begin;
+  int b_base;                  // index in the group of this launch's first matrix
   int sym;                     // symmetric output: only tiles reaching the diagonal, mirrored
   int per;                     // tiles per matrix
   float ca, cb, diag;
@@ -143,6 +144,7 @@ __device__ __forceinline__ int decode_tile(const GemmArgs& a, int t, int& b, int
   const int l = t - (g.tile_begin >> pairs);
   b = l / per;
   int r = l - b * per;
+  b += g.b_base;
   if (!g.sym) {
     const int tmu = r / g.tiles_n;
     tn = r - tmu * g.tiles_n;
@@ -817,6 +819,7 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
       g.sym = (bf16 && ph < 2) ? 1 : 0;
       g.per = tiles_per_matrix(g.tiles_m, g.tiles_n, g.BN, g.sym);
       g.tile_begin = tiles;
+      g.b_base = 0;
       tiles += g.batch * g.per;
       if (bf16) {
         // tensor maps: Gram reads X (set per run: one map per X buffer is
@@ -864,12 +867,42 @@ cudaError_t NSPlan::init(bool bf16, const std::vector<NSGroupSpec>& specs, std::
   return cudaSuccess;
 }
 
-cudaError_t NSPlan::run(int steps, const float coef[3], cudaStream_t s, int* flags, ProfileHook* prof) {
+// The launch arguments of groups [g0, g0 + cnt) of a prepared grouped
+// launch (their tiles are contiguous and keep their order), or with cnt = 1
+// of matrices [m0, m1) of group g0 (tiles are matrix-major within a group).
+// Returns whether the selection starts and ends on a two-tile cluster unit.
+static bool select_groups(GemmArgs& a, int g0, int cnt, int m0, int m1) {
+  if (g0 == 0 && cnt == a.n_groups && m0 == 0 && m1 == a.g[0].batch) return true;
+  int t0 = a.g[g0].tile_begin;
+  int t1 = (g0 + cnt < a.n_groups) ? a.g[g0 + cnt].tile_begin : a.total_tiles;
+  for (int j = 0; j < cnt; ++j) {
+    a.g[j] = a.g[g0 + j];
+    a.g[j].tile_begin -= t0;
+  }
+  a.n_groups = cnt;
+  if (cnt == 1 && (m0 != 0 || m1 != a.g[0].batch)) {
+    GemmGroup& g = a.g[0];
+    t0 += m0 * g.per;
+    t1 = t0 + (m1 - m0) * g.per;
+    g.batch = m1 - m0;
+    g.b_base = m0;
+  }
+  a.total_tiles = t1 - t0;
+  return (t0 & 1) == 0 && (t1 & 1) == 0;
+}
+
+cudaError_t NSPlan::run(int steps, const float coef[3], cudaStream_t s, int* flags, ProfileHook* prof, int g0,
+                        int cnt, int m0, int m1) {
   ProfileHook none;
   if (!prof) prof = &none;
   NSLaunches* L = static_cast<NSLaunches*>(tc_args_host_);
   if (!L) return cudaErrorInvalidValue;
   const int ng = static_cast<int>(groups_.size());
+  if (cnt < 0) cnt = ng - g0;
+  if (g0 < 0 || cnt < 1 || g0 + cnt > ng) return cudaErrorInvalidValue;
+  const int batch0 = groups_[g0].spec.batch;
+  if (m1 < 0) m1 = batch0;
+  if (m0 < 0 || m0 >= m1 || m1 > batch0 || (cnt > 1 && (m0 != 0 || m1 != batch0))) return cudaErrorInvalidValue;
   const float a = coef[0], b = coef[1], c = coef[2];
   for (int it = 0; it < steps; ++it) {
     const int in = (it == 0) ? 0 : ((it % 2 == 1) ? 1 : 2);
@@ -902,9 +935,10 @@ cudaError_t NSPlan::run(int steps, const float coef[3], cudaStream_t s, int* fla
     GemmArgs* ph[3] = {&gram, &poly, &upd};
     const int cls[3] = {kProfNsGram, kProfNsPoly, kProfNsUpdate};
     for (int p = 0; p < 3; ++p) {
+      const bool units = select_groups(*ph[p], g0, cnt, m0, m1);
       prof->begin(cls[p], s);
       if (bf16_) {
-        if (L->mc[p]) {
+        if (L->mc[p] && units) {
           cudaLaunchConfig_t cfg = {};
           cudaLaunchAttribute attr[1];
           pair_config(&cfg, attr, 2 * std::min(ph[p]->total_tiles / 2, max_pairs_), s);
@@ -926,16 +960,22 @@ cudaError_t NSPlan::run(int steps, const float coef[3], cudaStream_t s, int* fla
 }
 
 cudaError_t NSPlan::scale_from_count(const int* count, const int* const* group_mat_ids, float eps,
-                                     cudaStream_t s, ProfileHook* prof) {
+                                     cudaStream_t s, ProfileHook* prof, int g0, int cnt, int m0, int m1) {
+  const int ng = static_cast<int>(groups_.size());
+  if (cnt < 0) cnt = ng - g0;
+  if (g0 < 0 || cnt < 1 || g0 + cnt > ng) return cudaErrorInvalidValue;
+  const int batch0 = groups_[g0].spec.batch;
+  if (m1 < 0) m1 = batch0;
+  if (m0 < 0 || m0 >= m1 || m1 > batch0 || (cnt > 1 && (m0 != 0 || m1 != batch0))) return cudaErrorInvalidValue;
   ScaleArgs a;
   std::memset(&a, 0, sizeof(a));
-  a.n_groups = static_cast<int>(groups_.size());
+  a.n_groups = cnt;
   a.eps = eps;
   a.count = count;
-  for (int gi = 0; gi < a.n_groups; ++gi) {
-    a.inscale[gi] = groups_[gi].inscale;
-    a.mat_ids[gi] = group_mat_ids[gi];
-    a.batch[gi] = groups_[gi].spec.batch;
+  for (int j = 0; j < cnt; ++j) {
+    a.inscale[j] = groups_[g0 + j].inscale + m0;
+    a.mat_ids[j] = group_mat_ids[j] + m0;
+    a.batch[j] = (cnt == 1) ? m1 - m0 : groups_[g0 + j].spec.batch;
   }
   if (prof) prof->begin(kProfPrescale, s);
   k_scale_from_count<<<a.n_groups, 128, 0, s>>>(a);

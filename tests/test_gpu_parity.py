@@ -389,17 +389,61 @@ def test_deterministic(variant):
         assert np.array_equal(a, b)
 
 
-def test_host_entry_point_matches_device_step():
+@pytest.mark.parametrize("variant", ["G", "L", "muon"])
+def test_host_entry_point_matches_device_step(variant):
+    """Two consecutive host-buffer steps (row- then column-active) equal the
+    device-buffer steps bit for bit: the copies overlapped with the step move
+    each group's inputs in before its normalization and its results out after."""
     import torch
     from paper_2609_36692_gb300 import normpre as C
     cs = SMALL
-    opt, mats, W1, M1 = _run(cs, 0, "G", precision=0)
-    opt2 = _normpre([(m.rows, m.cols) for m in cs.matrices], ["f32"] * cs.n_mats, ["bf16"] * cs.n_mats,
-                    precision=0, seed=1234)
+    mats = S.make_param_set(cs, workers=min(16, os.cpu_count() or 1))
+    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON}[variant],
+              precision=0 if variant != "L" else 1, rank=cs.rank, oversample=cs.oversample,
+              power_iters=cs.power_iters, seed=1234)
+    shapes = [(m.rows, m.cols) for m in cs.matrices]
+    opt = _normpre(shapes, ["f32"] * cs.n_mats, ["bf16"] * cs.n_mats, **kw)
+    opt2 = _normpre(shapes, ["f32"] * cs.n_mats, ["bf16"] * cs.n_mats, **kw)
+    W, G, M = to_device(mats, cs.g_dtype, cs.w_dtype)
     Wh = [torch.from_numpy(m["W"].copy()).pin_memory() for m in mats]
     Gh = [torch.from_numpy(m["G"]).to(torch.bfloat16).pin_memory() for m in mats]
     Mh = [torch.from_numpy(m["M"].copy()).pin_memory() for m in mats]
-    opt2.step_host(0, LR, Wh, Gh, Mh)
-    for i in range(cs.n_mats):
-        assert np.array_equal(Wh[i].numpy(), W1[i])
-        assert np.array_equal(Mh[i].numpy(), M1[i])
+    for t in (0, 1):
+        opt.step(t, LR, W, G, M)
+        torch.cuda.synchronize()
+        opt.status()
+        opt2.step_host(t, LR, Wh, Gh, Mh)
+        for i in range(cs.n_mats):
+            assert np.array_equal(Wh[i].numpy(), to_host(W[i])), (t, i)
+            assert np.array_equal(Mh[i].numpy(), to_host(M[i])), (t, i)
+
+
+@pytest.mark.parametrize("variant", ["G", "muon"])
+def test_host_entry_point_in_units(variant):
+    """A group larger than one host-copy unit (8 x 4096^2 fp32/bf16: about
+    1.3 GB of input) is preconditioned in pieces of matrices between its copies;
+    the result equals the device-buffer step (one grouped launch) bit for bit."""
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    shapes = [(4096, 4096)] * 8 + [(1024, 4096)] * 3
+    gen = torch.Generator().manual_seed(7)
+    Wc = [torch.randn(r, c, generator=gen) * 0.02 for r, c in shapes]
+    Gc = [torch.randn(r, c, generator=gen).to(torch.bfloat16) for r, c in shapes]
+    Mc = [torch.randn(r, c, generator=gen) * 0.1 for r, c in shapes]
+    kw = dict(variant={"G": C.NORMPRE_G, "muon": C.NORMPRE_MUON}[variant], precision=0, seed=1234)
+    opt = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
+    opt2 = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
+    W = [w.cuda() for w in Wc]
+    G = [g.cuda() for g in Gc]
+    M = [m.cuda() for m in Mc]
+    Wh = [w.pin_memory() for w in Wc]
+    Gh = [g.pin_memory() for g in Gc]
+    Mh = [m.pin_memory() for m in Mc]
+    for t in (0, 1):
+        opt.step(t, LR, W, G, M)
+        torch.cuda.synchronize()
+        opt.status()
+        opt2.step_host(t, LR, Wh, Gh, Mh)
+        for i in range(len(shapes)):
+            assert torch.equal(Wh[i], W[i].cpu()), (t, i)
+            assert torch.equal(Mh[i], M[i].cpu()), (t, i)
