@@ -205,6 +205,8 @@ class NSPlan {
 // ----------------------------------------------------------------------------
 struct SketchGroup {
   int batch = 0;
+  int plan_batch = 0;           // batch the launch shapes are planned for (0: batch); a
+                                // slice keeps its group's, so its sums run in the same order
   int64_t rows = 0, cols = 0;   // stored shape
   int w_dtype = 0;
   int64_t ld = 0;               // row stride of Psi (fp32)
@@ -242,6 +244,9 @@ struct SketchParams {
 };
 
 cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::vector<void*>& allocs);
+// Matrices [b0, b1) of a group as a group of their own: the same workspaces
+// from its first matrix on, and tensor maps of Psi over those matrices only.
+cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup* out);
 cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* mat_ids,
                              const int* count, void* const* W, int* flags, cudaStream_t s,
                              ProfileHook* prof);

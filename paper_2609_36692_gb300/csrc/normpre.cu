@@ -93,11 +93,11 @@ struct Unit {
 // after its update (W is final).
 struct StepHooks {
   // the units in the order they are taken (empty: every group whole, in index
-  // order); NormPre-L takes whole groups only
+  // order)
   std::vector<Unit> units;
-  // NormPre-G / Muon: each unit through all three stages before the next one
-  // starts, instead of one grouped Newton-Schulz launch over every group
-  // (which needs whole groups)
+  // each unit through all stages before the next one starts; otherwise
+  // NormPre-G / Muon run one grouped Newton-Schulz launch over every group,
+  // which needs whole groups
   bool per_unit = false;
   virtual ~StepHooks() = default;
   virtual cudaError_t before_normalize(int, cudaStream_t) { return cudaSuccess; }
@@ -322,7 +322,7 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
   for (const Unit& u : units) {
     const int B = (u.g >= 0 && u.g < ng) ? static_cast<int>(h->groups[u.g].mats.size()) : 0;
     const bool whole = u.b0 == 0 && u.b1 == B;
-    if (u.g < 0 || u.g >= ng || u.b0 < 0 || u.b0 >= u.b1 || u.b1 > B || (!whole && !(is_g && hk.per_unit)))
+    if (u.g < 0 || u.g >= ng || u.b0 < 0 || u.b0 >= u.b1 || u.b1 > B || (!whole && !hk.per_unit))
       return fail(h, NORMPRE_ERR_ARG, "internal: bad unit of work");
   }
   std::vector<int64_t> mslot(ng, 0);   // first Muon partial slot of each group
@@ -466,13 +466,17 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
     p.lr = lr; p.wd = c.weight_decay; p.target = c.target_rms;
     for (int ui = 0; ui < nu; ++ui) {
       if ((rc = normalize(ui))) return rc;
-      const int gi = units[ui].g;
+      const Unit& u = units[ui];
+      const int gi = u.g;
       Group& g = h->groups[gi];
       std::vector<void*> wp;
-      for (int mid : g.mats) wp.push_back(W[mid]);
+      for (int b = u.b0; b < u.b1; ++b) wp.push_back(W[g.mats[b]]);
+      SketchGroup part;
+      const bool whole = u.b0 == 0 && u.b1 == static_cast<int>(g.mats.size());
+      if (!whole && (e = sketch_group_slice(g.sk, u.b0, u.b1, &part))) return cuda_fail(h, e, "sketch slice");
       cudaStream_t gs = fork ? h->side[gi] : s;
       if (fork && (e = cudaStreamWaitEvent(gs, h->side_fork[gi], 0))) return cuda_fail(h, e, "cudaStreamWaitEvent");
-      e = run_sketch_group(g.sk, p, g.mat_ids_dev, h->count, wp.data(), h->flags, gs, &h->prof);
+      e = run_sketch_group(whole ? g.sk : part, p, g.mat_ids_dev + u.b0, h->count, wp.data(), h->flags, gs, &h->prof);
       if (e) return cuda_fail(h, e, "sketch launch");
       if ((e = hk.after_update(ui, gs))) return cuda_fail(h, e, "copy out");
       if (fork && (e = cudaEventRecord(h->side_done[gi], gs))) return cuda_fail(h, e, "cudaEventRecord");
@@ -535,8 +539,7 @@ int normpre_sync_status(normpre_handle* h, void* stream) {
 namespace {
 
 // Copies of the host-buffer step, overlapped with it.  The step is cut into
-// units of at most kHostUnitBytes of input (whole groups for NormPre-L),
-// largest groups first; the host-to-device stream brings in each unit's W, G,
+// units of at most kHostUnitBytes of input, largest groups first; the host-to-device stream brings in each unit's W, G,
 // M (one event per unit, which the unit's normalize waits on), and one
 // device-to-host stream sends each unit's M_t back once its normalize is done
 // and its W once its update is done.  A small unit then starts the outgoing
@@ -600,11 +603,8 @@ std::vector<Unit> host_units(const normpre_handle* h) {
   for (auto& sz : by_size) {
     const Group& g = h->groups[sz.second];
     const int B = static_cast<int>(g.mats.size());
-    int pieces = 1;
-    if (h->cfg.variant != NORMPRE_L) {
-      const int64_t bytes = g.rows * g.cols * static_cast<int64_t>(dsize(g.w_dtype) + dsize(g.g_dtype) + 4) * B;
-      pieces = static_cast<int>(std::min<int64_t>(B, cdiv(bytes, kHostUnitBytes)));
-    }
+    const int64_t bytes = g.rows * g.cols * static_cast<int64_t>(dsize(g.w_dtype) + dsize(g.g_dtype) + 4) * B;
+    const int pieces = static_cast<int>(std::min<int64_t>(B, cdiv(bytes, kHostUnitBytes)));
     for (int p = 0; p < pieces; ++p)
       units.push_back({sz.second, static_cast<int>(static_cast<int64_t>(B) * p / pieces),
                        static_cast<int>(static_cast<int64_t>(B) * (p + 1) / pieces)});

@@ -1079,6 +1079,34 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
   return cudaGetLastError();
 }
 
+cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup* out) {
+  if (b0 < 0 || b0 >= b1 || b1 > g.batch) return cudaErrorInvalidValue;
+  SketchGroup s = g;
+  const int64_t vbs = std::max(g.rows, g.cols) * g.lmax;
+  const int64_t sq = static_cast<int64_t>(g.lmax) * g.lmax;
+  s.batch = b1 - b0;
+  s.plan_batch = g.plan_batch ? g.plan_batch : g.batch;
+  s.psi = g.psi + b0 * g.rows * g.ld;
+  float** vbufs[] = {&s.omega, &s.y0, &s.zt, &s.y, &s.q, &s.bt, &s.qk};
+  for (float** v : vbufs) *v += b0 * vbs;
+  s.kpart = g.kpart + b0 * vbs * kMaxKSplit;
+  s.part = g.part + b0 * static_cast<int64_t>(g.max_part) * sq;
+  s.kmat = g.kmat + b0 * sq;
+  s.zvec = g.zvec + b0 * sq;
+  s.ritz = g.ritz + static_cast<int64_t>(b0) * g.lmax;
+  s.stats = g.stats + static_cast<int64_t>(b0) * 8;
+  if (g.tc) {
+    const uint64_t dims[3] = {static_cast<uint64_t>(g.cols), static_cast<uint64_t>(g.rows),
+                              static_cast<uint64_t>(s.batch)};
+    const uint64_t strides[2] = {static_cast<uint64_t>(g.ld) * 4, static_cast<uint64_t>(g.rows * g.ld) * 4};
+    const uint32_t box_k[3] = {32, 128, 1}, box_mn[3] = {32, 32, 1};
+    s.tc = driver_encode_tiled(&s.psi_map_k, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, s.psi, dims, strides, box_k, nullptr) &&
+           driver_encode_tiled(&s.psi_map_mn, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, s.psi, dims, strides, box_mn, nullptr);
+  }
+  *out = s;
+  return cudaSuccess;
+}
+
 cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* mat_ids,
                              const int* count, void* const* W, int* flags, cudaStream_t s,
                              ProfileHook* prof) {
@@ -1119,7 +1147,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   auto contract = [&](bool trans, const float* v, float* out) -> cudaError_t {
     prof->begin(kProfContract, s);
     const int64_t P = trans ? g.cols : g.rows, K = trans ? g.rows : g.cols;
-    const int64_t tiles = cdiv(P, use_tc ? 128 : kCtP) * B;
+    const int64_t tiles = cdiv(P, use_tc ? 128 : kCtP) * (g.plan_batch ? g.plan_batch : B);
     int ks = 1;
     const int64_t want = (use_tc ? 1 : 2) * static_cast<int64_t>(device_sm_count());
     while (ks < kMaxKSplit && tiles * ks < want && K / (2 * ks) >= 256) ks *= 2;

@@ -418,11 +418,11 @@ def test_host_entry_point_matches_device_step(variant):
             assert np.array_equal(Mh[i].numpy(), to_host(M[i])), (t, i)
 
 
-@pytest.mark.parametrize("variant", ["G", "muon"])
+@pytest.mark.parametrize("variant", ["G", "L", "muon"])
 def test_host_entry_point_in_units(variant):
     """A group larger than one host-copy unit (8 x 4096^2 fp32/bf16: about
     1.3 GB of input) is preconditioned in pieces of matrices between its copies;
-    the result equals the device-buffer step (one grouped launch) bit for bit."""
+    the result equals the device-buffer step (whole groups) bit for bit."""
     import torch
     from paper_2609_36692_gb300 import normpre as C
     shapes = [(4096, 4096)] * 8 + [(1024, 4096)] * 3
@@ -430,7 +430,8 @@ def test_host_entry_point_in_units(variant):
     Wc = [torch.randn(r, c, generator=gen) * 0.02 for r, c in shapes]
     Gc = [torch.randn(r, c, generator=gen).to(torch.bfloat16) for r, c in shapes]
     Mc = [torch.randn(r, c, generator=gen) * 0.1 for r, c in shapes]
-    kw = dict(variant={"G": C.NORMPRE_G, "muon": C.NORMPRE_MUON}[variant], precision=0, seed=1234)
+    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON}[variant],
+              precision=0 if variant != "L" else 1, seed=1234)
     opt = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
     opt2 = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
     W = [w.cuda() for w in Wc]
