@@ -282,23 +282,36 @@ __global__ void __launch_bounds__(kCtThreads) k_contract(const __grid_constant__
 // A V = Ahi Vhi + Ahi Vlo + Alo Vhi up to the dropped Alo Vlo term and the
 // rounding of lo: below 2^-21 relative per product (fp32 FMA: 2^-24).
 //
-// The TF32 MMA takes only K-major operands, while V ([K][l]) and, for Psi^T,
-// Psi arrive MN-major, so the split pass also transposes: TMA copies 32-deep
-// K blocks as they lie (Psi K-major: box 32 x 128; Psi^T and V: boxes of
-// 32 K rows x 32 elements), and four warps write hi and lo tiles in the
-// K-major 128-byte-swizzle layout (row r, 16-byte chunk j at r * 128 +
-// ((j ^ (r & 7)) * 16)).  A quarter warp then reads one swizzled row or
-// writes eight consecutive rows of one chunk: no bank conflicts either way.
+// Psi, the streamed operand, goes to the tensor core through tensor memory:
+// TMA copies 32-deep K blocks into shared memory as they lie (Psi K-major:
+// box 32 x 128; Psi^T: four boxes of 32 K rows x 32 elements), eight warps
+// read each row of the 128-row A tile (a quarter warp reads eight rows of one
+// 16-byte chunk, or one word of 32 consecutive elements: no bank conflicts),
+// split it in registers and write hi and lo into TMEM with tcgen05.st (lane =
+// row, one 32-bit column per K element), where the MMAs read A.  Only the
+// small V operand ([K][l], MN-major) is split into shared memory: the TF32
+// MMA takes K-major shared-memory operands only, so its split also transposes
+// (hi and lo tiles in the K-major 128-byte-swizzle layout, row r, 16-byte
+// chunk j at r * 128 + ((j ^ (r & 7)) * 16)), while the TMEM stores drain.
+// (Splitting V once per contraction in a kernel of its own, or freeing the
+// Psi copies before the MMAs through a second ring, measured slower.)
 //
-// One CTA computes a 128 x l tile of one matrix over one K split: warp 0
-// issues the TMA copies into a 3-stage ring, warps 2-9 split, warp 1 issues
-// the 12 MMAs of a block (M = 128, N = l rounded up to 16, K = 8) into a TMEM
-// accumulator.  The tensor core's fp32 accumulation is biased toward zero by
-// up to an ulp per addition, which over thousands of K steps reaches 1e-4
-// relative; so every kCtcSeg blocks the MMAs switch to the other of two TMEM
-// accumulators and warps 2-5 drain the finished one into fp32 registers with
-// round-to-nearest additions (bias bounded by ~48 additions, ~3e-6); warps
-// 2-5 (one per TMEM lane quarter) drain and write the result.
+// A TF32 MMA of M = 128, K = 8 costs the same ~94 cycles for any N up to 128
+// (measured), so the three products take two instructions per K step: the V
+// hi and lo tiles lie one after the other (rows 0..63 and 64..127 of one
+// operand), and Ahi [Vhi; Vlo] (N = 64 + np, np = l rounded up to 16) fills
+// accumulator columns 0..63 with Ahi Vhi and 64.. with Ahi Vlo, then Alo Vhi
+// (N = np) adds into columns 0..np-1.
+//
+// The kernel is persistent: one CTA per SM walks the units (matrix, K split,
+// 128-row tile), carrying its 4-stage ring and accumulators from one unit to
+// the next.  Warp 0 issues the TMA copies, warps 2-9 split, warp 1 issues the
+// MMAs, which free the stage.  The tensor core's fp32 accumulation is biased
+// toward zero by up to an ulp per addition, which over thousands of K steps
+// reaches 1e-4 relative; so every kCtcSeg blocks the MMAs switch to the other
+// of two TMEM accumulators and warps 2-5 (one per TMEM lane quarter) drain the
+// finished one into fp32 registers with round-to-nearest additions (bias
+// bounded by ~32 additions, ~2e-6), and write each unit's result.
 // ---------------------------------------------------------------------------
 struct ContractTcArgs {
   CUtensorMap psi_map;    // {cols, rows, batch} fp32, 128-byte swizzle
@@ -307,16 +320,25 @@ struct ContractTcArgs {
   int64_t P, K;
   int l, np;              // np = MMA N = l rounded up to 16 (<= 64)
   int64_t kchunk;         // K range of one split (multiple of 32)
+  int ksplit, batch;      // K splits and matrices (the units are tiles x ksplit x batch)
   int* flags;
 };
-constexpr int kCtcStages = 3;
+// Stage st of the ring: copies of the Psi block and of the V block (TMA),
+// the split V hi / lo tiles in shared memory and the split A hi / lo in TMEM;
+// the MMAs free the stage.
+constexpr int kCtcStages = 4;
 constexpr int kCtcSeg = 4;                           // K blocks per accumulator segment
 constexpr int kCtcA = 128 * 32 * 4;                  // one A tile (128 rows x 32 K): 16 KB
 constexpr int kCtcV = 64 * 32 * 4;                   // one V tile (64 rows x 32 K): 8 KB
-constexpr int kCtcStage = 3 * kCtcA + 3 * kCtcV;     // copy, hi, lo of both: 72 KB
+constexpr int kCtcStage = kCtcA + 3 * kCtcV;         // A copy, V copy, V hi, V lo: 40 KB
 constexpr int kCtcSplitWarps = 8;
-constexpr int kCtcThreads = 64 + 32 * kCtcSplitWarps;
-constexpr size_t kCtcSmem = 1024 + kCtcStages * kCtcStage + 256;
+constexpr int kCtcThreads = 64 + 32 * kCtcSplitWarps; // TMA, MMA, 8 split warps
+constexpr size_t kCtcSmem = 1024 + kCtcStages * kCtcStage + 512;
+// TMEM columns: two 128-column accumulators, then per stage 32 columns of A
+// hi and 32 of A lo
+constexpr uint32_t kCtcTmemA = 256;
+constexpr uint32_t kCtcTmemCols = 512;
+static_assert(kCtcTmemA + 64 * kCtcStages <= kCtcTmemCols, "TMEM budget");
 
 // x rounded to the nearest TF32 value (ties away from zero), as an fp32 bit
 // pattern with the low 13 mantissa bits clear: adding half of the dropped
@@ -334,17 +356,6 @@ __device__ __forceinline__ void split4(const float4 x, float4& h, float4& l) {
 // byte offset of 16-byte chunk j of row r in a 128-byte-swizzled tile
 __device__ __forceinline__ uint32_t sw128(int r, int j) { return static_cast<uint32_t>(r * 128 + ((j ^ (r & 7)) << 4)); }
 
-// K-major source (nr rows of 32 K values, already swizzled): elementwise
-// split; the split warps take consecutive 16-byte chunks.
-__device__ __forceinline__ void split_kmajor(const uint8_t* src, uint8_t* hi, uint8_t* lo, int nr, int w, int lane) {
-  for (int i = w * 32 + lane; i < nr * 8; i += 32 * kCtcSplitWarps) {
-    const float4 x = *reinterpret_cast<const float4*>(src + 16 * i);
-    float4 h, l;
-    split4(x, h, l);
-    *reinterpret_cast<float4*>(hi + 16 * i) = h;
-    *reinterpret_cast<float4*>(lo + 16 * i) = l;
-  }
-}
 // MN-major source box (32 K rows x 32 elements, swizzled, rows = K) ->
 // K-major rows r0 + c (c = lane) of the hi / lo tiles, K chunks j0 .. j0 + NJ - 1.
 template <int NJ>
@@ -364,36 +375,65 @@ __device__ __forceinline__ void split_transpose(const uint8_t* box, uint8_t* hi,
     *reinterpret_cast<float4*>(lo + sw128(r, j)) = l;
   }
 }
+// 16 consecutive 32-bit TMEM columns of the warp's 32 lanes: thread i writes
+// lane (base + i).
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+      "%14, %15, %16};" ::"r"(taddr),
+      "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]), "f"(v[8]), "f"(v[9]),
+      "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// D[tmem] (+)= A[tmem] * B[smem]^T, kind::tf32
+__device__ __forceinline__ void mma_tf32_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 
 template <bool TRANS>
 __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_constant__ ContractTcArgs a) {
   extern __shared__ uint8_t ctc_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(ctc_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kCtcStages * kCtcStage);
-  uint64_t* splitb = full + kCtcStages;
-  uint64_t* empty = splitb + kCtcStages;
-  uint64_t* tfull = empty + kCtcStages;    // [2]
-  uint64_t* tempty = tfull + 2;            // [2]
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kCtcStages * kCtcStage);   // [kCtcStages] copies landed
+  uint64_t* splitb = full + kCtcStages;      // [kCtcStages] split written
+  uint64_t* empty = splitb + kCtcStages;     // [kCtcStages] MMAs done with the stage
+  uint64_t* tfull = empty + kCtcStages;      // [2] accumulator segment complete
+  uint64_t* tempty = tfull + 2;              // [2] accumulator drained
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [kCtcStages] last parity + 1
-  // stage layout: A copy | A hi | A lo | V copy | V hi | V lo
+  // stage layout: A copy | V copy | V hi | V lo
   auto a_copy = [&](int st) { return smem + st * kCtcStage; };
-  auto v_copy = [&](int st) { return smem + st * kCtcStage + 3 * kCtcA; };
+  auto v_copy = [&](int st) { return smem + st * kCtcStage + kCtcA; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.y;
-  const int64_t p0 = static_cast<int64_t>(blockIdx.x) * 128;
-  const int64_t kbeg = static_cast<int64_t>(blockIdx.z) * a.kchunk;
-  const int64_t kend = min(a.K, kbeg + a.kchunk);
-  const int nk = kend > kbeg ? static_cast<int>((kend - kbeg + 31) / 32) : 0;
   const int nvb = a.np > 32 ? 2 : 1;
+  // work units u = (matrix b, K split z, row tile p), matrix-major so that
+  // consecutive units share the V operand in L2; each CTA takes every
+  // gridDim.x-th unit and carries its ring and accumulators across units
+  const int tiles = static_cast<int>((a.P + 127) / 128);
+  const int units = tiles * a.ksplit * a.batch;
+  auto unit_of = [&](int u, int& b, int& z, int64_t& p0, int64_t& kbeg, int& nk) {
+    p0 = static_cast<int64_t>(u % tiles) * 128;
+    z = (u / tiles) % a.ksplit;
+    b = u / (tiles * a.ksplit);
+    kbeg = static_cast<int64_t>(z) * a.kchunk;
+    const int64_t kend = min(a.K, kbeg + a.kchunk);
+    nk = kend > kbeg ? static_cast<int>((kend - kbeg + 31) / 32) : 0;
+  };
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kCtcStages; ++s) {
-      tc::mbar_init(&full[s], 1);
-      tc::mbar_init(&splitb[s], kCtcSplitWarps);
-      tc::mbar_init(&empty[s], 1);
-      issued[s] = 0;
+    for (int st = 0; st < kCtcStages; ++st) {
+      tc::mbar_init(&full[st], 1);
+      tc::mbar_init(&splitb[st], kCtcSplitWarps);
+      tc::mbar_init(&empty[st], 1);
+      issued[st] = 0;
     }
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&tfull[i], 1);
@@ -405,99 +445,117 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
     tc::prefetch_map(&a.v_map);
   }
   if (warp == 1) {
-    tc::tmem_alloc(tmem_slot, 128);        // two accumulators of 64 columns
+    tc::tmem_alloc(tmem_slot, kCtcTmemCols);
     tc::tmem_relinquish();
     tc::fence_before();
   }
+  // with l <= 32 the split writes rows 0..31 of V hi and lo only; rows 32..63
+  // enter the wide MMA and must read as zero
+  if (nvb == 1)
+    for (int st = 0; st < kCtcStages; ++st)
+      for (int i = threadIdx.x; i < 2 * kCtcV / 16; i += blockDim.x)
+        reinterpret_cast<float4*>(v_copy(st) + kCtcV)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   __syncthreads();
   tc::fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int nseg = (nk + kCtcSeg - 1) / kCtcSeg;
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
     bool ok = true;
-    for (int kb = 0; kb < nk && ok; ++kb) {
-      const int st = kb % kCtcStages;
-      const uint32_t ph = (kb / kCtcStages) & 1;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[st], ph ^ 1u, abort_flag));
-      if (!ok) break;
-      if (lane == 0) {
-        tc::mbar_expect_tx(&full[st], static_cast<uint32_t>(kCtcA + nvb * 4096));
-        issued[st] = ph + 1;
-        const int k0 = static_cast<int>(kbeg) + 32 * kb, pr = static_cast<int>(p0);
-        if (!TRANS) {
-          tc::tma_load_3d(a_copy(st), &a.psi_map, &full[st], k0, pr, b);
-        } else {
+    uint32_t it = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      int b, z, nk;
+      int64_t p0, kbeg;
+      unit_of(u, b, z, p0, kbeg, nk);
+      for (int kb = 0; kb < nk && ok; ++kb, ++it) {
+        const int st = it % kCtcStages;
+        const uint32_t ph = (it / kCtcStages) & 1;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[st], ph ^ 1u, abort_flag));
+        if (!ok) break;
+        if (lane == 0) {
+          tc::mbar_expect_tx(&full[st], static_cast<uint32_t>(kCtcA + nvb * 4096));
+          issued[st] = ph + 1;
+          const int k0 = static_cast<int>(kbeg) + 32 * kb, pr = static_cast<int>(p0);
+          if (!TRANS) {
+            tc::tma_load_3d(a_copy(st), &a.psi_map, &full[st], k0, pr, b);
+          } else {
 #pragma unroll
-          for (int j = 0; j < 4; ++j) tc::tma_load_3d(a_copy(st) + j * 4096, &a.psi_map, &full[st], pr + 32 * j, k0, b);
+            for (int j = 0; j < 4; ++j) tc::tma_load_3d(a_copy(st) + j * 4096, &a.psi_map, &full[st], pr + 32 * j, k0, b);
+          }
+          for (int j = 0; j < nvb; ++j) tc::tma_load_3d(v_copy(st) + j * 4096, &a.v_map, &full[st], 32 * j, k0, b);
         }
-        for (int j = 0; j < nvb; ++j) tc::tma_load_3d(v_copy(st) + j * 4096, &a.v_map, &full[st], 32 * j, k0, b);
+        __syncwarp();
       }
-      __syncwarp();
     }
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
-    const uint32_t idesc = tc::idesc_tf32(128, a.np, 0, 0);
+    const uint32_t idesc_w = tc::idesc_tf32(128, 64 + a.np, 0, 0);   // Ahi [Vhi; Vlo]
+    const uint32_t idesc_n = tc::idesc_tf32(128, a.np, 0, 0);        // Alo Vhi
     bool ok = true;
-    for (int kb = 0; kb < nk && ok; ++kb) {
-      const int st = kb % kCtcStages;
-      const uint32_t ph = (kb / kCtcStages) & 1;
-      const int seg = kb / kCtcSeg, acc = seg & 1;
-      const bool seg_first = (kb % kCtcSeg) == 0;
-      const bool seg_last = (kb % kCtcSeg) == kCtcSeg - 1 || kb == nk - 1;
-      if (seg_first) {
-        // the accumulator's previous segment has been drained
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(&tempty[acc], ((seg >> 1) & 1) ^ 1u, abort_flag));
+    uint32_t it = 0, gseg = 0;   // stage counter; segment counter over all units
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      int b, z, nk;
+      int64_t p0, kbeg;
+      unit_of(u, b, z, p0, kbeg, nk);
+      for (int kb = 0; kb < nk && ok; ++kb, ++it) {
+        const int st = it % kCtcStages;
+        const uint32_t ph = (it / kCtcStages) & 1;
+        const bool seg_first = (kb % kCtcSeg) == 0;
+        const bool seg_last = (kb % kCtcSeg) == kCtcSeg - 1 || kb == nk - 1;
+        const int acc = gseg & 1;
+        if (seg_first) {
+          // the accumulator's previous segment has been drained
+          ok = __all_sync(0xffffffffu, tc::mbar_wait(&tempty[acc], ((gseg >> 1) & 1) ^ 1u, abort_flag));
+          if (!ok) break;
+          tc::fence_after();
+        }
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&splitb[st], ph, abort_flag));
         if (!ok) break;
         tc::fence_after();
-      }
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&splitb[st], ph, abort_flag));
-      if (!ok) break;
-      tc::fence_after();
-      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(64 * acc);
-      if (lane == 0) {
-        const uint32_t ahi = tc::su32(a_copy(st) + kCtcA), alo = ahi + kCtcA;
-        const uint32_t vhi = tc::su32(v_copy(st) + kCtcV), vlo = vhi + kCtcV;
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(128 * acc);
+        if (lane == 0) {
+          const uint32_t ahi = tmem_base + kCtcTmemA + 64u * st, alo = ahi + 32u;
+          const uint32_t vhi = tc::su32(v_copy(st) + kCtcV);   // V lo follows at row 64
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {       // K step of 8 fp32 = 32 bytes of a K-major row
-          const uint64_t dah = tc::sdesc(ahi + kk * 32, 16, 1024);
-          const uint64_t dal = tc::sdesc(alo + kk * 32, 16, 1024);
-          const uint64_t dvh = tc::sdesc(vhi + kk * 32, 16, 1024);
-          const uint64_t dvl = tc::sdesc(vlo + kk * 32, 16, 1024);
-          tc::mma_tf32(d_tmem, dah, dvh, idesc, (!seg_first || kk != 0) ? 1u : 0u);
-          tc::mma_tf32(d_tmem, dah, dvl, idesc, 1u);
-          tc::mma_tf32(d_tmem, dal, dvh, idesc, 1u);
+          for (int kk = 0; kk < 4; ++kk) {       // K step of 8: 8 TMEM columns of A, 32 bytes of a V row
+            const uint64_t dv = tc::sdesc(vhi + kk * 32, 16, 1024);
+            mma_tf32_ta(d_tmem, ahi + 8 * kk, dv, idesc_w, (!seg_first || kk != 0) ? 1u : 0u);
+            mma_tf32_ta(d_tmem, alo + 8 * kk, dv, idesc_n, 1u);
+          }
+          tc::mma_commit(&empty[st]);
+          if (seg_last) tc::mma_commit(&tfull[acc]);
         }
-        tc::mma_commit(&empty[st]);
-        if (seg_last) tc::mma_commit(&tfull[acc]);
+        __syncwarp();
+        if (seg_last) ++gseg;
       }
-      __syncwarp();
     }
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
   } else {
-    // ---------------- split (warps 2..9), segment drains and epilogue (warps 2..5) ----------------
+    // ---------------- split (warps 2..9), segment drains and epilogues (warps 2..5) ----------------
     const int w = warp - 2;
     const bool drainer = w < 4;
-    const int q = warp & 3;
+    const int q = warp & 3;        // TMEM lane quarter this warp may access
+    const int kh = w >> 2;         // half of each 32-deep K block this warp splits
     float sum[64];
-#pragma unroll
-    for (int j = 0; j < 64; ++j) sum[j] = 0.f;
     // adds the accumulator of segment `seg` into sum (round to nearest) and
     // hands the accumulator back to the MMA warp
-    auto drain = [&](int seg) -> bool {
+    auto drain = [&](uint32_t seg) -> bool {
       const int acc = seg & 1;
       if (!__all_sync(0xffffffffu, tc::mbar_wait(&tfull[acc], (seg >> 1) & 1, abort_flag))) return false;
       tc::fence_after();
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         if (32 * h < a.np) {
-          uint32_t r[32];
-          tc::tmem_ld32(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(64 * acc + 32 * h), r);
+          // Ahi Vhi + Alo Vhi in columns 32 h.., Ahi Vlo in 64 + 32 h..
+          uint32_t r[32], v[32];
+          const uint32_t col = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * acc + 32 * h);
+          tc::tmem_ld32(col, r);
+          tc::tmem_ld32(col + 64u, v);
           tc::tmem_ld_wait();
 #pragma unroll
-          for (int j = 0; j < 32; ++j) sum[32 * h + j] += __uint_as_float(r[j]);
+          for (int j = 0; j < 32; ++j) sum[32 * h + j] += __uint_as_float(r[j]) + __uint_as_float(v[j]);
         }
       }
       tc::fence_before();
@@ -506,49 +564,92 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
       return true;
     };
     bool ok = true;
-    for (int kb = 0; kb < nk && ok; ++kb) {
-      const int st = kb % kCtcStages;
-      const uint32_t ph = (kb / kCtcStages) & 1;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&full[st], ph, abort_flag));
-      if (!ok) break;
-      uint8_t* ac = a_copy(st);
-      uint8_t* vc = v_copy(st);
-      // A: K-major chunks, or box w / 2, chunk half w % 2; V: box w / 4,
-      // chunk pair w % 4 (two boxes) or box 0, chunk w (one box)
-      if (!TRANS) split_kmajor(ac, ac + kCtcA, ac + 2 * kCtcA, 128, w, lane);
-      else split_transpose<4>(ac + (w >> 1) * 4096, ac + kCtcA, ac + 2 * kCtcA, 32 * (w >> 1), lane, 4 * (w & 1));
-      if (nvb == 2) split_transpose<2>(vc + (w >> 2) * 4096, vc + kCtcV, vc + 2 * kCtcV, 32 * (w >> 2), lane, 2 * (w & 3));
-      else split_transpose<1>(vc, vc + kCtcV, vc + 2 * kCtcV, 0, lane, w);
-      // the MMAs read these tiles through the async proxy
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&splitb[st]);
-      // the previous segment ends with the block before this one: drain it
-      // while the MMAs of this segment start
-      if (drainer && kb % kCtcSeg == 0 && kb > 0) ok = drain(kb / kCtcSeg - 1);
-    }
-    if (drainer && ok && nseg > 0) ok = drain(nseg - 1);
-    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
-    const int64_t row = p0 + 32 * q + lane;
-    float* out = a.out + b * a.out_bs + static_cast<int64_t>(blockIdx.z) * a.P * a.l;
-    if (drainer && row < a.P) {
+    uint32_t it = 0, gseg = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      int b, z, nk;
+      int64_t p0, kbeg;
+      unit_of(u, b, z, p0, kbeg, nk);
 #pragma unroll
-      for (int j = 0; j < 64; ++j)
-        if (j < a.l) out[row * a.l + j] = ok ? sum[j] : 0.f;
+      for (int j = 0; j < 64; ++j) sum[j] = 0.f;
+      for (int kb = 0; kb < nk && ok; ++kb, ++it) {
+        const int st = it % kCtcStages;
+        const uint32_t ph = (it / kCtcStages) & 1;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&full[st], ph, abort_flag));
+        if (!ok) break;
+        // this stage's TMEM columns were last read by MMAs whose completion
+        // reached here through the empty -> TMA -> full chain
+        tc::fence_after();
+        const uint8_t* ac = a_copy(st);
+        uint8_t* vc = v_copy(st);
+        // A row r = 32 q + lane (the warp's TMEM lane quarter), K half kh
+        {
+          const int r = 32 * q + lane;
+          float x[16], hi[16], lo[16];
+          if (!TRANS) {
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc) {
+              const float4 v = *reinterpret_cast<const float4*>(ac + sw128(r, 4 * kh + cc));
+              x[4 * cc] = v.x; x[4 * cc + 1] = v.y; x[4 * cc + 2] = v.z; x[4 * cc + 3] = v.w;
+            }
+          } else {
+            const uint8_t* box = ac + q * 4096;   // elements 32 q .. 32 q + 31, K rows 0..31
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              x[e] = *reinterpret_cast<const float*>(box + sw128(16 * kh + e, lane >> 2) + 4 * (lane & 3));
+          }
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            hi[e] = tf32_rna(x[e]);
+            lo[e] = tf32_rna(x[e] - hi[e]);
+          }
+          const uint32_t ta = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + kCtcTmemA + 64u * st + 16u * kh;
+          tmem_st16(ta, hi);
+          tmem_st16(ta + 32u, lo);
+        }
+        // V (box w / 4, chunk pair w % 4 of two boxes, or box 0, chunk w of
+        // one) while the TMEM stores drain
+        if (nvb == 2) split_transpose<2>(vc + (w >> 2) * 4096, vc + kCtcV, vc + 2 * kCtcV, 32 * (w >> 2), lane, 2 * (w & 3));
+        else split_transpose<1>(vc, vc + kCtcV, vc + 2 * kCtcV, 0, lane, w);
+        tmem_st_wait();
+        // the MMAs read V through the async proxy and A from TMEM
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        tc::fence_before();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&splitb[st]);
+        // the previous segment of this unit ends with the block before this
+        // one: drain it while the MMAs of this segment start
+        if (kb % kCtcSeg == 0 && kb > 0) {
+          if (drainer) ok = drain(gseg);
+          ++gseg;
+        }
+      }
+      if (!ok) break;
+      if (nk > 0) {
+        if (drainer) ok = drain(gseg);
+        ++gseg;
+      }
+      const int64_t row = p0 + 32 * q + lane;
+      float* out = a.out + b * a.out_bs + static_cast<int64_t>(z) * a.P * a.l;
+      if (drainer && ok && row < a.P) {
+#pragma unroll
+        for (int j = 0; j < 64; ++j)
+          if (j < a.l) out[row * a.l + j] = sum[j];
+      }
     }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
   }
   __syncthreads();
   if (threadIdx.x == 0 && *abort_flag) {
     // let every TMA copy still in flight land before the CTA exits
     volatile int never = 0;
-    for (int s = 0; s < kCtcStages; ++s)
-      if (issued[s]) tc::mbar_wait(&full[s], issued[s] - 1, &never);
+    for (int st = 0; st < kCtcStages; ++st)
+      if (issued[st]) tc::mbar_wait(&full[st], issued[st] - 1, &never);
   }
   __syncthreads();
   if (warp == 1) {
     __syncwarp();
     tc::fence_after();
-    tc::tmem_dealloc(tmem_base, 128);
+    tc::tmem_dealloc(tmem_base, kCtcTmemCols);
   }
 }
 
@@ -1164,6 +1265,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     }
     cudaError_t err;
     if (use_tc) {
+      const int np = static_cast<int>(round_up(l, 16));
       ContractTcArgs ct;
       std::memset(static_cast<void*>(&ct), 0, sizeof(ct));
       ct.psi_map = trans ? g.psi_map_mn : g.psi_map_k;
@@ -1175,10 +1277,13 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
                                vbox, &why))
         return cudaErrorInvalidValue;
       ct.out = c.out; ct.out_bs = c.out_bs;
-      ct.P = P; ct.K = K; ct.l = l; ct.np = static_cast<int>(round_up(l, 16));
+      ct.P = P; ct.K = K; ct.l = l; ct.np = np;
       ct.kchunk = c.kchunk;
       ct.flags = flags;
-      const dim3 grid(static_cast<unsigned>(cdiv(P, 128)), static_cast<unsigned>(B), static_cast<unsigned>(ks));
+      ct.ksplit = ks; ct.batch = B;
+      // persistent: one CTA per SM (shared memory and TMEM admit one)
+      const int64_t units = cdiv(P, 128) * ks * B;
+      const unsigned grid = static_cast<unsigned>(std::min<int64_t>(units, device_sm_count()));
       if (trans) k_contract_tc<true><<<grid, kCtcThreads, kCtcSmem, s>>>(ct);
       else k_contract_tc<false><<<grid, kCtcThreads, kCtcSmem, s>>>(ct);
       err = cudaGetLastError();
@@ -1195,7 +1300,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       k_split_reduce<<<dim3(static_cast<unsigned>(cdiv(r.n, 256)), B), 256, 0, s>>>(r);
       err = cudaGetLastError();
       if (err) return err;
-      n_l = 2;
+      ++n_l;
     }
     prof->end(kProfContract, s, n_l);
     return cudaSuccess;
