@@ -42,8 +42,8 @@ LR = 0.02
 # (dram__bytes_read.sum + dram__bytes_write.sum), per workload; None until a
 # capture of the current kernel exists (profiles/ keeps the summaries).
 NCU_TRAFFIC_PER_LAUNCH = {
-    "gpt2_small_G": 211.1e6,   # mean of the Gram, poly and update launches of one NS iteration
-    "gpt2_small_L": 108.1e6,   # mean of six k_contract_tc launches (both operand orientations)
+    "gpt2_small_G": 208.1e6,   # mean of 15 launches: Gram, poly and update of five NS iterations
+    "gpt2_small_L": 108.0e6,   # mean of six k_contract_tc launches (both operand orientations)
 }
 
 
