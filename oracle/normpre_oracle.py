@@ -42,6 +42,8 @@ Readings taken where the paper is silent:
   fp64); normals by Box-Muller on word pairs (0,1), (2,3).
 * Top-r selection: Ritz values sorted in descending order with a stable sort
   (ties keep the lower index), r' = min(r, l), then C = {i <= r' : lam_i > 1}.
+* Spectral energies (App. E): "nonzero" eigenvalues are those above 1e-6 of
+  the largest.
 * Muon baseline (the comparison optimizer of Sec. 4 and App. A): the same
   momentum, the Newton-Schulz iteration applied to the momentum itself (no
   orientation, tangent or normalization step, Sec. 2.1), and the update
@@ -366,10 +368,45 @@ def muon_step(W: np.ndarray, G: np.ndarray, M_prev: np.ndarray, lr: float,
     return {"M": M, "T": T, "R": R, "W": weight_update(W, R, lr, cfg.weight_decay)}
 
 
+# --------------------------------------------------------------------------
+# Diagnostics (App. E: spectral dynamics and training dynamics)
+# --------------------------------------------------------------------------
+def spectral_energies(lam: np.ndarray, r: int, nonzero_rel: float = 1e-6) -> Dict[str, float]:
+    """Spectral transformation energies of App. E: with the eigenvalues lam of
+    Gamma = Psi Psi^T, each mode's energy is the squared change of its singular
+    value under global preconditioning, e_i = (sqrt(lam_i) - 1)^2.  E_top sums
+    over C (the at most r largest eigenvalues above one), E_remain over the
+    other eigenvalues above one, E_sub over the nonzero ones below one;
+    E_global is their sum.  "Nonzero" is read as lam_i > nonzero_rel * lam_max
+    (the paper's exact zeros are rounding-level values in floating point)."""
+    lam = np.sort(np.asarray(lam, dtype=np.float64))[::-1]
+    e = (np.sqrt(np.maximum(lam, 0.0)) - 1.0) ** 2
+    lmax = lam[0] if lam.size else 0.0
+    above = lam > 1.0
+    n_c = min(int(r), int(above.sum()))
+    top = float(e[:n_c].sum())
+    remain = float(e[n_c:][above[n_c:]].sum())
+    sub_mask = (lam > nonzero_rel * lmax) & (lam < 1.0)
+    sub = float(e[sub_mask].sum())
+    return {"E_top": top, "E_remain": remain, "E_sub": sub, "E_global": top + remain + sub}
+
+
+def descent_alignment(G: np.ndarray, Phi: np.ndarray) -> float:
+    """Per-matrix descent alignment of App. E: the cosine similarity
+    <G, Phi>_F / (||G||_F ||Phi||_F) of the gradient and the update direction
+    before learning-rate scaling and without weight decay (the paper averages
+    it over the matrices)."""
+    G = np.asarray(G, dtype=np.float64)
+    Phi = np.asarray(Phi, dtype=np.float64)
+    den = np.linalg.norm(G) * np.linalg.norm(Phi)
+    return float(np.sum(G * Phi) / den) if den > 0 else 0.0
+
+
 __all__ = [
     "MUON_QUINTIC", "OracleConfig", "philox4x32_10", "philox_uniform", "sketch_omega",
     "momentum_update", "orientation_of", "orient", "relaxed_tangent", "strict_tangent", "tangent_step",
     "diag_gram_normalize",
     "newton_schulz", "ns_scalar_map", "interaction_sketch", "exact_interaction_eigs",
     "localized_apply", "rms_matched", "weight_update", "normpre_step", "muon_step",
+    "spectral_energies", "descent_alignment",
 ]

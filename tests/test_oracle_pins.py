@@ -508,3 +508,51 @@ def test_strict_tangent_of_a_parallel_row_is_zero():
     # one-element rows are always parallel
     X1 = O.strict_tangent(rng.standard_normal((5, 1)), rng.standard_normal((5, 1)))
     assert np.all(X1 == 0.0)
+
+
+# --------------------------------------------------------------------------
+# Diagnostics (App. E)
+# --------------------------------------------------------------------------
+def test_spectral_energies_hand_worked():
+    """lam = (4, 2.25, 1, 0.25, 0) with r = 1: C = {4} gives (2 - 1)^2 = 1;
+    2.25 remains (0.5^2); lam = 1 contributes nothing; 0.25 gives (0.5 - 1)^2;
+    the zero eigenvalue is not a mode."""
+    e = O.spectral_energies(np.array([0.25, 4.0, 0.0, 1.0, 2.25]), r=1)
+    assert e["E_top"] == 1.0 and e["E_remain"] == 0.25 and e["E_sub"] == 0.25
+    assert e["E_global"] == 1.5
+    # r larger than the modes above one: everything above one is in C
+    e = O.spectral_energies(np.array([4.0, 2.25, 0.25]), r=8)
+    assert e["E_top"] == 1.25 and e["E_remain"] == 0.0
+
+
+def test_spectral_energies_match_singular_values():
+    """E_global = sum over the nonzero singular values of (sigma - 1)^2
+    = ||Psi||_F^2 - 2 ||Psi||_* + rank(Psi), taken here from an SVD of Psi
+    (the energies come from the eigenvalues of Psi Psi^T)."""
+    rng = np.random.default_rng(5)
+    Psi, _ = O.diag_gram_normalize(rng.standard_normal((24, 7)) @ rng.standard_normal((7, 40)))
+    sv = np.linalg.svd(Psi, compute_uv=False)
+    sv = sv[sv > 1e-8]
+    want = np.sum(Psi ** 2) - 2 * sv.sum() + sv.size
+    ex = O.exact_interaction_eigs(Psi, r=3)
+    e = O.spectral_energies(ex["lam"], r=3)
+    assert abs(e["E_global"] - want) < 1e-9 * max(1.0, want)
+    assert abs(e["E_global"] - np.sum((sv - 1.0) ** 2)) < 1e-9 * max(1.0, want)
+    # C holds the three largest singular values' modes (all above one here)
+    assert np.all(sv[:3] > 1.0)
+    assert abs(e["E_top"] - np.sum((sv[:3] - 1.0) ** 2)) < 1e-9
+
+
+def test_descent_alignment_identities():
+    rng = np.random.default_rng(6)
+    G = rng.standard_normal((9, 13))
+    assert abs(O.descent_alignment(G, G) - 1.0) < 1e-15
+    assert abs(O.descent_alignment(G, -3.0 * G) + 1.0) < 1e-15
+    H = rng.standard_normal((9, 13))
+    H -= np.sum(G * H) / np.sum(G * G) * G          # orthogonal to G
+    assert abs(O.descent_alignment(G, H)) < 1e-12
+    # the RMS matching of Sec. 3.1 is a positive scale: it leaves the cosine
+    T = rng.standard_normal((13, 9))
+    R = O.rms_matched(T, 1, 0.2)
+    assert abs(O.descent_alignment(G, R) - O.descent_alignment(G, T.T)) < 1e-12
+    assert O.descent_alignment(G, np.zeros_like(G)) == 0.0
