@@ -47,10 +47,17 @@ typedef struct normpre_handle normpre_handle;
 enum normpre_variant {
   NORMPRE_G = 0,   /* global: T = msign(Psi) by Newton-Schulz (Sec. 3.2) */
   NORMPRE_L = 1,   /* localized: randomized interaction sketch (Alg. 2) */
-  NORMPRE_MUON = 2 /* not NormPre: the paper's comparison optimizer Muon (Sec. 2.1, Sec. 4),
+  NORMPRE_MUON = 2, /* not NormPre: the paper's comparison optimizer Muon (Sec. 2.1, Sec. 4),
                       i.e. Newton-Schulz applied to the momentum itself, with no orientation,
                       tangent or normalization step, and the same RMS-matched update; it
                       shares the Newton-Schulz kernels and serves the latency comparison */
+  NORMPRE_L_EXACT = 3 /* localized with exact eigenspace extraction (Sec. 3.2, App. B): the
+                      interaction matrix Gamma = Psi_a Psi_a^T (m_a x m_a) formed on the GPU, its
+                      full symmetric eigendecomposition, the up to r largest eigenvalues above
+                      one.  Costs O(m_a^2 n_a + m_a^3) per matrix: the reference for the sketch
+                      and the source of the spectral diagnostics, not a fast path.  The dense
+                      eigensolver is cuSOLVER's syevd, loaded at run time (NORMPRE_ERR_UNAVAILABLE
+                      when it cannot be loaded) */
 };
 
 /* Storage dtypes of caller tensors. */
@@ -69,7 +76,8 @@ enum normpre_status {
   NORMPRE_ERR_CUDA = 5,       /* a CUDA runtime call failed (message has the CUDA error) */
   NORMPRE_ERR_NONFINITE = 6,  /* NaN or Inf met in the momentum or weights (device flag) */
   NORMPRE_ERR_NUMERIC = 7,    /* CholeskyQR breakdown or Jacobi sweep cap reached (device flag) */
-  NORMPRE_ERR_TIMEOUT = 8     /* a bounded device-side wait gave up (device flag) */
+  NORMPRE_ERR_TIMEOUT = 8,    /* a bounded device-side wait gave up (device flag) */
+  NORMPRE_ERR_UNAVAILABLE = 9 /* NORMPRE_L_EXACT: the cuSOLVER library could not be loaded */
 };
 
 /* Which precision the spectral stage computes in. */
@@ -98,6 +106,9 @@ typedef struct normpre_config {
   int tangent;            /* momentum treatment before normalization: 0 relaxed tangent (paper,
                              x_i = m_i - <m_i, w_i> w_i); 1 none (x_i = m_i); 2 strict tangent
                              (x_i = m_i - <m_i, w_i> w_i / ||w_i||^2) -- the Table 5a ablations */
+  int diagnostics;        /* 1: every step also accumulates, per matrix, <G, T>, ||G||^2 and
+                             ||T||^2 of the raw gradient G and the preconditioned update T (one
+                             more read of G and T), for the descent alignment of NORMPRE_BUF_DIAG */
 } normpre_config;
 
 /* Fills `cfg` with the paper's defaults (NormPre-G, bf16 Newton-Schulz). */
@@ -168,7 +179,17 @@ enum normpre_buffer {
   NORMPRE_BUF_RITZ = 3,   /* NormPre-L: all l Ritz values, descending, fp32 (1 x l) */
   NORMPRE_BUF_Z = 4,      /* NormPre-L: Ritz vectors Z (l x l, column j = j-th Ritz value), fp32 */
   NORMPRE_BUF_OMEGA = 5,  /* NormPre-L: sketch matrix Omega of the last step, n_a x l, fp32 */
-  NORMPRE_BUF_STATS = 6   /* 1 x 8 fp32: [k, m', ||T||_F^2, |C|, l, n_a, m_a, 0] of the last step */
+  NORMPRE_BUF_STATS = 6,  /* 1 x 8 fp32: [k, m', ||T||_F^2, |C|, l, n_a, m_a, 0] of the last step */
+  NORMPRE_BUF_EIGS = 7,   /* NORMPRE_L_EXACT: all m_a eigenvalues of Gamma, descending (1 x m_a) */
+  NORMPRE_BUF_DIAG = 8    /* 1 x 8 fp32 diagnostics of the last step: [E_top, E_remain, E_sub,
+                             E_global, cos(G, Phi), ||G||_F, ||T||_F, <G, T>].  The spectral
+                             transformation energies sum e_i = (sqrt(lambda_i) - 1)^2 over the
+                             eigenvalues of Gamma in C (top, at most r above one), above one but
+                             not in C (remain), and in (0, 1) (sub); "nonzero" means lambda_i >
+                             1e-6 lambda_max; NaN unless NORMPRE_L_EXACT.  Phi = R_k(T) is the
+                             update direction before the learning rate, without weight decay, so
+                             cos(G, Phi) = <G, T> / (||G|| ||T||) in the stored layout: the
+                             descent alignment of one matrix; NaN unless cfg.diagnostics */
 };
 
 /*

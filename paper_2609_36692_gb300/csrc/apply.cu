@@ -74,4 +74,41 @@ cudaError_t launch_apply_g(const ApplyLaunch& a, cudaStream_t s) {
   return go((bf16*)0, (bf16*)0);
 }
 
+// Descent-alignment sums of a Newton-Schulz step: <G, T>, ||G||^2, ||T||^2 of
+// every matrix, T in the stored layout (row stride t_ld), accumulated into
+// diag[4..6] with fp64 atomics (diagnostics: not bitwise reproducible).
+__global__ void __launch_bounds__(256) k_diag_gt(const __grid_constant__ DiagLaunch a) {
+  __shared__ double red[32];
+  const int b = blockIdx.y;
+  double gt = 0, gg = 0, tt = 0;
+  const int64_t n = a.rows * a.cols;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i / a.cols, c = i - r * a.cols;
+    const float g = a.g_dtype ? to_f32(static_cast<const bf16*>(a.G[b])[i]) : static_cast<const float*>(a.G[b])[i];
+    const float t = a.t_dtype ? to_f32(static_cast<const bf16*>(a.T[b])[r * a.t_ld + c])
+                              : static_cast<const float*>(a.T[b])[r * a.t_ld + c];
+    gt += static_cast<double>(g) * t;
+    gg += static_cast<double>(g) * g;
+    tt += static_cast<double>(t) * t;
+  }
+  gt = block_sum(gt, red);
+  gg = block_sum(gg, red);
+  tt = block_sum(tt, red);
+  if (threadIdx.x == 0) {
+    atomicAdd(a.diag[b] + 4, gt);
+    atomicAdd(a.diag[b] + 5, gg);
+    atomicAdd(a.diag[b] + 6, tt);
+  }
+}
+
+cudaError_t launch_diag_gt(const DiagLaunch& a, cudaStream_t s) {
+  if (a.n <= 0) return cudaSuccess;
+  int64_t per = cdiv(a.rows * a.cols, 256 * 8);
+  const int64_t cap = cdiv(static_cast<int64_t>(device_sm_count()) * 4, a.n);
+  per = std::max<int64_t>(1, std::min(per, cap));
+  k_diag_gt<<<dim3(static_cast<unsigned>(per), static_cast<unsigned>(a.n)), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
 }  // namespace normpre

@@ -138,6 +138,18 @@ struct ApplyLaunch {
   float lr = 0, wd = 0, target = 0.2f;
 };
 cudaError_t launch_apply_g(const ApplyLaunch& a, cudaStream_t s);
+// Descent-alignment sums <G, T>, ||G||^2, ||T||^2 per matrix into diag[4..6].
+struct DiagLaunch {
+  int n = 0;
+  int64_t rows = 0, cols = 0;
+  const void* G[kMaxBatch] = {};
+  int g_dtype = 0;
+  const void* T[kMaxBatch] = {};      // stored layout, row stride t_ld
+  int t_dtype = 0;
+  int64_t t_ld = 0;
+  double* diag[kMaxBatch] = {};
+};
+cudaError_t launch_diag_gt(const DiagLaunch& a, cudaStream_t s);
 
 // ----------------------------------------------------------------------------
 // Newton-Schulz (ns.cu)
@@ -229,6 +241,16 @@ struct SketchGroup {
   float* stats = nullptr;       // [8] per matrix
   int lmax = 0;
   int max_part = 0;
+  // NORMPRE_L_EXACT: Gamma of one matrix (then its eigenvectors), its
+  // eigenvalues, all eigenvalues of every matrix (descending), the eigensolver
+  // workspace and status, and the cuSOLVER handle
+  float* gamma = nullptr;
+  float* eig_w = nullptr;
+  float* eig_all = nullptr;     // [batch][max(rows, cols)]
+  float* eig_work = nullptr;
+  int* eig_info = nullptr;
+  int eig_lwork = 0;
+  void* solver = nullptr;
   // tensor-core contractions: TMA maps of Psi as the K-major (box 32 x 128)
   // and MN-major (box 32 x 32) A operand; tc = false keeps the SIMT kernel
   CUtensorMap psi_map_k, psi_map_mn;
@@ -241,9 +263,23 @@ struct SketchParams {
   int64_t t = 0;
   int k = 0;                    // orientation of this step
   float lr = 0, wd = 0, target = 0.2f;
+  bool exact = false;           // NORMPRE_L_EXACT: exact eigenpairs instead of the sketch
+  const int* mat_ids_host = nullptr;   // the group's (or slice's) matrix ids, host copy
+  double* diag = nullptr;       // [n_mats][8] diagnostics (energies, alignment sums) or null
+  const void* const* G = nullptr;      // with diag: the step's gradients (same order as W)
+  int g_dtype = 0;
 };
 
 cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::vector<void*>& allocs);
+// NORMPRE_L_EXACT (exact.cu): whether cuSOLVER could be loaded; the Gamma and
+// eigensolver workspaces of a group (one matrix at a time); the solver handle's
+// release; and the exact eigenpairs of every matrix of g into q, ritz, zvec,
+// kmat, stats (and the spectral energies into diag).
+int exact_available(std::string* why);
+cudaError_t exact_group_alloc(SketchGroup& g, std::vector<void*>& allocs, std::string* why);
+void exact_group_free(SketchGroup& g);
+cudaError_t exact_eigs(SketchGroup& g, const SketchParams& p, int l, const int* mat_ids_host, const int* count,
+                       double* diag, int* flags, cudaStream_t s);
 // Matrices [b0, b1) of a group as a group of their own: the same workspaces
 // from its first matrix on, and tensor maps of Psi over those matrices only.
 cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup* out);

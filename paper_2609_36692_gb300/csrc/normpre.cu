@@ -5,6 +5,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <limits>
 #include <map>
 #include <memory>
 #include <string>
@@ -53,6 +54,7 @@ struct normpre_handle {
   double* col_part = nullptr;  // column-active scratch
   float2* col_coef = nullptr;
   double* muon_part = nullptr; // Muon: ||M||^2 partials, [group slot][kMuonBlocks] per group
+  double* diag = nullptr;      // [n_mats][8]: spectral energies (exact), alignment sums
   std::unique_ptr<NSPlan> ns;  // NormPre-G and Muon
   int last_k = -1;
   bool stepped = false;
@@ -105,18 +107,25 @@ struct StepHooks {
   virtual cudaError_t after_update(int, cudaStream_t) { return cudaSuccess; }
 };
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+// Newton-Schulz preconditioning (NormPre-G, Muon) or the localized one (L, L exact)
+bool uses_ns(int variant) { return variant == NORMPRE_G || variant == NORMPRE_MUON; }
+constexpr int64_t kExactMaxDim = 16384;   // Gamma of one matrix is the L-exact workspace
 
 int check_config(const normpre_config* c, std::string* msg) {
-  if (c->variant != NORMPRE_G && c->variant != NORMPRE_L && c->variant != NORMPRE_MUON) {
-    *msg = "variant must be NORMPRE_G, NORMPRE_L or NORMPRE_MUON"; return NORMPRE_ERR_ARG;
+  if (c->variant != NORMPRE_G && c->variant != NORMPRE_L && c->variant != NORMPRE_MUON &&
+      c->variant != NORMPRE_L_EXACT) {
+    *msg = "variant must be NORMPRE_G, NORMPRE_L, NORMPRE_MUON or NORMPRE_L_EXACT"; return NORMPRE_ERR_ARG;
   }
+  if (c->diagnostics != 0 && c->diagnostics != 1) { *msg = "diagnostics must be 0 or 1"; return NORMPRE_ERR_ARG; }
   if (!std::isfinite(c->momentum) || !std::isfinite(c->weight_decay) || !std::isfinite(c->target_rms)) {
     *msg = "momentum, weight_decay and target_rms must be finite"; return NORMPRE_ERR_ARG;
   }
   if (c->precision != NORMPRE_PREC_BF16 && c->precision != NORMPRE_PREC_F32) { *msg = "bad precision"; return NORMPRE_ERR_ARG; }
   if (c->orientation < 0 || c->orientation > 2) { *msg = "orientation must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
   if (c->tangent < 0 || c->tangent > 2) { *msg = "tangent must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
-  if (c->variant != NORMPRE_L) {
+  if (c->variant == NORMPRE_L_EXACT) {
+    if (c->rank < 1 || c->rank > 64) { *msg = "need 1 <= rank <= 64"; return NORMPRE_ERR_ARG; }
+  } else if (uses_ns(c->variant)) {
     if (c->ns_steps < 1 || c->ns_steps > 100) { *msg = "ns_steps must be in [1, 100]"; return NORMPRE_ERR_ARG; }
     if (!std::isfinite(c->ns_coef[0]) || !std::isfinite(c->ns_coef[1]) || !std::isfinite(c->ns_coef[2]) ||
         !(c->ns_eps >= 0.f)) { *msg = "bad Newton-Schulz coefficients or eps"; return NORMPRE_ERR_ARG; }
@@ -179,6 +188,7 @@ void normpre_free(normpre_handle* h) {
   cudaSetDevice(h->device);
   cudaDeviceSynchronize();
   h->ns.reset();
+  for (Group& g : h->groups) exact_group_free(g.sk);
   for (cudaStream_t st : h->side) cudaStreamDestroy(st);
   for (cudaEvent_t ev : h->side_done) cudaEventDestroy(ev);
   for (cudaEvent_t ev : h->side_fork) cudaEventDestroy(ev);
@@ -205,6 +215,9 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
   for (int i = 0; i < n_mats; ++i) {
     if (rows[i] < 1 || cols[i] < 1 || rows[i] > 65536 || cols[i] > 65536)
       return fail(nullptr, NORMPRE_ERR_SHAPE, "matrix " + std::to_string(i) + ": each dimension must be in [1, 65536]");
+    if (cfg->variant == NORMPRE_L_EXACT && std::max(rows[i], cols[i]) > kExactMaxDim)
+      return fail(nullptr, NORMPRE_ERR_SHAPE, "matrix " + std::to_string(i) + ": NORMPRE_L_EXACT supports " +
+                  "dimensions up to " + std::to_string(kExactMaxDim));
     if ((w_dtype[i] != NORMPRE_F32 && w_dtype[i] != NORMPRE_BF16) || (g_dtype[i] != NORMPRE_F32 && g_dtype[i] != NORMPRE_BF16))
       return fail(nullptr, NORMPRE_ERR_DTYPE, "matrix " + std::to_string(i) + ": dtype must be NORMPRE_F32 or NORMPRE_BF16");
   }
@@ -232,13 +245,14 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
     h->mats[i] = MatInfo{rows[i], cols[i], w_dtype[i], g_dtype[i], gi, static_cast<int>(h->groups[gi].mats.size())};
     h->groups[gi].mats.push_back(i);
   }
-  if (cfg->variant != NORMPRE_L && h->groups.size() > static_cast<size_t>(kMaxGroups))
+  if (uses_ns(cfg->variant) && h->groups.size() > static_cast<size_t>(kMaxGroups))
     return fail(nullptr, NORMPRE_ERR_SHAPE, "the Newton-Schulz variants support at most " + std::to_string(kMaxGroups) +
                 " distinct (shape, dtype) groups per handle");
   normpre_handle* hp = h.get();
   if ((e = dalloc(hp, &h->count, sizeof(int) * n_mats))) return cuda_fail(nullptr, e, "cudaMalloc");
   if ((e = dalloc(hp, &h->flags, sizeof(int) * 4))) return cuda_fail(nullptr, e, "cudaMalloc");
   if ((e = dalloc(hp, &h->stats, sizeof(float) * 8 * n_mats))) return cuda_fail(nullptr, e, "cudaMalloc");
+  if ((e = dalloc(hp, &h->diag, sizeof(double) * 8 * n_mats))) return cuda_fail(nullptr, e, "cudaMalloc");
   size_t scratch = 0;
   for (Group& g : h->groups) {
     if ((e = dalloc(hp, &g.mat_ids_dev, sizeof(int) * g.mats.size()))) return cuda_fail(nullptr, e, "cudaMalloc");
@@ -256,7 +270,7 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
   if (cfg->variant == NORMPRE_MUON &&
       (e = dalloc(hp, &h->muon_part, sizeof(double) * kMuonBlocks * n_mats)))
     return cuda_fail(nullptr, e, "cudaMalloc");
-  if (cfg->variant != NORMPRE_L) {
+  if (uses_ns(cfg->variant)) {
     std::vector<NSGroupSpec> specs;
     for (Group& g : h->groups) specs.push_back(NSGroupSpec{static_cast<int>(g.mats.size()), g.rows, g.cols});
     h->ns.reset(new NSPlan());
@@ -267,8 +281,20 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
       g.sk.batch = static_cast<int>(g.mats.size());
       g.sk.rows = g.rows; g.sk.cols = g.cols; g.sk.w_dtype = g.w_dtype;
       g.sk.ld = round_up(g.cols, 8);
-      e = sketch_group_alloc(g.sk, cfg->rank, cfg->oversample, h->allocs);
+      const bool exact = cfg->variant == NORMPRE_L_EXACT;
+      e = sketch_group_alloc(g.sk, cfg->rank, exact ? 0 : cfg->oversample, h->allocs);
       if (e != cudaSuccess) return cuda_fail(nullptr, e, "sketch workspace");
+      if (exact) {
+        std::string why;
+        e = exact_group_alloc(g.sk, h->allocs, &why);
+        if (e == cudaErrorNotSupported) {
+          for (Group& gg : h->groups) exact_group_free(gg.sk);
+          for (void* p : h->allocs) cudaFree(p);
+          h->allocs.clear();
+          return fail(nullptr, NORMPRE_ERR_UNAVAILABLE, "NORMPRE_L_EXACT: " + why);
+        }
+        if (e != cudaSuccess) return cuda_fail(nullptr, e, "exact eigensolver workspace");
+      }
     }
     if (h->groups.size() > 1) {
       for (size_t gi = 0; gi < h->groups.size(); ++gi) {
@@ -308,7 +334,11 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
   cudaError_t e = cudaMemsetAsync(h->count, 0, sizeof(int) * h->n_mats, s);
   if (e) return cuda_fail(h, e, "cudaMemsetAsync");
   const bool is_muon = (c.variant == NORMPRE_MUON);
-  const bool is_g = (c.variant == NORMPRE_G) || is_muon;   // Newton-Schulz preconditioning
+  const bool is_g = uses_ns(c.variant);                     // Newton-Schulz preconditioning
+  const bool exact = (c.variant == NORMPRE_L_EXACT);
+  const bool diag_on = c.diagnostics != 0;
+  if ((diag_on || exact) && (e = cudaMemsetAsync(h->diag, 0, sizeof(double) * 8 * h->n_mats, s)))
+    return cuda_fail(h, e, "cudaMemsetAsync");
   const bool psi_bf16 = is_g && c.precision == NORMPRE_PREC_BF16;
   // NormPre-L: each group's sketch pipeline runs on its own side stream, from
   // the end of the group's normalization (joined back into `s` at the end),
@@ -442,6 +472,19 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
       a.lr = lr; a.wd = c.weight_decay; a.target = c.target_rms;
       if ((e = launch_apply_g(a, s))) return cuda_fail(h, e, "apply launch");
       ++n_apply;
+      if (diag_on) {
+        // descent alignment: <G, T> with T = the Newton-Schulz output
+        DiagLaunch d;
+        d.n = a.n; d.rows = g.rows; d.cols = g.cols;
+        d.g_dtype = g.g_dtype; d.t_dtype = a.t_dtype; d.t_ld = a.t_ld;
+        for (int i = 0; i < a.n; ++i) {
+          d.G[i] = G[a.mat_id[i]];
+          d.T[i] = a.T[i];
+          d.diag[i] = h->diag + 8 * static_cast<int64_t>(a.mat_id[i]);
+        }
+        if ((e = launch_diag_gt(d, s))) return cuda_fail(h, e, "diagnostics launch");
+        ++n_apply;
+      }
     }
     h->prof.end(kProfApplyG, s, n_apply);
     if ((e = hk.after_update(ui, s))) return cuda_fail(h, e, "copy out");
@@ -470,7 +513,16 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
       const int gi = u.g;
       Group& g = h->groups[gi];
       std::vector<void*> wp;
-      for (int b = u.b0; b < u.b1; ++b) wp.push_back(W[g.mats[b]]);
+      std::vector<const void*> gp;
+      for (int b = u.b0; b < u.b1; ++b) {
+        wp.push_back(W[g.mats[b]]);
+        gp.push_back(G[g.mats[b]]);
+      }
+      p.exact = exact;
+      p.mat_ids_host = g.mats.data() + u.b0;
+      p.diag = (diag_on || exact) ? h->diag : nullptr;
+      p.G = diag_on ? gp.data() : nullptr;
+      p.g_dtype = g.g_dtype;
       SketchGroup part;
       const bool whole = u.b0 == 0 && u.b1 == static_cast<int>(g.mats.size());
       if (!whole && (e = sketch_group_slice(g.sk, u.b0, u.b1, &part))) return cuda_fail(h, e, "sketch slice");
@@ -672,7 +724,7 @@ int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* row
   if (mat < 0 || mat >= h->n_mats) return fail(hh, NORMPRE_ERR_ARG, "bad matrix index");
   if (!h->stepped) return fail(hh, NORMPRE_ERR_ARG, "no step has run yet");
   const MatInfo& m = h->mats[mat];
-  const bool is_g = h->cfg.variant != NORMPRE_L;
+  const bool is_g = uses_ns(h->cfg.variant);
   const bool rows_active = h->last_k == 0;
   const int64_t m_a = rows_active ? m.rows : m.cols, n_a = rows_active ? m.cols : m.rows;
   int64_t r = 0, c = 0;
@@ -689,6 +741,8 @@ int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* row
       break;
     case NORMPRE_BUF_Q: case NORMPRE_BUF_RITZ: case NORMPRE_BUF_Z: case NORMPRE_BUF_OMEGA: {
       if (is_g) return fail(hh, NORMPRE_ERR_ARG, "sketch buffers exist only for NormPre-L");
+      if (what == NORMPRE_BUF_OMEGA && h->cfg.variant == NORMPRE_L_EXACT)
+        return fail(hh, NORMPRE_ERR_ARG, "NORMPRE_L_EXACT draws no sketch matrix");
       const SketchGroup& sk = h->groups[m.group].sk;
       const int64_t l = rows_active ? sk.ell_rows : sk.ell_cols;
       if (what == NORMPRE_BUF_Q) { r = m_a; c = l; }
@@ -698,6 +752,13 @@ int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* row
       break;
     }
     case NORMPRE_BUF_STATS:
+      r = 1; c = 8;
+      break;
+    case NORMPRE_BUF_EIGS:
+      if (h->cfg.variant != NORMPRE_L_EXACT) return fail(hh, NORMPRE_ERR_ARG, "all eigenvalues exist only for NORMPRE_L_EXACT");
+      r = 1; c = m_a;
+      break;
+    case NORMPRE_BUF_DIAG:
       r = 1; c = 8;
       break;
     default:
@@ -723,7 +784,24 @@ int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capaci
   if (e) return cuda_fail(h, e, "cudaDeviceSynchronize");
   const MatInfo& m = h->mats[mat];
   const Group& g = h->groups[m.group];
-  const bool is_g = h->cfg.variant != NORMPRE_L;
+  const bool is_g = uses_ns(h->cfg.variant);
+  if (what == NORMPRE_BUF_DIAG) {
+    // fp64 sums on the device -> [E_top, E_remain, E_sub, E_global, cos, ||G||, ||T||, <G, T>]
+    double d[8];
+    e = cudaMemcpy(d, h->diag + 8 * static_cast<int64_t>(mat), sizeof(d), cudaMemcpyDeviceToHost);
+    if (e) return cuda_fail(h, e, "cudaMemcpy");
+    const float nan = std::numeric_limits<float>::quiet_NaN();
+    float out[8];
+    const bool ex = h->cfg.variant == NORMPRE_L_EXACT, al = h->cfg.diagnostics != 0;
+    for (int i = 0; i < 4; ++i) out[i] = ex ? static_cast<float>(d[i]) : nan;
+    const double gn = std::sqrt(d[5]), tn = std::sqrt(d[6]);
+    out[4] = al ? ((gn > 0 && tn > 0) ? static_cast<float>(d[4] / (gn * tn)) : 0.f) : nan;
+    out[5] = al ? static_cast<float>(gn) : nan;
+    out[6] = al ? static_cast<float>(tn) : nan;
+    out[7] = al ? static_cast<float>(d[4]) : nan;
+    std::memcpy(dst, out, sizeof(out));
+    return NORMPRE_OK;
+  }
   const void* src = nullptr;
   int64_t src_ld = c;
   if (what == NORMPRE_BUF_PSI || what == NORMPRE_BUF_T) {
@@ -746,6 +824,7 @@ int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capaci
     if (what == NORMPRE_BUF_OMEGA) src = sk.omega + m.slot * vbs;
     if (what == NORMPRE_BUF_RITZ) src = sk.ritz + m.slot * sk.lmax;
     if (what == NORMPRE_BUF_Z) src = sk.zvec + m.slot * sq;
+    if (what == NORMPRE_BUF_EIGS) src = sk.eig_all + m.slot * std::max(sk.rows, sk.cols);
   }
   e = cudaMemcpy2D(dst, c * el, src, src_ld * el, c * el, r, cudaMemcpyDeviceToHost);
   if (e) return cuda_fail(h, e, "cudaMemcpy2D");

@@ -1021,11 +1021,26 @@ struct LApplyArgs {
   int64_t rows, cols;
   int l;
   float lr, wd, target;
+  // DIAG: the step's gradients and, per matrix, where <G, T>, ||G||^2 and
+  // ||T||^2 accumulate (fp64 atomics: diagnostics, not bitwise reproducible)
+  const void* G[kMaxBatch];
+  int g_dtype;
+  double* diag[kMaxBatch];
 };
-template <typename TW, bool VEC>
+template <typename TW, bool VEC, bool DIAG>
 __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyArgs a) {
   __shared__ __align__(16) float Ls[kLmax][64 + 4];   // [p][row]
   __shared__ __align__(16) float Rs[kLmax][64 + 4];   // [p][col]
+  double dgt = 0, dgg = 0, dtt = 0;
+  auto diag_add = [&](int64_t idx, float t) {
+    if (DIAG) {
+      const float g = a.g_dtype ? to_f32(static_cast<const bf16*>(a.G[blockIdx.z])[idx])
+                                : static_cast<const float*>(a.G[blockIdx.z])[idx];
+      dgt += static_cast<double>(g) * t;
+      dgg += static_cast<double>(g) * g;
+      dtt += static_cast<double>(t) * t;
+    }
+  };
   const int b = blockIdx.z;
   const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
   const int64_t r0 = static_cast<int64_t>(blockIdx.y) * 64, c0 = static_cast<int64_t>(blockIdx.x) * 64;
@@ -1072,7 +1087,10 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
         w[0] = bf16lo(wv.x); w[1] = bf16hi(wv.x); w[2] = bf16lo(wv.y); w[3] = bf16hi(wv.y);
       }
 #pragma unroll
-      for (int c = 0; c < 4; ++c) w[c] = fmaf(cw, w[c], ct * (ps[c] + acc[r][c]));
+      for (int c = 0; c < 4; ++c) {
+        w[c] = fmaf(cw, w[c], ct * (ps[c] + acc[r][c]));
+        diag_add(i * a.cols + j0 + c, ps[c] + acc[r][c]);
+      }
       if (std::is_same<TW, float>::value) {
         *reinterpret_cast<float4*>(reinterpret_cast<float*>(W) + i * a.cols + j0) = make_float4(w[0], w[1], w[2], w[3]);
       } else {
@@ -1087,7 +1105,19 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
         const float t = psi[i * a.psi_ld + j] + acc[r][c];
         const float w = to_f32(W[i * a.cols + j]);
         W[i * a.cols + j] = from_f32<TW>(fmaf(cw, w, ct * t));
+        diag_add(i * a.cols + j, t);
       }
+    }
+  }
+  if (DIAG) {
+    __shared__ double red[32];
+    dgt = block_sum(dgt, red);
+    dgg = block_sum(dgg, red);
+    dtt = block_sum(dtt, red);
+    if (threadIdx.x == 0) {
+      atomicAdd(a.diag[b] + 4, dgt);
+      atomicAdd(a.diag[b] + 5, dgg);
+      atomicAdd(a.diag[b] + 6, dtt);
     }
   }
 }
@@ -1196,6 +1226,7 @@ cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup
   s.zvec = g.zvec + b0 * sq;
   s.ritz = g.ritz + static_cast<int64_t>(b0) * g.lmax;
   s.stats = g.stats + static_cast<int64_t>(b0) * 8;
+  if (g.eig_all) s.eig_all = g.eig_all + b0 * std::max(g.rows, g.cols);
   if (g.tc) {
     const uint64_t dims[3] = {static_cast<uint64_t>(g.cols), static_cast<uint64_t>(g.rows),
                               static_cast<uint64_t>(s.batch)};
@@ -1227,8 +1258,8 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   cudaError_t e;
 #define NP_CHECK() do { e = cudaGetLastError(); if (e != cudaSuccess) return e; } while (0)
 
-  // Omega [n_a x l]
-  {
+  // Omega [n_a x l] (the sketch only)
+  if (!p.exact) {
     OmegaArgs o;
     o.omega = g.omega; o.bstride = vbs; o.n_a = n_a; o.l = l;
     o.key0 = static_cast<uint32_t>(p.seed); o.key1 = static_cast<uint32_t>(p.seed >> 32);
@@ -1316,52 +1347,60 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     k_gram_part<<<dim3(ga.nsplit, B), 256, 0, s>>>(ga);
     return ga.nsplit;
   };
-  // Y0 = Psi_a Omega; p times Y <- Psi_a (Psi_a^T Y)
-  if ((e = contract(ta, g.omega, g.y0))) return e;
-  float* ycur = g.y0;
-  for (int it = 0; it < p.power_iters; ++it) {
-    if ((e = contract(tb, ycur, g.zt))) return e;
-    if ((e = contract(ta, g.zt, g.y))) return e;
-    ycur = g.y;
-  }
-  // Q = qr(Y): three CholeskyQR passes (a pass shifts when its Gram matrix is
-  // numerically singular): y -> q -> zt -> q
-  prof->begin(kProfQR, s);
-  {
-    const float* src = ycur;
-    for (int pass = 0; pass < 3; ++pass) {
-      const int ns = gram(src, m_a);
-      NP_CHECK();
-      float* dst = (pass == 1) ? g.zt : g.q;
-      CholQRArgs cq;
-      cq.part = g.part; cq.part_bs = static_cast<int64_t>(g.max_part) * sq; cq.nsplit = ns;
-      cq.y = src; cq.q = dst; cq.v_bs = vbs;
-      cq.n = m_a; cq.l = l; cq.flags = flags;
-      if ((e = launch_cholqr(cq, B, lp, s))) return e;
-      src = dst;
+  if (p.exact) {
+    // exact eigenpairs of Gamma = Psi_a Psi_a^T (exact.cu), then B^T = Psi_a^T Q
+    prof->begin(kProfEig, s);
+    if ((e = exact_eigs(g, p, l, p.mat_ids_host, count, p.diag, flags, s))) return e;
+    prof->end(kProfEig, s, 3 * B);
+    if ((e = contract(tb, g.q, g.bt))) return e;
+  } else {
+    // Y0 = Psi_a Omega; p times Y <- Psi_a (Psi_a^T Y)
+    if ((e = contract(ta, g.omega, g.y0))) return e;
+    float* ycur = g.y0;
+    for (int it = 0; it < p.power_iters; ++it) {
+      if ((e = contract(tb, ycur, g.zt))) return e;
+      if ((e = contract(ta, g.zt, g.y))) return e;
+      ycur = g.y;
     }
-  }
-  prof->end(kProfQR, s, 6);
-  // B^T = Psi_a^T Q  [n_a x l];  Gamma_Q = B B^T
-  if ((e = contract(tb, g.q, g.bt))) return e;
-  prof->begin(kProfEig, s);
-  {
-    const int ns = gram(g.bt, n_a);
-    NP_CHECK();
-    EigArgs ea;
-    ea.part = g.part; ea.part_bs = static_cast<int64_t>(g.max_part) * sq; ea.nsplit = ns;
-    ea.ritz = g.ritz; ea.ritz_bs = g.lmax;
-    ea.z = g.zvec; ea.z_bs = sq;
-    ea.kmat = g.kmat; ea.k_bs = sq;
-    ea.stats = g.stats; ea.stats_bs = 8;
-    ea.count = count; ea.mat_id = mat_ids;
-    ea.l = l; ea.rank = p.rank; ea.k_orient = p.k;
-    ea.m_a = m_a; ea.n_a = n_a;
-    ea.max_sweeps = 30;
-    ea.flags = flags;
-    const int jthreads = static_cast<int>(std::min<int64_t>(1024, round_up(static_cast<int64_t>((l + 1) / 2) * l, 32)));
-    k_jacobi<<<B, std::max(jthreads, 32), small_smem, s>>>(ea);
-    NP_CHECK();
+    // Q = qr(Y): three CholeskyQR passes (a pass shifts when its Gram matrix is
+    // numerically singular): y -> q -> zt -> q
+    prof->begin(kProfQR, s);
+    {
+      const float* src = ycur;
+      for (int pass = 0; pass < 3; ++pass) {
+        const int ns = gram(src, m_a);
+        NP_CHECK();
+        float* dst = (pass == 1) ? g.zt : g.q;
+        CholQRArgs cq;
+        cq.part = g.part; cq.part_bs = static_cast<int64_t>(g.max_part) * sq; cq.nsplit = ns;
+        cq.y = src; cq.q = dst; cq.v_bs = vbs;
+        cq.n = m_a; cq.l = l; cq.flags = flags;
+        if ((e = launch_cholqr(cq, B, lp, s))) return e;
+        src = dst;
+      }
+    }
+    prof->end(kProfQR, s, 6);
+    // B^T = Psi_a^T Q  [n_a x l];  Gamma_Q = B B^T
+    if ((e = contract(tb, g.q, g.bt))) return e;
+    prof->begin(kProfEig, s);
+    {
+      const int ns = gram(g.bt, n_a);
+      NP_CHECK();
+      EigArgs ea;
+      ea.part = g.part; ea.part_bs = static_cast<int64_t>(g.max_part) * sq; ea.nsplit = ns;
+      ea.ritz = g.ritz; ea.ritz_bs = g.lmax;
+      ea.z = g.zvec; ea.z_bs = sq;
+      ea.kmat = g.kmat; ea.k_bs = sq;
+      ea.stats = g.stats; ea.stats_bs = 8;
+      ea.count = count; ea.mat_id = mat_ids;
+      ea.l = l; ea.rank = p.rank; ea.k_orient = p.k;
+      ea.m_a = m_a; ea.n_a = n_a;
+      ea.max_sweeps = 30;
+      ea.flags = flags;
+      const int jthreads = static_cast<int>(std::min<int64_t>(1024, round_up(static_cast<int64_t>((l + 1) / 2) * l, 32)));
+      k_jacobi<<<B, std::max(jthreads, 32), small_smem, s>>>(ea);
+      NP_CHECK();
+    }
   }
   // QK = Q K  [m_a x l]
   {
@@ -1388,14 +1427,23 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     for (int i = 0; i < nb; ++i) la.W[i] = W[c0 + i];
     la.rows = g.rows; la.cols = g.cols; la.l = l;
     la.lr = p.lr; la.wd = p.wd; la.target = p.target;
-    const dim3 grid(static_cast<unsigned>(cdiv(g.cols, 64)), static_cast<unsigned>(cdiv(g.rows, 64)), nb);
-    if (g.w_dtype == 0) {
-      if (vec) k_apply_l<float, true><<<grid, 256, 0, s>>>(la);
-      else k_apply_l<float, false><<<grid, 256, 0, s>>>(la);
-    } else {
-      if (vec) k_apply_l<bf16, true><<<grid, 256, 0, s>>>(la);
-      else k_apply_l<bf16, false><<<grid, 256, 0, s>>>(la);
+    const bool diag = p.diag && p.G;
+    la.g_dtype = p.g_dtype;
+    for (int i = 0; i < nb; ++i) {
+      la.G[i] = diag ? p.G[c0 + i] : nullptr;
+      la.diag[i] = diag ? p.diag + 8 * static_cast<int64_t>(p.mat_ids_host[c0 + i]) : nullptr;
     }
+    const dim3 grid(static_cast<unsigned>(cdiv(g.cols, 64)), static_cast<unsigned>(cdiv(g.rows, 64)), nb);
+#define NP_APPLY_L(TWT, V) \
+    (diag ? k_apply_l<TWT, V, true><<<grid, 256, 0, s>>>(la) : k_apply_l<TWT, V, false><<<grid, 256, 0, s>>>(la))
+    if (g.w_dtype == 0) {
+      if (vec) NP_APPLY_L(float, true);
+      else NP_APPLY_L(float, false);
+    } else {
+      if (vec) NP_APPLY_L(bf16, true);
+      else NP_APPLY_L(bf16, false);
+    }
+#undef NP_APPLY_L
     NP_CHECK();
   }
   prof->end(kProfApplyL, s, n_apply);

@@ -15,16 +15,18 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libnormpre.so")
 
 # enums (mirror include/normpre.h)
-NORMPRE_G, NORMPRE_L, NORMPRE_MUON = 0, 1, 2
+NORMPRE_G, NORMPRE_L, NORMPRE_MUON, NORMPRE_L_EXACT = 0, 1, 2, 3
 NORMPRE_F32, NORMPRE_BF16 = 0, 1
 NORMPRE_PREC_BF16, NORMPRE_PREC_F32 = 0, 1
 (NORMPRE_OK, NORMPRE_ERR_ARG, NORMPRE_ERR_SHAPE, NORMPRE_ERR_DTYPE, NORMPRE_ERR_ALIGN,
- NORMPRE_ERR_CUDA, NORMPRE_ERR_NONFINITE, NORMPRE_ERR_NUMERIC, NORMPRE_ERR_TIMEOUT) = range(9)
+ NORMPRE_ERR_CUDA, NORMPRE_ERR_NONFINITE, NORMPRE_ERR_NUMERIC, NORMPRE_ERR_TIMEOUT,
+ NORMPRE_ERR_UNAVAILABLE) = range(10)
 (NORMPRE_BUF_PSI, NORMPRE_BUF_T, NORMPRE_BUF_Q, NORMPRE_BUF_RITZ, NORMPRE_BUF_Z,
- NORMPRE_BUF_OMEGA, NORMPRE_BUF_STATS) = range(7)
+ NORMPRE_BUF_OMEGA, NORMPRE_BUF_STATS, NORMPRE_BUF_EIGS, NORMPRE_BUF_DIAG) = range(9)
 
 STATUS_NAMES = {0: "OK", 1: "ERR_ARG", 2: "ERR_SHAPE", 3: "ERR_DTYPE", 4: "ERR_ALIGN",
-                5: "ERR_CUDA", 6: "ERR_NONFINITE", 7: "ERR_NUMERIC", 8: "ERR_TIMEOUT"}
+                5: "ERR_CUDA", 6: "ERR_NONFINITE", 7: "ERR_NUMERIC", 8: "ERR_TIMEOUT",
+                9: "ERR_UNAVAILABLE"}
 
 
 class normpre_config(ctypes.Structure):
@@ -43,6 +45,7 @@ class normpre_config(ctypes.Structure):
         ("precision", ctypes.c_int),
         ("orientation", ctypes.c_int),
         ("tangent", ctypes.c_int),
+        ("diagnostics", ctypes.c_int),
     ]
 
 

@@ -48,6 +48,7 @@ def test_default_config_is_the_papers(lib):
     assert (cfg.rank, cfg.oversample, cfg.power_iters) == (32, 8, 1)
     assert cfg.precision == lib.NORMPRE_PREC_BF16 and cfg.orientation == 0
     assert cfg.tangent == 0      # the paper's relaxed tangent
+    assert cfg.diagnostics == 0
 
 
 def test_host_side_argument_errors(lib):
@@ -78,10 +79,23 @@ def test_host_side_argument_errors(lib):
     with pytest.raises(C.NormPreError) as e:
         C.normpre_init(bad, [(4, 5)], [0], [0])
     assert "tangent" in C.normpre_last_error()
-    bad = C.normpre_default_config(variant=3)
+    bad = C.normpre_default_config(variant=4)
     with pytest.raises(C.NormPreError) as e:
         C.normpre_init(bad, [(4, 5)], [0], [0])
     assert e.value.status == C.NORMPRE_ERR_ARG
+    bad = C.normpre_default_config(diagnostics=2)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    assert "diagnostics" in C.normpre_last_error()
+    # exact eigenspace extraction: rank budget and the Gamma workspace limit
+    bad = C.normpre_default_config(variant=C.NORMPRE_L_EXACT, rank=65)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    assert e.value.status == C.NORMPRE_ERR_ARG
+    ex = C.normpre_default_config(variant=C.NORMPRE_L_EXACT)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(ex, [(16, 20000)], [0], [0])
+    assert e.value.status == C.NORMPRE_ERR_SHAPE
     # stand-alone Newton-Schulz: argument checks come before any device work
     with pytest.raises(C.NormPreError) as e:
         C.normpre_newton_schulz(cfg, 1, 4, 4, 0, 0)

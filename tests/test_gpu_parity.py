@@ -49,7 +49,8 @@ def _run(cfgset: S.ParamSetConfig, t: int, variant: str, precision: int, indices
     else:
         mats = S.make_param_set(cfgset, workers=min(16, os.cpu_count() or 1))
     W, G, M = to_device(mats, cfgset.g_dtype, cfgset.w_dtype)
-    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON}[variant], precision=precision,
+    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON,
+                       "L_exact": C.NORMPRE_L_EXACT}[variant], precision=precision,
               rank=cfgset.rank, oversample=cfgset.oversample, power_iters=cfgset.power_iters,
               seed=1234)
     kw.update(extra or {})
@@ -448,3 +449,66 @@ def test_host_entry_point_in_units(variant):
         for i in range(len(shapes)):
             assert torch.equal(Wh[i], W[i].cpu()), (t, i)
             assert torch.equal(Mh[i], M[i].cpu()), (t, i)
+
+
+
+# --------------------------------------------------------------------------
+# NormPre-L with exact eigenspace extraction (Sec. 3.2, App. B)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("cfgset", [SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("t", [0, 1])
+def test_l_exact(cfgset, t):
+    """Gamma = Psi_a Psi_a^T, all its eigenvalues, the selected eigenvectors,
+    the updated weights and the spectral energies, against the oracle."""
+    from paper_2609_36692_gb300 import normpre as C
+    opt, mats, W1, _ = _run(cfgset, t, "L_exact", precision=1)
+    n_sel = 0
+    for i in range(cfgset.n_mats):
+        ref = _oracle(mats, i, t, "L_exact", cfgset)
+        ex = ref["exact"]
+        lam = ex["lam"]
+        eig = opt.read(i, C.NORMPRE_BUF_EIGS)[0].astype(np.float64)
+        assert eig.shape == lam.shape, (cfgset.name, i)
+        # fp32 Gamma and eigensolver: errors of a few ulp of lambda_max
+        assert np.max(np.abs(eig - lam)) <= 2e-5 * max(1.0, lam[0]), (cfgset.name, i)
+        st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
+        if ritz_gaps_ok(lam, cfgset.rank):
+            nc = int(st[3])
+            assert nc == ex["n_active"], (cfgset.name, i, nc, ex["n_active"])
+            Q = opt.read(i, C.NORMPRE_BUF_Q)
+            assert principal_sine(Q[:, :nc], ex["U_C"]) <= 1e-3, (cfgset.name, i)
+            n_sel += nc
+        dW = W1[i].astype(np.float64) - mats[i]["W"]
+        assert rel_fro(dW, ref["W"] - mats[i]["W"]) <= 2e-3, (cfgset.name, i)
+        d = opt.read(i, C.NORMPRE_BUF_DIAG)[0].astype(np.float64)
+        e = O.spectral_energies(lam, cfgset.rank)
+        scale = max(1.0, e["E_global"])
+        for j, key in enumerate(("E_top", "E_remain", "E_sub", "E_global")):
+            assert abs(d[j] - e[key]) <= 1e-3 * scale, (cfgset.name, i, key, d[j], e[key])
+        assert np.all(np.isnan(d[4:])), "alignment is off without cfg.diagnostics"
+    assert n_sel > 0 or cfgset is RAGGED
+
+
+# --------------------------------------------------------------------------
+# Diagnostics: descent alignment (App. E)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("variant", ["G", "L", "muon"])
+@pytest.mark.parametrize("t", [0, 1])
+def test_descent_alignment(variant, t):
+    from paper_2609_36692_gb300 import normpre as C
+    cs = SMALL
+    opt, mats, W1, _ = _run(cs, t, variant, precision=1, extra={"diagnostics": 1})
+    for i in range(cs.n_mats):
+        m = mats[i]
+        if variant == "muon":
+            T_stored = O.muon_step(m["W"], m["G"], m["M"], f32(LR), oracle_config("G"))["T"]
+        else:
+            ref = _oracle(mats, i, t, variant, cs)
+            T_stored = _stored(ref["T"], ref["k"])
+        want = O.descent_alignment(m["G"], T_stored)
+        d = opt.read(i, C.NORMPRE_BUF_DIAG)[0].astype(np.float64)
+        assert abs(d[4] - want) <= 2e-3, (variant, i, d[4], want)
+        assert abs(d[5] - np.linalg.norm(m["G"])) <= 1e-5 * np.linalg.norm(m["G"]), (variant, i)
+        assert abs(d[6] - np.linalg.norm(T_stored)) <= 2e-3 * np.linalg.norm(T_stored), (variant, i)
+        assert np.all(np.isnan(d[:4])), "spectral energies exist only for NORMPRE_L_EXACT"
+        assert -1.0 <= d[4] <= 1.0
