@@ -114,3 +114,16 @@ def test_null_handle_calls(lib):
     assert so.normpre_step(None, 0, 0.1, None, None, None, None) == C.NORMPRE_ERR_ARG
     assert so.normpre_sync_status(None, None) == C.NORMPRE_ERR_ARG
     so.normpre_free(None)
+
+
+def test_torch_optimizer_validates_parameters():
+    """NormPreOptimizer takes 2-D CUDA matrices only; the checks run on the
+    host before any device work."""
+    torch = pytest.importorskip("torch")
+    from paper_2609_36692_gb300.optim import NormPreOptimizer
+    with pytest.raises(ValueError, match="2-D"):
+        NormPreOptimizer([torch.nn.Parameter(torch.zeros(3))])
+    with pytest.raises(ValueError, match="CUDA"):
+        NormPreOptimizer([torch.nn.Parameter(torch.zeros(3, 4))])
+    with pytest.raises(ValueError, match="variant"):
+        NormPreOptimizer([torch.nn.Parameter(torch.zeros(3, 4))], variant="X")
