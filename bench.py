@@ -41,6 +41,8 @@ LR = 0.02
 # Traffic of one launch of the dominant kernel class from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum), per workload; None until a
 # capture of the current kernel exists (profiles/ keeps the summaries).
+FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # 80.5 TFLOP/s, for the ALU-bound k_gamma
+
 NCU_TRAFFIC_PER_LAUNCH = {
     "gpt2_small_G": 208.1e6,   # mean of 15 launches: Gram, poly and update of five NS iterations
     "gpt2_small_L": 108.0e6,   # mean of six k_contract_tc launches (both operand orientations)
@@ -92,7 +94,7 @@ def ns_executed_flops(cfg: S.ParamSetConfig, steps: int) -> float:
 def bytes_per_elt(cfg: S.ParamSetConfig, variant: str):
     g = 2 if cfg.g_dtype == "bf16" else 4
     w = 2 if cfg.w_dtype == "bf16" else 4
-    psi = 2 if variant == "G" else 4
+    psi = 2 if variant == "G" else 4        # bf16 Newton-Schulz input, fp32 for the L variants
     normalize = g + 4 + 4 + w + psi          # read G, M, W; write M, Psi
     apply = psi + 2 * w                      # read T (or Psi), read/write W
     return normalize, apply
@@ -161,7 +163,7 @@ def oracle_sample(cfg: S.ParamSetConfig, variant: str, seconds_budget: float = 2
     shapes = {}
     for i, m in enumerate(cfg.matrices):
         shapes.setdefault((m.rows, m.cols), []).append(i)
-    oc = O.OracleConfig(variant=variant, rank=cfg.rank, oversample=cfg.oversample,
+    oc = O.OracleConfig(variant=variant, rank=cfg.rank, oversample=0 if variant == "L_exact" else cfg.oversample,
                         power_iters=cfg.power_iters, seed=1234)
     total_ms = 0.0
     sampled = []
@@ -229,8 +231,9 @@ def run_ours(args, cfg, variant, rank, world):
     G = [torch.from_numpy(m["G"]).to(tdt[cfg.g_dtype]).cuda() for m in mats]
     M = [torch.from_numpy(m["M"]).cuda() for m in mats]
     prec = C.NORMPRE_PREC_BF16 if variant == "G" else C.NORMPRE_PREC_F32
+    vcode = {"G": C.NORMPRE_G, "L": C.NORMPRE_L, "L_exact": C.NORMPRE_L_EXACT}[variant]
     opt = NormPre([(m.rows, m.cols) for m in cfg.matrices], [cfg.w_dtype] * cfg.n_mats,
-                  [cfg.g_dtype] * cfg.n_mats, variant=C.NORMPRE_G if variant == "G" else C.NORMPRE_L,
+                  [cfg.g_dtype] * cfg.n_mats, variant=vcode,
                   precision=prec, rank=cfg.rank, oversample=cfg.oversample,
                   power_iters=cfg.power_iters, ns_steps=cfg.ns_steps, seed=1234)
     h = opt.handle
@@ -324,6 +327,22 @@ def run_ours(args, cfg, variant, rank, world):
                 "achieved_executed": fl_exec / (ns_ms * 1e-3) / 1e12,
                 "frac_executed": fl_exec / (ns_ms * 1e-3) / 1e12 / peak,
                 "traffic": NCU_TRAFFIC_PER_LAUNCH.get(cfg.name)}
+    elif variant == "L_exact":
+        # k_gamma: Gamma = Psi_a Psi_a^T on the fp32 FMA pipes (both triangles,
+        # 2 m_a^2 n_a flops per matrix); the dense eigensolver is a library call
+        gam_ms = prof["gamma"][0] / args.steps
+        gam_launches = prof["gamma"][1] / args.steps
+        k_even = sum(2.0 * m.rows * m.rows * m.cols for m in cfg.matrices)
+        k_odd = sum(2.0 * m.cols * m.cols * m.rows for m in cfg.matrices)
+        fl = (k_even + k_odd) / 2.0          # row- and column-active steps alternate
+        achieved = fl / (gam_ms * 1e-3) / 1e12
+        fp32_peak = FP32_FMA_TFLOPS
+        roof = {"bound": "alu", "kernel": "k_gamma (Gamma = Psi_a Psi_a^T, fp32 FMA)",
+                "achieved": achieved, "peak": fp32_peak, "unit": "TFLOP/s", "frac": achieved / fp32_peak,
+                "peak_source": "nominal fp32 FMA rate: 152 SMs x 128 lanes x 2 flops x 2.07 GHz",
+                "flops_per_launch": fl / gam_launches, "ms_per_launch": gam_ms / gam_launches,
+                "syevd_ms_per_step": prof["syevd"][0] / args.steps,
+                "traffic": None}
     else:
         con_ms = prof["contract"][0] / args.steps
         con_launches = prof["contract"][1] / args.steps
@@ -399,7 +418,7 @@ def run_ours(args, cfg, variant, rank, world):
                 "dtype": "bf16" if variant == "G" else "f32", "data": "synthetic",
                 "config": {"workload": cfg.name, "variant": variant, "n_mats": cfg.n_mats,
                            "elements": n_el, "ns_steps": cfg.ns_steps if variant == "G" else None,
-                           "rank": cfg.rank if variant == "L" else None,
+                           "rank": cfg.rank if variant in ("L", "L_exact") else None,
                            "l2": "inputs larger than L2 (W, G, M = %.0f MB)" % (h2d / 1e6),
                            "parallelism": "replicas" if world > 1 else "single"},
                 "e2e": {"value": e2e_ms / world, "unit": "ms", "h2d_bytes_per_step": h2d,
@@ -424,7 +443,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(S.CONFIGS))
-    ap.add_argument("--variant", default=None, choices=[None, "G", "L"])
+    ap.add_argument("--variant", default=None, choices=[None, "G", "L", "L_exact"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-muon", action="store_true", help="skip timing the Muon comparison step")
     args = ap.parse_args()

@@ -241,7 +241,9 @@ enum normpre_profile_class {
   NORMPRE_PROF_EIG = 8,        /* Rayleigh-Ritz Gram, Jacobi eigensolver, Q K */
   NORMPRE_PROF_APPLY_L = 9,    /* NormPre-L projector apply + weight update */
   NORMPRE_PROF_PRESCALE = 10,  /* Newton-Schulz input scale 1/(sqrt(m') + eps) */
-  NORMPRE_PROF_CLASSES = 11
+  NORMPRE_PROF_GAMMA = 11,     /* NORMPRE_L_EXACT: Gamma = Psi_a Psi_a^T */
+  NORMPRE_PROF_SYEVD = 12,     /* NORMPRE_L_EXACT: dense eigensolver and the selection */
+  NORMPRE_PROF_CLASSES = 13
 };
 
 /*

@@ -266,7 +266,9 @@ void exact_group_free(SketchGroup& g) {
 }
 
 cudaError_t exact_eigs(SketchGroup& g, const SketchParams& p, int l, const int* mat_ids_host, const int* count,
-                       double* diag, int* flags, cudaStream_t s) {
+                       double* diag, int* flags, cudaStream_t s, ProfileHook* prof) {
+  ProfileHook none;
+  if (!prof) prof = &none;
   const CusolverApi& api = cusolver();
   if (!api.ok || !g.solver) return cudaErrorNotSupported;
   const bool rows_active = (p.k == 0);
@@ -284,10 +286,13 @@ cudaError_t exact_eigs(SketchGroup& g, const SketchParams& p, int l, const int* 
     ga.k = n_a;
     ga.gamma = g.gamma;
     const dim3 grid(static_cast<unsigned>(cdiv(m_a, 64)), static_cast<unsigned>(cdiv(m_a, 64)));
+    prof->begin(kProfGamma, s);
     if (rows_active) k_gamma<false><<<grid, 256, 0, s>>>(ga);
     else k_gamma<true><<<grid, 256, 0, s>>>(ga);
     cudaError_t e = cudaGetLastError();
     if (e) return e;
+    prof->end(kProfGamma, s, 1);
+    prof->begin(kProfSyevd, s);
     if (api.syevd(h, CUSOLVER_EIG_MODE_VECTOR, CUBLAS_FILL_MODE_LOWER, static_cast<int>(m_a), g.gamma,
                   static_cast<int>(m_a), g.eig_w, g.eig_work, g.eig_lwork, g.eig_info) != CUSOLVER_STATUS_SUCCESS)
       return cudaErrorUnknown;
@@ -313,6 +318,7 @@ cudaError_t exact_eigs(SketchGroup& g, const SketchParams& p, int l, const int* 
     const int blocks = static_cast<int>(std::min<int64_t>(cdiv(m_a * l, 256), 1024));
     k_exact_select<<<std::max(blocks, 1), 256, 0, s>>>(sa);
     if ((e = cudaGetLastError())) return e;
+    prof->end(kProfSyevd, s, 1);
   }
   return cudaSuccess;
 }

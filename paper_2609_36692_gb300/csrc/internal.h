@@ -24,7 +24,7 @@ inline int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 enum ProfClass {
   kProfNormalize = 0, kProfNsGram = 1, kProfNsPoly = 2, kProfNsUpdate = 3, kProfApplyG = 4,
   kProfOmega = 5, kProfContract = 6, kProfQR = 7, kProfEig = 8, kProfApplyL = 9,
-  kProfPrescale = 10, kProfClasses = 11
+  kProfPrescale = 10, kProfGamma = 11, kProfSyevd = 12, kProfClasses = 13
 };
 
 // Counts kernel launches and, when enabled, brackets launch groups with CUDA
@@ -279,7 +279,7 @@ int exact_available(std::string* why);
 cudaError_t exact_group_alloc(SketchGroup& g, std::vector<void*>& allocs, std::string* why);
 void exact_group_free(SketchGroup& g);
 cudaError_t exact_eigs(SketchGroup& g, const SketchParams& p, int l, const int* mat_ids_host, const int* count,
-                       double* diag, int* flags, cudaStream_t s);
+                       double* diag, int* flags, cudaStream_t s, ProfileHook* prof);
 // Matrices [b0, b1) of a group as a group of their own: the same workspaces
 // from its first matrix on, and tensor maps of Psi over those matrices only.
 cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup* out);

@@ -1349,10 +1349,9 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   };
   if (p.exact) {
     // exact eigenpairs of Gamma = Psi_a Psi_a^T (exact.cu), then B^T = Psi_a^T Q
-    prof->begin(kProfEig, s);
-    if ((e = exact_eigs(g, p, l, p.mat_ids_host, count, p.diag, flags, s))) return e;
-    prof->end(kProfEig, s, 3 * B);
+    if ((e = exact_eigs(g, p, l, p.mat_ids_host, count, p.diag, flags, s, prof))) return e;
     if ((e = contract(tb, g.q, g.bt))) return e;
+    prof->begin(kProfEig, s);   // Q K below
   } else {
     // Y0 = Psi_a Omega; p times Y <- Psi_a (Psi_a^T Y)
     if ((e = contract(ta, g.omega, g.y0))) return e;
@@ -1410,7 +1409,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     k_rowmul<<<dim3(static_cast<unsigned>(cdiv(m_a * l, 256)), B), 256, 0, s>>>(rm);
     NP_CHECK();
   }
-  prof->end(kProfEig, s, 3);
+  prof->end(kProfEig, s, p.exact ? 1 : 3);
   // T_s = Psi + Lm R^T with (Lm, R) = (QK, B^T) row-active or (B^T, QK) column-active,
   // in launches of at most kMaxBatch matrices (W pointers travel as kernel arguments)
   prof->begin(kProfApplyL, s);
