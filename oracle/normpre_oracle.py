@@ -44,6 +44,9 @@ Readings taken where the paper is silent:
   (ties keep the lower index), r' = min(r, l), then C = {i <= r' : lam_i > 1}.
 * Spectral energies (App. E): "nonzero" eigenvalues are those above 1e-6 of
   the largest.
+* "Row+Column/Step" (Table 5b): rows of the row-active tangent momentum
+  normalized, then the columns of the result; preconditioning and the update
+  in the row orientation.
 * Muon baseline (the comparison optimizer of Sec. 4 and App. A): the same
   momentum, the Newton-Schulz iteration applied to the momentum itself (no
   orientation, tangent or normalization step, Sec. 2.1), and the update
@@ -76,7 +79,8 @@ class OracleConfig:
     oversample: int = 8             # o
     power_iters: int = 1            # p
     seed: int = 0                   # Philox key for Omega
-    orientation: int = 0            # 0 alternate (paper), 1 row only, 2 column only
+    orientation: int = 0            # 0 alternate (paper), 1 row only, 2 column only,
+                                    # 3 rows then columns every step (Table 5b "Row+Column/Step")
     tangent: str = "relaxed"        # "relaxed" (paper), "strict" or "none" (Table 5a ablations)
 
 
@@ -160,8 +164,9 @@ def orientation_of(t: int, mode: int = 0) -> int:
     """k_t = t mod 2 (Sec. 3.1, alternating row/column orientation).
 
     mode 1 / 2 fix the orientation to rows / columns (the paper's row-only
-    ablation and its column counterpart)."""
-    if mode == 1:
+    ablation and its column counterpart); mode 3 (both axes every step) works
+    in the row orientation."""
+    if mode in (1, 3):
         return 0
     if mode == 2:
         return 1
@@ -220,6 +225,16 @@ def diag_gram_normalize(X: np.ndarray):
     nz = d > 0
     inv[nz] = 1.0 / d[nz]
     return X * inv[:, None], d
+
+
+def both_axes_normalize(X: np.ndarray):
+    """The "Row+Column/Step" ablation of Table 5b, read as: the rows of the
+    (row-active) tangent momentum normalized as in Eq. 3, then the columns of
+    the result normalized the same way (zero columns stay zero).  Returns
+    (Psi, row norms)."""
+    Psi, d = diag_gram_normalize(X)
+    PsiT, _ = diag_gram_normalize(Psi.T)
+    return PsiT.T, d
 
 
 def newton_schulz(Psi: np.ndarray, steps: int = 5, coef=MUON_QUINTIC, eps: float = 1e-7) -> np.ndarray:
@@ -331,7 +346,10 @@ def normpre_step(W: np.ndarray, G: np.ndarray, M_prev: np.ndarray, t: int, lr: f
     k = orientation_of(t, cfg.orientation)
     Wbar, Mbar = orient(W, k), orient(M, k)
     X = tangent_step(Mbar, Wbar, cfg.tangent)
-    Psi, d = diag_gram_normalize(X)
+    if cfg.orientation == 3:
+        Psi, d = both_axes_normalize(X)
+    else:
+        Psi, d = diag_gram_normalize(X)
     out = {"M": M, "k": k, "X": X, "Psi": Psi, "d": d}
     if cfg.variant == "G":
         T = newton_schulz(Psi, cfg.ns_steps, cfg.ns_coef, cfg.ns_eps)
@@ -405,7 +423,7 @@ def descent_alignment(G: np.ndarray, Phi: np.ndarray) -> float:
 __all__ = [
     "MUON_QUINTIC", "OracleConfig", "philox4x32_10", "philox_uniform", "sketch_omega",
     "momentum_update", "orientation_of", "orient", "relaxed_tangent", "strict_tangent", "tangent_step",
-    "diag_gram_normalize",
+    "diag_gram_normalize", "both_axes_normalize",
     "newton_schulz", "ns_scalar_map", "interaction_sketch", "exact_interaction_eigs",
     "localized_apply", "rms_matched", "weight_update", "normpre_step", "muon_step",
     "spectral_energies", "descent_alignment",

@@ -556,3 +556,44 @@ def test_descent_alignment_identities():
     R = O.rms_matched(T, 1, 0.2)
     assert abs(O.descent_alignment(G, R) - O.descent_alignment(G, T.T)) < 1e-12
     assert O.descent_alignment(G, np.zeros_like(G)) == 0.0
+
+
+# --------------------------------------------------------------------------
+# "Row+Column/Step" orientation ablation (Table 5b), the reading: rows, then columns
+# --------------------------------------------------------------------------
+def test_both_axes_normalize_rank_one_closed_form():
+    """X = a b^T: the rows become sign(a_i) b / ||b||, then every column j is
+    sign(a) sign(b_j) / sqrt(m)."""
+    a = np.array([2.0, -0.5, 3.0, -1.0])
+    b = np.array([0.3, -4.0, 1.5])
+    Psi, _ = O.both_axes_normalize(np.outer(a, b))
+    want = np.outer(np.sign(a), np.sign(b)) / np.sqrt(a.size)
+    assert np.max(np.abs(Psi - want)) < 1e-15
+
+
+def test_both_axes_normalize_fixed_point_and_zero_lines():
+    rng = np.random.default_rng(7)
+    P = np.eye(5)[rng.permutation(5)]
+    D = np.diag(rng.uniform(0.5, 3.0, 5))
+    Psi, _ = O.both_axes_normalize(D @ P)      # rows and columns already one-hot
+    assert np.array_equal(Psi, P)
+    X = rng.standard_normal((6, 9))
+    X[2] = 0.0
+    X[:, 4] = 0.0
+    Psi, _ = O.both_axes_normalize(X)
+    nc = np.linalg.norm(Psi, axis=0)
+    assert np.all(Psi[2] == 0.0) and np.all(Psi[:, 4] == 0.0)
+    assert np.allclose(np.delete(nc, 4), 1.0, atol=1e-14)
+    # ||Psi||_F^2 = number of nonzero columns
+    assert abs(np.sum(Psi ** 2) - 8) < 1e-12
+
+
+def test_orientation_3_step_uses_rows():
+    rng = np.random.default_rng(8)
+    W = rng.standard_normal((5, 7)) * 0.1
+    G = rng.standard_normal((5, 7))
+    M = rng.standard_normal((5, 7))
+    for t in (0, 1, 2):
+        out = O.normpre_step(W, G, M, t, 0.01, O.OracleConfig(variant="G", orientation=3))
+        assert out["k"] == 0
+        assert np.allclose(np.linalg.norm(out["Psi"], axis=0), 1.0)
