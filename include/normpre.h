@@ -102,7 +102,10 @@ typedef struct normpre_config {
   int power_iters;        /* p = 1 */
   uint64_t seed;          /* Philox4x32-10 key of the sketch matrix Omega */
   int precision;          /* normpre_precision */
-  int orientation;        /* 0: alternate rows/columns with t (paper); 1: rows only; 2: columns only */
+  int orientation;        /* 0: alternate rows/columns with t (paper); 1: rows only; 2: columns only;
+                             3: rows then columns every step (Table 5b "Row+Column/Step", read as:
+                             the rows of the row-active tangent momentum normalized, then the columns
+                             of the result; preconditioning and update in the row orientation) */
   int tangent;            /* momentum treatment before normalization: 0 relaxed tangent (paper,
                              x_i = m_i - <m_i, w_i> w_i); 1 none (x_i = m_i); 2 strict tangent
                              (x_i = m_i - <m_i, w_i> w_i / ||w_i||^2) -- the Table 5a ablations */

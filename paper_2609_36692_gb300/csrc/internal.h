@@ -116,6 +116,9 @@ cudaError_t launch_muon_prescale(const double* part, int nblk, int stride, int b
                                  cudaStream_t s);
 constexpr int kMuonBlocks = 64;   // row blocks per matrix of the Muon momentum pass
 cudaError_t launch_normalize_cols(const NormLaunch& a, cudaStream_t s);
+// Orientation 3 ("Row+Column/Step"): the columns of a row-normalized Psi
+// normalized in place; count[] becomes the number of nonzero columns.
+cudaError_t launch_normalize_psi_cols(const NormLaunch& a, cudaStream_t s);
 size_t normalize_cols_scratch_bytes(int64_t rows, int64_t cols, int n);
 size_t normalize_cols_part_bytes(int64_t rows, int64_t cols, int n);   // col_part share of it
 

@@ -325,6 +325,71 @@ __global__ void __launch_bounds__(kColThreads) k_norm_cols_apply(const __grid_co
 }
 
 // ---------------------------------------------------------------------------
+// "Row+Column/Step" (orientation 3, Table 5b): after the row normalization,
+// the columns of Psi (stored layout, row stride psi_ld) are normalized in
+// place.  Pass 1 sums psi^2 per (block of kColStatsRB rows, column) into fp64
+// partials; a fold (one CTA per matrix, fixed order) writes 1 / ||column||
+// and sets count[] to the number of nonzero columns (then ||Psi||_F^2);
+// pass 2 scales.
+// ---------------------------------------------------------------------------
+template <typename TP>
+__global__ void __launch_bounds__(256) k_psi_colsq(const __grid_constant__ NormLaunch a) {
+  const int b = blockIdx.z, rb = blockIdx.y;
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+  if (j >= a.cols) return;
+  const TP* psi = static_cast<const TP*>(a.psi[b]);
+  const int64_t r0 = static_cast<int64_t>(rb) * kColStatsRB, r1 = min(r0 + kColStatsRB, a.rows);
+  float s = 0.f;
+  for (int64_t r = r0; r < r1; ++r) {
+    const float v = to_f32(psi[r * a.psi_ld + j]);
+    s = fmaf(v, v, s);
+  }
+  a.col_part[(static_cast<int64_t>(b) * gridDim.y + rb) * a.cols + j] = s;
+}
+
+__global__ void __launch_bounds__(256) k_psi_colfold(const __grid_constant__ NormLaunch a, int nrb) {
+  __shared__ float red[32];
+  const int b = blockIdx.x;
+  float nz = 0.f;
+  for (int64_t j = threadIdx.x; j < a.cols; j += blockDim.x) {
+    double s = 0;
+    for (int rb = 0; rb < nrb; ++rb) s += a.col_part[(static_cast<int64_t>(b) * nrb + rb) * a.cols + j];
+    const float inv = s > 0.0 ? static_cast<float>(1.0 / sqrt(s)) : 0.f;
+    a.col_coef[static_cast<int64_t>(b) * a.cols + j] = make_float2(0.f, inv);
+    nz += s > 0.0 ? 1.f : 0.f;
+  }
+  nz = block_sum(nz, red);
+  if (threadIdx.x == 0) a.count[a.mat_id[b]] = static_cast<int>(nz);
+}
+
+template <typename TP>
+__global__ void __launch_bounds__(256) k_psi_colscale(const __grid_constant__ NormLaunch a) {
+  const int b = blockIdx.z;
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+  if (j >= a.cols) return;
+  const float inv = a.col_coef[static_cast<int64_t>(b) * a.cols + j].y;
+  TP* psi = static_cast<TP*>(a.psi[b]);
+  const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kColApplyRB, r1 = min(r0 + kColApplyRB, a.rows);
+  for (int64_t r = r0; r < r1; ++r) psi[r * a.psi_ld + j] = from_f32<TP>(to_f32(psi[r * a.psi_ld + j]) * inv);
+}
+
+cudaError_t launch_normalize_psi_cols(const NormLaunch& a, cudaStream_t s) {
+  if (a.n <= 0 || a.rows <= 0 || a.cols <= 0) return cudaSuccess;
+  const int nrb = static_cast<int>(cdiv(a.rows, kColStatsRB));
+  const unsigned cb = static_cast<unsigned>(cdiv(a.cols, 256));
+  if (a.psi_dtype == 1) k_psi_colsq<bf16><<<dim3(cb, nrb, a.n), 256, 0, s>>>(a);
+  else k_psi_colsq<float><<<dim3(cb, nrb, a.n), 256, 0, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_psi_colfold<<<a.n, 256, 0, s>>>(a, nrb);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const dim3 g2(cb, static_cast<unsigned>(cdiv(a.rows, kColApplyRB)), a.n);
+  if (a.psi_dtype == 1) k_psi_colscale<bf16><<<g2, 256, 0, s>>>(a);
+  else k_psi_colscale<float><<<g2, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // launchers
 // ---------------------------------------------------------------------------
 template <typename F>

@@ -121,7 +121,7 @@ int check_config(const normpre_config* c, std::string* msg) {
     *msg = "momentum, weight_decay and target_rms must be finite"; return NORMPRE_ERR_ARG;
   }
   if (c->precision != NORMPRE_PREC_BF16 && c->precision != NORMPRE_PREC_F32) { *msg = "bad precision"; return NORMPRE_ERR_ARG; }
-  if (c->orientation < 0 || c->orientation > 2) { *msg = "orientation must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
+  if (c->orientation < 0 || c->orientation > 3) { *msg = "orientation must be 0, 1, 2 or 3"; return NORMPRE_ERR_ARG; }
   if (c->tangent < 0 || c->tangent > 2) { *msg = "tangent must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
   if (c->variant == NORMPRE_L_EXACT) {
     if (c->rank < 1 || c->rank > 64) { *msg = "need 1 <= rank <= 64"; return NORMPRE_ERR_ARG; }
@@ -139,7 +139,7 @@ int check_config(const normpre_config* c, std::string* msg) {
 }
 
 int orientation_of(const normpre_config& c, int64_t t) {
-  if (c.orientation == 1) return 0;
+  if (c.orientation == 1 || c.orientation == 3) return 0;
   if (c.orientation == 2) return 1;
   return static_cast<int>(((t % 2) + 2) % 2);
 }
@@ -404,6 +404,10 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
       } else {
         e = (k == 0) ? launch_normalize_rows(a, s) : launch_normalize_cols(a, s);
         n_norm += (k == 0) ? 1 : 3;
+        if (!e && c.orientation == 3) {
+          e = launch_normalize_psi_cols(a, s);
+          n_norm += 3;
+        }
       }
       if (e) return cuda_fail(h, e, "normalize launch");
     }

@@ -274,7 +274,7 @@ def test_tangent_ablation_g_step(mode, t):
         assert rel_fro(W1[i].astype(np.float64) - mats[i]["W"], ref["W"] - mats[i]["W"]) <= 1e-4, (i, mode)
 
 
-@pytest.mark.parametrize("orientation", [1, 2], ids=["rows_only", "columns_only"])
+@pytest.mark.parametrize("orientation", [1, 2, 3], ids=["rows_only", "columns_only", "rows_then_columns"])
 @pytest.mark.parametrize("variant", ["G", "L"])
 def test_fixed_orientation(orientation, variant):
     # t = 1 would be column-active under the alternating default
@@ -282,9 +282,14 @@ def test_fixed_orientation(orientation, variant):
     opt, mats, W1, _ = _run(SMALL, 1, variant, precision=1, extra={"orientation": orientation})
     for i in range(SMALL.n_mats):
         ref = _oracle(mats, i, 1, variant, SMALL, orientation=orientation)
-        assert ref["k"] == (0 if orientation == 1 else 1)
+        assert ref["k"] == (1 if orientation == 2 else 0)
         st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
         assert int(st[0]) == ref["k"]
+        if orientation == 3:
+            # Psi has unit columns; ||Psi||_F^2 (stats m') = number of nonzero columns
+            psi = opt.read(i, C.NORMPRE_BUF_PSI).astype(np.float64)
+            assert np.max(np.abs(psi - ref["Psi"])) <= 1e-5, (i, variant)
+            assert int(st[1]) == int(np.sum(np.linalg.norm(ref["Psi"], axis=0) > 0))
         dW = W1[i].astype(np.float64) - mats[i]["W"]
         dW_ref = ref["W"] - mats[i]["W"]
         assert rel_fro(dW, dW_ref) <= (1e-4 if variant == "G" else 2e-3), (i, variant)
