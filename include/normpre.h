@@ -97,8 +97,9 @@ typedef struct normpre_config {
   float ns_coef[3];       /* (a, b, c) of X <- aX + b(XX^T)X + c(XX^T)^2 X; default Muon's
                              quintic (3.4445, -4.7750, 2.0315) */
   float ns_eps;           /* 1e-7: X is divided by ||X||_F + eps before the iteration */
-  int rank;               /* r = 32 (interaction rank budget) */
-  int oversample;         /* o = 8 */
+  int rank;               /* r = 32 (interaction rank budget); rank + oversample <= 72 */
+  int oversample;         /* o = 8 (the sketch width is l = min(m_a, r + o); l > 64 runs the
+                             contractions on the fp32 SIMT kernel instead of the tensor cores) */
   int power_iters;        /* p = 1 */
   uint64_t seed;          /* Philox4x32-10 key of the sketch matrix Omega */
   int precision;          /* normpre_precision */

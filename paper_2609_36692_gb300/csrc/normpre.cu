@@ -124,14 +124,14 @@ int check_config(const normpre_config* c, std::string* msg) {
   if (c->orientation < 0 || c->orientation > 3) { *msg = "orientation must be 0, 1, 2 or 3"; return NORMPRE_ERR_ARG; }
   if (c->tangent < 0 || c->tangent > 2) { *msg = "tangent must be 0, 1 or 2"; return NORMPRE_ERR_ARG; }
   if (c->variant == NORMPRE_L_EXACT) {
-    if (c->rank < 1 || c->rank > 64) { *msg = "need 1 <= rank <= 64"; return NORMPRE_ERR_ARG; }
+    if (c->rank < 1 || c->rank > 72) { *msg = "need 1 <= rank <= 72"; return NORMPRE_ERR_ARG; }
   } else if (uses_ns(c->variant)) {
     if (c->ns_steps < 1 || c->ns_steps > 100) { *msg = "ns_steps must be in [1, 100]"; return NORMPRE_ERR_ARG; }
     if (!std::isfinite(c->ns_coef[0]) || !std::isfinite(c->ns_coef[1]) || !std::isfinite(c->ns_coef[2]) ||
         !(c->ns_eps >= 0.f)) { *msg = "bad Newton-Schulz coefficients or eps"; return NORMPRE_ERR_ARG; }
   } else {
-    if (c->rank < 1 || c->oversample < 0 || c->rank + c->oversample > 64) {
-      *msg = "need rank >= 1, oversample >= 0 and rank + oversample <= 64"; return NORMPRE_ERR_ARG;
+    if (c->rank < 1 || c->oversample < 0 || c->rank + c->oversample > 72) {
+      *msg = "need rank >= 1, oversample >= 0 and rank + oversample <= 72"; return NORMPRE_ERR_ARG;
     }
     if (c->power_iters < 0 || c->power_iters > 8) { *msg = "power_iters must be in [0, 8]"; return NORMPRE_ERR_ARG; }
   }

@@ -15,7 +15,7 @@
 // GB300 notes.  FP64 runs at a small fraction of the FP32 rate on this part,
 // so every l x l kernel (Gram folds, Cholesky, triangular solve, Jacobi)
 // works in fp32; sums that fold many partial results use compensated
-// (Kahan) addition.  The l <= 64 wide products (contractions with Psi, the
+// (Kahan) addition.  The l <= 72 wide products (contractions with Psi, the
 // projector apply) keep one output row per thread with its l accumulators in
 // registers and read the small operand from shared memory by broadcast, so
 // they are bound by FMA issue rather than by shared-memory bandwidth; K is
@@ -37,7 +37,9 @@
 
 namespace normpre {
 
-constexpr int kLmax = 64;        // largest supported sketch width l
+constexpr int kLmax = 72;        // largest supported sketch width l (r = 64 with o = 8)
+// (pair, row) items of one Jacobi rotation step per thread, with at most 1024 threads
+constexpr int kJacItems = ((kLmax / 2) * kLmax + 1023) / 1024;
 constexpr int kGramRows = 64;    // rows per fp32 chunk of the split Gram sums
 constexpr int kMaxKSplit = 8;    // split-K factor bound of the contractions
 
@@ -876,9 +878,9 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
     frob2 = block_sum(s, red);
   }
   // this thread's (pair, row) items: e = tid + nt * it, pair = e / l, row = e % l
-  int ik[2], ir[2];
+  int ik[kJacItems], ir[kJacItems];
 #pragma unroll
-  for (int it = 0; it < 2; ++it) {
+  for (int it = 0; it < kJacItems; ++it) {
     const int e = tid + nt * it;
     ik[it] = (e < npairs * l) ? e / l : -1;
     ir[it] = (e < npairs * l) ? e % l : 0;
@@ -911,7 +913,7 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
       __syncthreads();
       // columns: A <- A J, V <- V J
 #pragma unroll
-      for (int it = 0; it < 2; ++it) {
+      for (int it = 0; it < kJacItems; ++it) {
         if (ik[it] < 0) continue;
         const int k = ik[it], r = ir[it];
         const int i = pp[k], j = qq[k];
@@ -927,7 +929,7 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
       __syncthreads();
       // rows: A <- J^T A
 #pragma unroll
-      for (int it = 0; it < 2; ++it) {
+      for (int it = 0; it < kJacItems; ++it) {
         if (ik[it] < 0) continue;
         const int k = ik[it], r = ir[it];
         const int i = pp[k], j = qq[k];
@@ -1125,7 +1127,7 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
 // ---------------------------------------------------------------------------
 // host orchestration
 // ---------------------------------------------------------------------------
-#define NP_FOR_LP(X) X(8) X(16) X(24) X(32) X(40) X(48) X(56) X(64)
+#define NP_FOR_LP(X) X(8) X(16) X(24) X(32) X(40) X(48) X(56) X(64) X(72)
 
 template <bool TRANS>
 static cudaError_t launch_contract(const ContractArgs& c, int batch, int cpt, cudaStream_t s) {
@@ -1136,6 +1138,7 @@ static cudaError_t launch_contract(const ContractArgs& c, int batch, int cpt, cu
 #define NP_CT(N) case N: k_contract<TRANS, N><<<grid, kCtThreads, kCtSmem, s>>>(c); break;
     NP_CT(1) NP_CT(2) NP_CT(3) NP_CT(4) NP_CT(5) NP_CT(6) NP_CT(7) NP_CT(8)
     NP_CT(9) NP_CT(10) NP_CT(11) NP_CT(12) NP_CT(13) NP_CT(14) NP_CT(15) NP_CT(16)
+    NP_CT(17) NP_CT(18)
 #undef NP_CT
     default:
       return cudaErrorInvalidValue;
@@ -1149,6 +1152,7 @@ static void contract_attrs() {
   cudaFuncSetAttribute(k_contract<TRANS, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kCtSmem));
   NP_CT(1) NP_CT(2) NP_CT(3) NP_CT(4) NP_CT(5) NP_CT(6) NP_CT(7) NP_CT(8)
   NP_CT(9) NP_CT(10) NP_CT(11) NP_CT(12) NP_CT(13) NP_CT(14) NP_CT(15) NP_CT(16)
+  NP_CT(17) NP_CT(18)
 #undef NP_CT
 }
 

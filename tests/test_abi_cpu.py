@@ -67,7 +67,7 @@ def test_host_side_argument_errors(lib):
     with pytest.raises(C.NormPreError) as e:
         C.normpre_init(bad, [(4, 5)], [0], [0])
     assert e.value.status == C.NORMPRE_ERR_ARG
-    bad = C.normpre_default_config(variant=C.NORMPRE_L, rank=60, oversample=8)
+    bad = C.normpre_default_config(variant=C.NORMPRE_L, rank=66, oversample=8)
     with pytest.raises(C.NormPreError) as e:
         C.normpre_init(bad, [(4, 5)], [0], [0])
     assert e.value.status == C.NORMPRE_ERR_ARG
@@ -88,7 +88,7 @@ def test_host_side_argument_errors(lib):
         C.normpre_init(bad, [(4, 5)], [0], [0])
     assert "diagnostics" in C.normpre_last_error()
     # exact eigenspace extraction: rank budget and the Gamma workspace limit
-    bad = C.normpre_default_config(variant=C.NORMPRE_L_EXACT, rank=65)
+    bad = C.normpre_default_config(variant=C.NORMPRE_L_EXACT, rank=73)
     with pytest.raises(C.NormPreError) as e:
         C.normpre_init(bad, [(4, 5)], [0], [0])
     assert e.value.status == C.NORMPRE_ERR_ARG

@@ -295,6 +295,29 @@ def test_fixed_orientation(orientation, variant):
         assert rel_fro(dW, dW_ref) <= (1e-4 if variant == "G" else 2e-3), (i, variant)
 
 
+@pytest.mark.parametrize("t", [0, 1])
+def test_rank_64(t):
+    """Table 6's largest rank budget: r = 64 with o = 8 (l = 72, beyond the
+    tensor-core contraction's l <= 64: the SIMT kernel takes it)."""
+    import dataclasses
+    cs = dataclasses.replace(SMALL, rank=64, oversample=8)
+    _check_l(cs, t)
+
+
+def test_rank_64_exact():
+    import dataclasses
+    from paper_2609_36692_gb300 import normpre as C
+    cs = dataclasses.replace(SMALL, rank=64, oversample=0)
+    opt, mats, W1, _ = _run(cs, 0, "L_exact", precision=1)
+    for i in range(cs.n_mats):
+        ref = _oracle(mats, i, 0, "L_exact", cs)
+        st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
+        if ritz_gaps_ok(ref["exact"]["lam"], cs.rank):
+            assert int(st[3]) == ref["exact"]["n_active"]
+        dW = W1[i].astype(np.float64) - mats[i]["W"]
+        assert rel_fro(dW, ref["W"] - mats[i]["W"]) <= 2e-3, i
+
+
 def test_two_power_iterations():
     import dataclasses
     cs = dataclasses.replace(SMALL, power_iters=2)
