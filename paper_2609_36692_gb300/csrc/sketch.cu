@@ -1028,6 +1028,7 @@ struct LApplyArgs {
   const void* G[kMaxBatch];
   int g_dtype;
   double* diag[kMaxBatch];
+  int vec_panels;   // l % 4 == 0 and 16-byte aligned panel rows: float4 panel loads
 };
 template <typename TW, bool VEC, bool DIAG>
 __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyArgs a) {
@@ -1049,13 +1050,31 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
   const int l = a.l;
   const float* lm = a.lm + b * a.lm_bs;
   const float* rm = a.rm + b * a.rm_bs;
-  for (int e = tid; e < 64 * l; e += 256) {
-    const int i = e / l, p = e - i * l;
-    Ls[p][i] = (r0 + i < a.rows) ? lm[(r0 + i) * l + p] : 0.f;
-    Rs[p][i] = (c0 + i < a.cols) ? rm[(c0 + i) * l + p] : 0.f;
+  {
+    // the 64 rows of Lm and the 64 of Rm, two threads per row (no division
+    // by l: the load loop is a good part of the kernel's instructions)
+    const int row = tid >> 1, half = tid & 1, i = row & 63;
+    const bool right = row >= 64;
+    const int64_t grow = (right ? c0 : r0) + i;
+    const bool ok = grow < (right ? a.cols : a.rows);
+    const float* src = (right ? rm : lm) + grow * l;
+    float (*dst)[64 + 4] = right ? Rs : Ls;
+    if (a.vec_panels) {
+      // 16-byte pieces: q and q + 1 go to different halves of the bank space
+      for (int q = half; q < (l >> 2); q += 2) {
+        const float4 v = ok ? *reinterpret_cast<const float4*>(src + 4 * q) : make_float4(0.f, 0.f, 0.f, 0.f);
+        dst[4 * q][i] = v.x;
+        dst[4 * q + 1][i] = v.y;
+        dst[4 * q + 2][i] = v.z;
+        dst[4 * q + 3][i] = v.w;
+      }
+    } else {
+      for (int p = half; p < l; p += 2) dst[p][i] = ok ? src[p] : 0.f;
+    }
   }
   __syncthreads();
   float acc[4][4] = {};
+#pragma unroll 4
   for (int p = 0; p < l; ++p) {
     const float4 lv = *reinterpret_cast<const float4*>(&Ls[p][ty * 4]);
     const float4 rv = *reinterpret_cast<const float4*>(&Rs[p][tx * 4]);
@@ -1430,6 +1449,8 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     for (int i = 0; i < nb; ++i) la.W[i] = W[c0 + i];
     la.rows = g.rows; la.cols = g.cols; la.l = l;
     la.lr = p.lr; la.wd = p.wd; la.target = p.target;
+    la.vec_panels = (l % 4 == 0) && (vbs % 4 == 0) &&
+                    (reinterpret_cast<uintptr_t>(la.lm) % 16 == 0) && (reinterpret_cast<uintptr_t>(la.rm) % 16 == 0);
     const bool diag = p.diag && p.G;
     la.g_dtype = p.g_dtype;
     for (int i = 0; i < nb; ++i) {
