@@ -418,7 +418,7 @@ def test_deterministic(variant):
         assert np.array_equal(a, b)
 
 
-@pytest.mark.parametrize("variant", ["G", "L", "muon"])
+@pytest.mark.parametrize("variant", ["G", "L", "muon", "L_exact"])
 def test_host_entry_point_matches_device_step(variant):
     """Two consecutive host-buffer steps (row- then column-active) equal the
     device-buffer steps bit for bit: the copies overlapped with the step move
@@ -427,9 +427,10 @@ def test_host_entry_point_matches_device_step(variant):
     from paper_2609_36692_gb300 import normpre as C
     cs = SMALL
     mats = S.make_param_set(cs, workers=min(16, os.cpu_count() or 1))
-    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON}[variant],
-              precision=0 if variant != "L" else 1, rank=cs.rank, oversample=cs.oversample,
-              power_iters=cs.power_iters, seed=1234)
+    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON,
+                       "L_exact": C.NORMPRE_L_EXACT}[variant],
+              precision=0 if variant in ("G", "muon") else 1, rank=cs.rank, oversample=cs.oversample,
+              power_iters=cs.power_iters, seed=1234, diagnostics=1)
     shapes = [(m.rows, m.cols) for m in cs.matrices]
     opt = _normpre(shapes, ["f32"] * cs.n_mats, ["bf16"] * cs.n_mats, **kw)
     opt2 = _normpre(shapes, ["f32"] * cs.n_mats, ["bf16"] * cs.n_mats, **kw)
@@ -447,7 +448,7 @@ def test_host_entry_point_matches_device_step(variant):
             assert np.array_equal(Mh[i].numpy(), to_host(M[i])), (t, i)
 
 
-@pytest.mark.parametrize("variant", ["G", "L", "muon"])
+@pytest.mark.parametrize("variant", ["G", "L", "muon", "L_exact"])
 def test_host_entry_point_in_units(variant):
     """A group larger than one host-copy unit (8 x 4096^2 fp32/bf16: about
     1.3 GB of input) is preconditioned in pieces of matrices between its copies;
@@ -459,8 +460,9 @@ def test_host_entry_point_in_units(variant):
     Wc = [torch.randn(r, c, generator=gen) * 0.02 for r, c in shapes]
     Gc = [torch.randn(r, c, generator=gen).to(torch.bfloat16) for r, c in shapes]
     Mc = [torch.randn(r, c, generator=gen) * 0.1 for r, c in shapes]
-    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON}[variant],
-              precision=0 if variant != "L" else 1, seed=1234)
+    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON,
+                       "L_exact": C.NORMPRE_L_EXACT}[variant],
+              precision=0 if variant in ("G", "muon") else 1, seed=1234)
     opt = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
     opt2 = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
     W = [w.cuda() for w in Wc]
