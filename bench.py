@@ -154,6 +154,18 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(self.rows)}
 
 
+def max_over_ranks(x: float, world: int, device: str) -> float:
+    """The largest value over the ranks of the process group (the job's time
+    is its slowest rank's); x itself when there is one rank."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    tt = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+    return float(tt.item())
+
+
 def oracle_sample(cfg: S.ParamSetConfig, variant: str, seconds_budget: float = 20.0):
     """Times the fp64 oracle on a bounded sample of the workload (one layer's
     matrices of each distinct shape) and scales to the whole parameter set by
@@ -286,10 +298,7 @@ def run_ours(args, cfg, variant, rank, world):
         clocks = soak.summary()
         clocks["source"] = "1.5 s soak of the same step right after the timed region (too short to sample)"
     ms_step = ms_total / args.steps
-    if world > 1:
-        tt = torch.tensor([ms_step], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_step = float(tt.item())
+    ms_step = max_over_ranks(ms_step, world, "cuda")
 
     # ---- per-kernel-class time of the same workload (events on the launch stream) ----
     C.normpre_profile(h, True)
@@ -372,10 +381,7 @@ def run_ours(args, cfg, variant, rank, world):
         opt.step_host(t, LR, Wh, Gh, Mh)
         t += 1
     e2e_ms = (time.perf_counter() - t0) * 1e3 / n_e2e
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e_ms = max_over_ranks(e2e_ms, world, "cuda")
 
     # ---- the paper's comparison optimizer (Muon) on the same workload and kernels ----
     muon = None
@@ -397,10 +403,7 @@ def run_ours(args, cfg, variant, rank, world):
         ms_muon = ev0.elapsed_time(ev1) / args.steps
         opt_m.status()
         opt_m.close()
-        if world > 1:
-            tt = torch.tensor([ms_muon], device="cuda")
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            ms_muon = float(tt.item())
+        ms_muon = max_over_ranks(ms_muon, world, "cuda")
         muon = {"ms_per_step": ms_muon, "normpre_vs_muon": ms_step / ms_muon - 1.0,
                 "paper_a100_context": "optimizer latency vs Muon on A100: NormPre-G +5.76 % / +4.37 % / +6.77 %, "
                                       "NormPre-L -38.12 % / -67.00 % / -57.16 % (GPT-2 Small / LLaMA-1.3B / "
