@@ -239,6 +239,7 @@ struct SketchGroup {
   float* kpart = nullptr;       // split-K partials of the contractions
   float* part = nullptr;        // partial Gram sums (fp32, folded with compensation)
   float* kmat = nullptr;        // [l][l] R^{-1} of a CholeskyQR pass, then K = Z_C (Lam_C^{-1/2} - I) Z_C^T
+  float* gram = nullptr;        // [l][l] folded Gram of a panel (CholeskyQR, Rayleigh-Ritz)
   float* ritz = nullptr;        // [l]
   float* zvec = nullptr;        // [l][l]
   float* stats = nullptr;       // [8] per matrix

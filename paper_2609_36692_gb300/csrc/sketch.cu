@@ -721,6 +721,33 @@ __device__ __forceinline__ void fold_partials(const float* part, int nsplit, int
   }
 }
 
+// The nsplit partial l x l sums of each matrix folded once (one thread per
+// entry, fixed order, compensated) into gram [batch][sq]: the consumers then
+// read one value per entry instead of each walking the partials.
+struct GramFoldArgs {
+  const float* part; int64_t part_bs; int nsplit;
+  float* gram; int64_t gram_bs;
+  int l;
+};
+__global__ void __launch_bounds__(256) k_gram_fold(const __grid_constant__ GramFoldArgs a) {
+  const int b = blockIdx.y;
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= a.l * a.l) return;
+  const float* part = a.part + b * a.part_bs;
+  const int64_t stride = static_cast<int64_t>(a.l) * a.l;
+  Kahan k;
+  int s = 0;
+  for (; s + 8 <= a.nsplit; s += 8) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = __ldcg(part + (s + u) * stride + e);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) k.add(v[u]);
+  }
+  for (; s < a.nsplit; ++s) k.add(__ldcg(part + s * stride + e));
+  a.gram[b * a.gram_bs + e] = k.s;
+}
+
 // ---------------------------------------------------------------------------
 // One CholeskyQR pass, fused: every CTA folds the Gram partials of Y,
 // factors G = R^T R (upper R, fp32; one diagonal shift when a pivot falls
@@ -1208,6 +1235,7 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
   if ((e = alloc((void**)&g.kpart, vec * kMaxKSplit))) return e;
   if ((e = alloc((void**)&g.part, static_cast<size_t>(g.batch) * g.max_part * g.lmax * g.lmax * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.kmat, sq * sizeof(float)))) return e;
+  if ((e = alloc((void**)&g.gram, sq * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.ritz, static_cast<size_t>(g.batch) * g.lmax * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.zvec, sq * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.stats, static_cast<size_t>(g.batch) * 8 * sizeof(float)))) return e;
@@ -1246,6 +1274,7 @@ cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup
   s.kpart = g.kpart + b0 * vbs * kMaxKSplit;
   s.part = g.part + b0 * static_cast<int64_t>(g.max_part) * sq;
   s.kmat = g.kmat + b0 * sq;
+  s.gram = g.gram + b0 * sq;
   s.zvec = g.zvec + b0 * sq;
   s.ritz = g.ritz + static_cast<int64_t>(b0) * g.lmax;
   s.stats = g.stats + static_cast<int64_t>(b0) * 8;
@@ -1361,14 +1390,25 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   };
   const bool ta = !rows_active;     // Psi_a V:   row contract (k = 0) or column contract (k = 1)
   const bool tb = rows_active;      // Psi_a^T U: the other one
-  auto gram = [&](const float* y, int64_t n) -> int {
+  // Gram partials of an n x l panel, folded once per matrix into g.gram when
+  // there is more than one; returns where the consumer reads them (pointer,
+  // matrix stride, count of partial sums)
+  struct GramOut { const float* p; int64_t bs; int n; };
+  int n_fold = 0;   // fold launches (for the per-class launch counts)
+  auto gram = [&](const float* y, int64_t n) -> GramOut {
     GramArgs ga;
     ga.y = y; ga.y_bs = vbs; ga.part = g.part;
     ga.part_bs = static_cast<int64_t>(g.max_part) * sq;
     ga.n = n; ga.l = l;
     ga.nsplit = static_cast<int>(cdiv(n, kGramRows));
     k_gram_part<<<dim3(ga.nsplit, B), 256, 0, s>>>(ga);
-    return ga.nsplit;
+    if (ga.nsplit == 1) return GramOut{g.part, ga.part_bs, 1};
+    GramFoldArgs fa;
+    fa.part = g.part; fa.part_bs = ga.part_bs; fa.nsplit = ga.nsplit;
+    fa.gram = g.gram; fa.gram_bs = sq; fa.l = l;
+    k_gram_fold<<<dim3(static_cast<unsigned>(cdiv(static_cast<int64_t>(l) * l, 256)), B), 256, 0, s>>>(fa);
+    ++n_fold;
+    return GramOut{g.gram, sq, 1};
   };
   if (p.exact) {
     // exact eigenpairs of Gamma = Psi_a Psi_a^T (exact.cu), then B^T = Psi_a^T Q
@@ -1390,26 +1430,27 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     {
       const float* src = ycur;
       for (int pass = 0; pass < 3; ++pass) {
-        const int ns = gram(src, m_a);
+        const GramOut go = gram(src, m_a);
         NP_CHECK();
         float* dst = (pass == 1) ? g.zt : g.q;
         CholQRArgs cq;
-        cq.part = g.part; cq.part_bs = static_cast<int64_t>(g.max_part) * sq; cq.nsplit = ns;
+        cq.part = go.p; cq.part_bs = go.bs; cq.nsplit = go.n;
         cq.y = src; cq.q = dst; cq.v_bs = vbs;
         cq.n = m_a; cq.l = l; cq.flags = flags;
         if ((e = launch_cholqr(cq, B, lp, s))) return e;
         src = dst;
       }
     }
-    prof->end(kProfQR, s, 6);
+    prof->end(kProfQR, s, 6 + n_fold);
+    n_fold = 0;
     // B^T = Psi_a^T Q  [n_a x l];  Gamma_Q = B B^T
     if ((e = contract(tb, g.q, g.bt))) return e;
     prof->begin(kProfEig, s);
     {
-      const int ns = gram(g.bt, n_a);
+      const GramOut go = gram(g.bt, n_a);
       NP_CHECK();
       EigArgs ea;
-      ea.part = g.part; ea.part_bs = static_cast<int64_t>(g.max_part) * sq; ea.nsplit = ns;
+      ea.part = go.p; ea.part_bs = go.bs; ea.nsplit = go.n;
       ea.ritz = g.ritz; ea.ritz_bs = g.lmax;
       ea.z = g.zvec; ea.z_bs = sq;
       ea.kmat = g.kmat; ea.k_bs = sq;
@@ -1432,7 +1473,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     k_rowmul<<<dim3(static_cast<unsigned>(cdiv(m_a * l, 256)), B), 256, 0, s>>>(rm);
     NP_CHECK();
   }
-  prof->end(kProfEig, s, p.exact ? 1 : 3);
+  prof->end(kProfEig, s, (p.exact ? 1 : 3) + n_fold);
   // T_s = Psi + Lm R^T with (Lm, R) = (QK, B^T) row-active or (B^T, QK) column-active,
   // in launches of at most kMaxBatch matrices (W pointers travel as kernel arguments)
   prof->begin(kProfApplyL, s);
