@@ -38,8 +38,6 @@
 namespace normpre {
 
 constexpr int kLmax = 72;        // largest supported sketch width l (r = 64 with o = 8)
-// (pair, row) items of one Jacobi rotation step per thread, with at most 1024 threads
-constexpr int kJacItems = ((kLmax / 2) * kLmax + 1023) / 1024;
 constexpr int kGramRows = 64;    // rows per fp32 chunk of the split Gram sums
 constexpr int kMaxKSplit = 8;    // split-K factor bound of the contractions
 
@@ -749,33 +747,40 @@ __global__ void __launch_bounds__(256) k_gram_fold(const __grid_constant__ GramF
 }
 
 // ---------------------------------------------------------------------------
-// One CholeskyQR pass, fused: every CTA folds the Gram partials of Y,
-// factors G = R^T R (upper R, fp32; one diagonal shift when a pivot falls
-// below 1e-6 tr(G)) and then solves q R = y for 256 rows of Y, one row per
-// thread (forward substitution, R read by broadcast).  The factorization is
-// repeated by each CTA of a matrix: it is tiny next to the row solves.
+// One CholeskyQR pass, fused: every CTA loads the Gram matrix G of Y, factors
+// G = R^T R (upper R, fp32; one diagonal shift when a pivot falls below
+// 1e-6 tr(G)) and then solves q R = y for 256 rows of Y, one row per thread.
+// The factorization is right-looking over the whole CTA (one pivot per
+// barrier, the trailing square updated by a 16 x 16 thread grid); the solve
+// is column-oriented (x_k final, then every later x_j updated from row k of
+// R), so its dependent chain is l steps long, not l^2 / 2.  The
+// factorization is repeated by each CTA of a matrix: it is tiny next to the
+// row solves.
 // ---------------------------------------------------------------------------
 struct CholQRArgs {
   const float* part; int64_t part_bs; int nsplit;
   const float* y; float* q; int64_t v_bs;    // [n][l] panels
   int64_t n;
   int l;
+  int vec;       // l % 4 == 0 and 16-byte aligned rows: float4 row loads / stores
   int* flags;
 };
 template <int LP>
 __global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRArgs a) {
-  __shared__ float Gm[LP][LP + 1];
-  __shared__ float Rm[LP][LP + 1];
-  __shared__ int bad;
+  // G (row stride LP + 1) until the factorization ends, then R strictly above
+  // the diagonal and zero elsewhere (row stride LP, 16-byte rows)
+  __shared__ __align__(16) float GR[LP * (LP + 1)];
+  __shared__ float Wm[LP][LP + 1];             // G + shift I, reduced in place
+  __shared__ float rinv[LP];                   // 1 / R_jj (zero past l)
   __shared__ float tr;
   const int b = blockIdx.y, l = a.l, tid = threadIdx.x;
-  if (tid == 0) bad = 0;
-  fold_partials(a.part + b * a.part_bs, a.nsplit, l, &Gm[0][0], LP + 1);
+  fold_partials(a.part + b * a.part_bs, a.nsplit, l, GR, LP + 1);
   __syncthreads();
-  if (tid == 0) {
+  if (tid < 32) {
     float t = 0.f;
-    for (int i = 0; i < l; ++i) t += Gm[i][i];
-    tr = t;
+    for (int i = tid; i < l; i += 32) t += GR[i * (LP + 1) + i];
+    t = warp_sum(t);
+    if (tid == 0) tr = t;
   }
   __syncthreads();
   const int64_t row = static_cast<int64_t>(blockIdx.x) * 256 + tid;
@@ -787,48 +792,74 @@ __global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRAr
       for (int j = 0; j < l; ++j) q[j] = 0.f;
     return;
   }
-  // G = R^T R, row by row in one warp (row j needs rows 0 .. j-1); the whole
-  // CTA then solves its rows of Y against R.
-  if (tid < 32) {
-    for (int attempt = 0; attempt < 2; ++attempt) {
-      const float shift = attempt == 0 ? 0.f : 1e-5f * tr;
-      int bd = 0;
-      for (int j = 0; j < l; ++j) {
-        float d = Gm[j][j] + shift;
-        for (int k = 0; k < j; ++k) d = fmaf(-Rm[k][j], Rm[k][j], d);
-        if (!(d > 1e-6f * tr)) bd = 1;
-        const float rjj = sqrtf(fmaxf(d, 1e-30f * tr));
-        for (int i = j + 1 + tid; i < l; i += 32) {
-          float v = Gm[j][i];
-          for (int k = 0; k < j; ++k) v = fmaf(-Rm[k][j], Rm[k][i], v);
-          Rm[j][i] = v / rjj;
-        }
-        if (tid == 0) Rm[j][j] = rjj;
-        __syncwarp();
-      }
-      if (!bd) break;
-      if (attempt == 1 && tid == 0) bad = 1;
+  // right-looking Cholesky: at pivot j, W[p][q] -= W[j][p] W[j][q] / W[j][j]
+  // for p, q > j (the whole trailing square, so W stays symmetric); row j is
+  // final from then on and R[j][i] = W[j][i] / sqrt(W[j][j])
+  const int ty = tid >> 4, tx = tid & 15;
+  bool bad = false;
+  for (int attempt = 0; attempt < 2; ++attempt) {
+    const float shift = attempt == 0 ? 0.f : 1e-5f * tr;
+    for (int e = tid; e < l * l; e += 256) {
+      const int i = e / l, j = e - i * l;
+      Wm[i][j] = GR[i * (LP + 1) + j] + (i == j ? shift : 0.f);
     }
+    __syncthreads();
+    bad = false;
+    for (int j = 0; j < l; ++j) {
+      const float d = Wm[j][j];
+      if (!(d > 1e-6f * tr)) bad = true;
+      const float dinv = 1.f / fmaxf(d, 1e-30f * tr);
+      for (int p = j + 1 + ty; p < l; p += 16) {
+        const float wp = Wm[j][p] * dinv;
+        for (int c = j + 1 + tx; c < l; c += 16) Wm[p][c] = fmaf(-wp, Wm[j][c], Wm[p][c]);
+      }
+      __syncthreads();
+    }
+    if (!bad) break;     // every thread saw the same pivots
+  }
+  if (tid == 0 && bad && blockIdx.x == 0) raise_flag(a.flags, kFlagNumeric);
+  for (int i = tid; i < LP; i += 256) rinv[i] = (i < l) ? 1.f / sqrtf(fmaxf(Wm[i][i], 1e-30f * tr)) : 0.f;
+  __syncthreads();
+  for (int e = tid; e < LP * LP; e += 256) {
+    const int i = e / LP, j = e % LP;
+    GR[e] = (i < l && j < l && j > i) ? Wm[i][j] * rinv[i] : 0.f;
   }
   __syncthreads();
-  if (tid == 0 && bad && blockIdx.x == 0) raise_flag(a.flags, kFlagNumeric);
   if (row >= a.n) return;
   float x[LP];
+  if (a.vec) {
 #pragma unroll
-  for (int j = 0; j < LP; ++j) x[j] = (j < l) ? y[j] : 0.f;
-  // q R = y  =>  q_j = (y_j - sum_{k<j} q_k R_kj) / R_jj
+    for (int j = 0; j < LP; j += 4) {
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (j < l) v = *reinterpret_cast<const float4*>(y + j);
+      x[j] = v.x; x[j + 1] = v.y; x[j + 2] = v.z; x[j + 3] = v.w;
+    }
+  } else {
 #pragma unroll
-  for (int j = 0; j < LP; ++j) {
-    if (j < l) {
-      float s = x[j];
+    for (int j = 0; j < LP; ++j) x[j] = (j < l) ? y[j] : 0.f;
+  }
+  // q R = y: x_k = x_k / R_kk is final, then x_j -= x_k R_kj for j > k
 #pragma unroll
-      for (int k = 0; k < j; ++k) s = fmaf(-x[k], Rm[k][j], s);
-      x[j] = s / Rm[j][j];
+  for (int k = 0; k < LP; ++k) {
+    x[k] *= rinv[k];
+#pragma unroll
+    for (int j4 = ((k + 1) / 4) * 4; j4 < LP; j4 += 4) {
+      const float4 r = *reinterpret_cast<const float4*>(&GR[k * LP + j4]);
+      if (j4 + 0 > k) x[j4 + 0] = fmaf(-x[k], r.x, x[j4 + 0]);
+      if (j4 + 1 > k) x[j4 + 1] = fmaf(-x[k], r.y, x[j4 + 1]);
+      if (j4 + 2 > k) x[j4 + 2] = fmaf(-x[k], r.z, x[j4 + 2]);
+      if (j4 + 3 > k) x[j4 + 3] = fmaf(-x[k], r.w, x[j4 + 3]);
     }
   }
+  if (a.vec) {
 #pragma unroll
-  for (int j = 0; j < LP; ++j)
-    if (j < l) q[j] = x[j];
+    for (int j = 0; j < LP; j += 4)
+      if (j < l) *reinterpret_cast<float4*>(q + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < LP; ++j)
+      if (j < l) q[j] = x[j];
+  }
 }
 
 // out[N x l] = Y[N x l] * S[l x l] (S fp32 row-major), one thread per output
@@ -857,11 +888,15 @@ __global__ void __launch_bounds__(256) k_rowmul(const __grid_constant__ RowMulAr
 
 // ---------------------------------------------------------------------------
 // Parallel cyclic Jacobi (round-robin pairing) of Gamma_Q in fp32, then the
-// descending sort, the selection C and K.  One CTA per matrix; each thread
-// owns up to two (pair, row) items of every rotation step, with the item
-// indices computed once, so a step is three barriers and a handful of
-// shared-memory updates per thread.
+// descending sort, the selection C and K.  One CTA per matrix.  A rotation
+// step applies J^T A J as 2 x 2 blocks: the thread that owns block (k, k')
+// (rows of pair k, columns of pair k') computes both rotations from the
+// current copy of A, writes the rotated block into the other copy and rotates
+// two rows of V, so a step is one barrier.  When l is odd the matrices are
+// padded with a zero row and column whose pair is never rotated.
 // ---------------------------------------------------------------------------
+constexpr int kJacBlocks = ((kLmax / 2) * (kLmax / 2) + 1023) / 1024;   // blocks per thread
+constexpr size_t kJacSmem = 3 * static_cast<size_t>(kLmax) * (kLmax + 1) * sizeof(float);
 struct EigArgs {
   const float* part; int64_t part_bs; int nsplit;   // Gram partials of B^T
   float* ritz; int64_t ritz_bs;      // [l]
@@ -874,104 +909,116 @@ struct EigArgs {
   int max_sweeps;
   int* flags;
 };
+// players (i, j), i < j, of pair k at rotation step `step` of n players
+__device__ __forceinline__ void jac_pair(int k, int step, int n, int& i, int& j) {
+  int p = 0;
+  if (k != 0) { p = k - 1 + step; if (p >= n - 1) p -= n - 1; p += 1; }
+  int q = n - 2 - k + step; if (q >= n - 1) q -= n - 1; q += 1;
+  i = min(p, q);
+  j = max(p, q);
+}
+// the rotation (c, s) that annihilates A(i, j): t = tan(theta) is the smaller
+// root of t^2 + 2 t cot(2 theta) - 1 = 0, written without cot(2 theta)
+// (t = 2 a_ij sgn(d) / (|d| + sqrt(d^2 + 4 a_ij^2)), d = a_jj - a_ii)
+__device__ __forceinline__ void jac_rot(const float* A, int ld, int i, int j, int l, float& c, float& s) {
+  c = 1.f;
+  s = 0.f;
+  if (j >= l) return;                 // the padding player: not rotated
+  const float apq = A[i * ld + j];
+  if (!(fabsf(apq) > 1e-30f)) return;
+  const float d = A[j * ld + j] - A[i * ld + i];
+  const float num = (d >= 0.f) ? 2.f * apq : -2.f * apq;
+  const float t = __fdividef(num, fabsf(d) + sqrtf(fmaf(d, d, 4.f * apq * apq)));
+  c = rsqrtf(fmaf(t, t, 1.f));
+  s = t * c;
+}
 __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs a) {
   extern __shared__ float4 jc_smem4[];
   float* dsm = reinterpret_cast<float*>(jc_smem4);
-  __shared__ float cs[kLmax / 2], sn[kLmax / 2];
-  __shared__ int pp[kLmax / 2], qq[kLmax / 2];
   __shared__ float red[32];
   __shared__ int order[kLmax];
   const int b = blockIdx.x, l = a.l, tid = threadIdx.x, nt = blockDim.x;
-  const int n = (l + 1) & ~1;          // even number of "players" (one dummy if l is odd)
+  const int n = (l + 1) & ~1;          // even number of players (one padding player if l is odd)
   const int npairs = n / 2;
-  const int ld = l + 1;
-  float* Am = dsm;              // [l][l+1]
-  float* Vm = dsm + l * ld;     // [l][l+1]
-#define A(i, j) Am[(i) * ld + (j)]
+  const int ld = n + 1;
+  float* cur = dsm;                    // A [n][ld], two copies
+  float* nxt = dsm + n * ld;
+  float* Vm = dsm + 2 * n * ld;        // V [n][ld]
 #define V(i, j) Vm[(i) * ld + (j)]
-  fold_partials(a.part + b * a.part_bs, a.nsplit, l, Am, ld);
-  for (int e = tid; e < l * l; e += nt) V(e / l, e % l) = (e / l == e % l) ? 1.f : 0.f;
+  fold_partials(a.part + b * a.part_bs, a.nsplit, l, cur, ld);
+  for (int e = tid; e < n * n; e += nt) {
+    const int i = e / n, j = e - (e / n) * n;
+    if (i >= l || j >= l) cur[i * ld + j] = 0.f;
+    V(i, j) = (i == j) ? 1.f : 0.f;
+  }
   __syncthreads();
   // exact symmetry
   for (int e = tid; e < l * l; e += nt) {
     const int i = e / l, j = e % l;
-    if (i < j) { const float v = 0.5f * (A(i, j) + A(j, i)); A(i, j) = v; A(j, i) = v; }
+    if (i < j) {
+      const float v = 0.5f * (cur[i * ld + j] + cur[j * ld + i]);
+      cur[i * ld + j] = v;
+      cur[j * ld + i] = v;
+    }
   }
   __syncthreads();
   float frob2;
   {
     float s = 0.f;
-    for (int e = tid; e < l * l; e += nt) s += A(e / l, e % l) * A(e / l, e % l);
+    for (int e = tid; e < l * l; e += nt) {
+      const float v = cur[(e / l) * ld + e % l];
+      s += v * v;
+    }
     frob2 = block_sum(s, red);
   }
-  // this thread's (pair, row) items: e = tid + nt * it, pair = e / l, row = e % l
-  int ik[kJacItems], ir[kJacItems];
+  // this thread's blocks (k, k'), computed once
+  int bk[kJacBlocks], bk2[kJacBlocks];
 #pragma unroll
-  for (int it = 0; it < kJacItems; ++it) {
+  for (int it = 0; it < kJacBlocks; ++it) {
     const int e = tid + nt * it;
-    ik[it] = (e < npairs * l) ? e / l : -1;
-    ir[it] = (e < npairs * l) ? e % l : 0;
+    bk[it] = (e < npairs * npairs) ? e / npairs : -1;
+    bk2[it] = (e < npairs * npairs) ? e % npairs : 0;
   }
   int sweep = 0;
   float off = frob2, prev = frob2;
   for (; sweep < a.max_sweeps; ++sweep) {
     for (int step = 0; step < n - 1; ++step) {
-      if (tid < npairs) {
-        // round-robin pairing: position 0 fixed, the others rotate by `step`
-        const int k = tid, pa = k, pb = n - 1 - k;
-        int p = 0;
-        if (pa != 0) { p = pa - 1 + step; if (p >= n - 1) p -= n - 1; p += 1; }
-        int q = pb - 1 + step; if (q >= n - 1) q -= n - 1; q += 1;
-        int i = min(p, q), j = max(p, q);
-        float c = 1.f, s = 0.f;
-        if (j < l) {
-          const float apq = A(i, j);
-          if (fabsf(apq) > 1e-30f) {
-            const float th = (A(j, j) - A(i, i)) / (2.f * apq);
-            const float t = copysignf(1.f, th) / (fabsf(th) + sqrtf(fmaf(th, th, 1.f)));
-            c = rsqrtf(fmaf(t, t, 1.f));
-            s = t * c;
-          }
-        } else {
-          i = j = -1;
+#pragma unroll
+      for (int it = 0; it < kJacBlocks; ++it) {
+        if (bk[it] < 0) continue;
+        const int k = bk[it], k2 = bk2[it];
+        int i, j, i2, j2;
+        jac_pair(k, step, n, i, j);
+        jac_pair(k2, step, n, i2, j2);
+        // the block's entries do not depend on the rotations: load them first
+        const float a00 = cur[i * ld + i2], a01 = cur[i * ld + j2];
+        const float a10 = cur[j * ld + i2], a11 = cur[j * ld + j2];
+        float c, s, c2, s2;
+        jac_rot(cur, ld, i, j, l, c, s);
+        if (k2 == k) { c2 = c; s2 = s; } else { jac_rot(cur, ld, i2, j2, l, c2, s2); }
+        // columns i2, j2 (A J), then rows i, j (J^T A)
+        const float u0 = c2 * a00 - s2 * a01, w0 = s2 * a00 + c2 * a01;
+        const float u1 = c2 * a10 - s2 * a11, w1 = s2 * a10 + c2 * a11;
+        nxt[i * ld + i2] = c * u0 - s * u1;
+        nxt[j * ld + i2] = s * u0 + c * u1;
+        nxt[i * ld + j2] = c * w0 - s * w1;
+        nxt[j * ld + j2] = s * w0 + c * w1;
+        // V <- V J: rows k' and k' + n/2, columns of pair k
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int r = k2 + h * npairs;
+          const float vi = V(r, i), vj = V(r, j);
+          V(r, i) = c * vi - s * vj;
+          V(r, j) = s * vi + c * vj;
         }
-        pp[k] = i; qq[k] = j; cs[k] = c; sn[k] = s;
       }
       __syncthreads();
-      // columns: A <- A J, V <- V J
-#pragma unroll
-      for (int it = 0; it < kJacItems; ++it) {
-        if (ik[it] < 0) continue;
-        const int k = ik[it], r = ir[it];
-        const int i = pp[k], j = qq[k];
-        if (i < 0) continue;
-        const float c = cs[k], s = sn[k];
-        const float ai = A(r, i), aj = A(r, j);
-        A(r, i) = c * ai - s * aj;
-        A(r, j) = s * ai + c * aj;
-        const float vi = V(r, i), vj = V(r, j);
-        V(r, i) = c * vi - s * vj;
-        V(r, j) = s * vi + c * vj;
-      }
-      __syncthreads();
-      // rows: A <- J^T A
-#pragma unroll
-      for (int it = 0; it < kJacItems; ++it) {
-        if (ik[it] < 0) continue;
-        const int k = ik[it], r = ir[it];
-        const int i = pp[k], j = qq[k];
-        if (i < 0) continue;
-        const float c = cs[k], s = sn[k];
-        const float ai = A(i, r), aj = A(j, r);
-        A(i, r) = c * ai - s * aj;
-        A(j, r) = s * ai + c * aj;
-      }
-      __syncthreads();
+      float* t = cur; cur = nxt; nxt = t;
     }
     float so = 0.f;
     for (int e = tid; e < l * l; e += nt) {
       const int i = e / l, j = e % l;
-      if (i != j) so += A(i, j) * A(i, j);
+      if (i != j) so += cur[i * ld + j] * cur[i * ld + j];
     }
     prev = off;
     off = block_sum(so, red);
@@ -980,6 +1027,7 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
     // off-diagonal mass once it is tiny has reached that floor
     if (off <= 1e-12f * frob2 || (off <= 1e-9f * frob2 && off > 0.5f * prev)) { ++sweep; break; }
   }
+#define A(i, j) cur[(i) * ld + (j)]
   if (tid == 0 && sweep >= a.max_sweeps && off > 1e-8f * frob2) raise_flag(a.flags, kFlagNumeric);
   // sort eigenvalues descending, ties by lower index (stable)
   for (int i = tid; i < l; i += nt) {
@@ -1035,6 +1083,7 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
 #undef A
 #undef V
 }
+
 
 // ---------------------------------------------------------------------------
 // Fused apply: T = Psi + Lm R^T (Lm [rows x l], R [cols x l]) and
@@ -1256,8 +1305,8 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
       cudaFuncSetAttribute(k_contract_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kCtcSmem));
     }
   }
-  const int smem = 2 * g.lmax * (g.lmax + 1) * static_cast<int>(sizeof(float));
-  cudaFuncSetAttribute(k_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  // the largest Jacobi footprint, so that groups of any width can share the kernel
+  cudaFuncSetAttribute(k_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kJacSmem));
   return cudaGetLastError();
 }
 
@@ -1306,7 +1355,6 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   const int lp = static_cast<int>(round_up(l, 8));   // register width of the QR solves
   const int cpt = (l + 3) / 4;                         // columns per thread of the contractions
   const int64_t sq = static_cast<int64_t>(g.lmax) * g.lmax;
-  const size_t small_smem = 2 * static_cast<size_t>(l) * (l + 1) * sizeof(float);
   cudaError_t e;
 #define NP_CHECK() do { e = cudaGetLastError(); if (e != cudaSuccess) return e; } while (0)
 
@@ -1437,6 +1485,8 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
         cq.part = go.p; cq.part_bs = go.bs; cq.nsplit = go.n;
         cq.y = src; cq.q = dst; cq.v_bs = vbs;
         cq.n = m_a; cq.l = l; cq.flags = flags;
+        cq.vec = (l % 4 == 0) && (vbs % 4 == 0) && (reinterpret_cast<uintptr_t>(src) % 16 == 0) &&
+                 (reinterpret_cast<uintptr_t>(dst) % 16 == 0);
         if ((e = launch_cholqr(cq, B, lp, s))) return e;
         src = dst;
       }
@@ -1460,8 +1510,11 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       ea.m_a = m_a; ea.n_a = n_a;
       ea.max_sweeps = 30;
       ea.flags = flags;
-      const int jthreads = static_cast<int>(std::min<int64_t>(1024, round_up(static_cast<int64_t>((l + 1) / 2) * l, 32)));
-      k_jacobi<<<B, std::max(jthreads, 32), small_smem, s>>>(ea);
+      const int64_t np2 = static_cast<int64_t>((l + 1) / 2) * ((l + 1) / 2);
+      const int jthreads = static_cast<int>(std::min<int64_t>(1024, round_up(np2, 32)));
+      const int nj = (l + 1) & ~1;
+      const size_t jsmem = 3 * static_cast<size_t>(nj) * (nj + 1) * sizeof(float);
+      k_jacobi<<<B, jthreads, jsmem, s>>>(ea);
       NP_CHECK();
     }
   }
