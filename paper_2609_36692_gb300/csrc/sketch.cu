@@ -888,14 +888,16 @@ __global__ void __launch_bounds__(256) k_rowmul(const __grid_constant__ RowMulAr
 
 // ---------------------------------------------------------------------------
 // Parallel cyclic Jacobi (round-robin pairing) of Gamma_Q in fp32, then the
-// descending sort, the selection C and K.  One CTA per matrix.  A rotation
-// step applies J^T A J as 2 x 2 blocks: the thread that owns block (k, k')
-// (rows of pair k, columns of pair k') computes both rotations from the
-// current copy of A, writes the rotated block into the other copy and rotates
-// two rows of V, so a step is one barrier.  When l is odd the matrices are
-// padded with a zero row and column whose pair is never rotated.
+// descending sort, the selection C and K.  One CTA per matrix; a rotation
+// step has two phases.  First, thread k < n/2 owns pair k (its two players in
+// registers, advanced every step), computes the pair's rotation from the
+// current copy of A and publishes {c, s, i, j}.  Then the thread that owns
+// 2 x 2 block (k, k') of the n/2 x n/2 block grid writes J^T A J for it (rows
+// rotated by pair k, columns by pair k') into the other copy of A and rotates
+// rows k', k' + n/2 of V in pair k's columns.  With two copies of A each
+// phase ends in one barrier.  When l is odd the matrices are padded with a
+// zero row and column whose pair is never rotated.
 // ---------------------------------------------------------------------------
-constexpr int kJacBlocks = ((kLmax / 2) * (kLmax / 2) + 1023) / 1024;   // blocks per thread
 constexpr size_t kJacSmem = 3 * static_cast<size_t>(kLmax) * (kLmax + 1) * sizeof(float);
 struct EigArgs {
   const float* part; int64_t part_bs; int nsplit;   // Gram partials of B^T
@@ -909,28 +911,25 @@ struct EigArgs {
   int max_sweeps;
   int* flags;
 };
-// players (i, j), i < j, of pair k at rotation step `step` of n players
-__device__ __forceinline__ void jac_pair(int k, int step, int n, int& i, int& j) {
-  int p = 0;
-  if (k != 0) { p = k - 1 + step; if (p >= n - 1) p -= n - 1; p += 1; }
-  int q = n - 2 - k + step; if (q >= n - 1) q -= n - 1; q += 1;
-  i = min(p, q);
-  j = max(p, q);
+// threads of k_jacobi for width l: one per 2 x 2 block (two each past 1024 blocks)
+constexpr int kJacBlocks = ((kLmax / 2) * (kLmax / 2) + 1023) / 1024;
+inline int64_t jacobi_threads(int l) {
+  const int64_t np = (l + 1) / 2;
+  return std::min<int64_t>(1024, ((np * np + 31) / 32) * 32);
 }
-// the rotation (c, s) that annihilates A(i, j): t = tan(theta) is the smaller
-// root of t^2 + 2 t cot(2 theta) - 1 = 0, written without cot(2 theta)
-// (t = 2 a_ij sgn(d) / (|d| + sqrt(d^2 + 4 a_ij^2)), d = a_jj - a_ii)
-__device__ __forceinline__ void jac_rot(const float* A, int ld, int i, int j, int l, float& c, float& s) {
-  c = 1.f;
-  s = 0.f;
-  if (j >= l) return;                 // the padding player: not rotated
-  const float apq = A[i * ld + j];
-  if (!(fabsf(apq) > 1e-30f)) return;
-  const float d = A[j * ld + j] - A[i * ld + i];
-  const float num = (d >= 0.f) ? 2.f * apq : -2.f * apq;
-  const float t = __fdividef(num, fabsf(d) + sqrtf(fmaf(d, d, 4.f * apq * apq)));
-  c = rsqrtf(fmaf(t, t, 1.f));
-  s = t * c;
+// the rotation (c, s) that annihilates a_ij: t = tan(theta) is the smaller
+// root of t^2 + 2 t cot(2 theta) - 1 = 0, cot(2 theta) = (a_jj - a_ii) / (2 a_ij)
+__device__ __forceinline__ void jac_rot(float aii, float ajj, float aij, bool pad, float& c, float& s) {
+  // branch-free: both branches of the guard are evaluated, then selected
+  const bool skip = pad || !(fabsf(aij) > 1e-30f);
+  const float th = __fdividef(ajj - aii, 2.f * aij);
+  const float w = fmaf(th, th, 1.f);
+  const float t_far = __fdividef(0.5f, th);    // t -> 1 / (2 cot(2 theta))
+  const float t_near = __fdividef(copysignf(1.f, th), fabsf(th) + w * rsqrtf(w));
+  const float t = fabsf(th) > 1e15f ? t_far : t_near;
+  const float cc = rsqrtf(fmaf(t, t, 1.f));
+  c = skip ? 1.f : cc;
+  s = skip ? 0.f : t * cc;
 }
 __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs a) {
   extern __shared__ float4 jc_smem4[];
@@ -971,7 +970,10 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
     }
     frob2 = block_sum(s, red);
   }
-  // this thread's blocks (k, k'), computed once
+  // pair k plays (p, q) = (k or 0, n - 1 - k) at step 0; every step moves
+  // each player but player 0 on by one place in 1 .. n - 1
+  __shared__ float4 rot4[kLmax / 2];
+  int pk = (tid == 0) ? 0 : tid, qk = n - 1 - tid;
   int bk[kJacBlocks], bk2[kJacBlocks];
 #pragma unroll
   for (int it = 0; it < kJacBlocks; ++it) {
@@ -983,33 +985,41 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
   float off = frob2, prev = frob2;
   for (; sweep < a.max_sweeps; ++sweep) {
     for (int step = 0; step < n - 1; ++step) {
+      if (tid < npairs) {
+        const int i = min(pk, qk), j = max(pk, qk);
+        float c, s;
+        jac_rot(cur[i * ld + i], cur[j * ld + j], cur[i * ld + j], j >= l, c, s);
+        rot4[tid] = make_float4(c, s, __int_as_float(i), __int_as_float(j));
+        if (tid != 0) pk = (pk == n - 1) ? 1 : pk + 1;
+        qk = (qk == n - 1) ? 1 : qk + 1;
+      }
+      __syncthreads();
 #pragma unroll
       for (int it = 0; it < kJacBlocks; ++it) {
-        if (bk[it] < 0) continue;
         const int k = bk[it], k2 = bk2[it];
-        int i, j, i2, j2;
-        jac_pair(k, step, n, i, j);
-        jac_pair(k2, step, n, i2, j2);
-        // the block's entries do not depend on the rotations: load them first
-        const float a00 = cur[i * ld + i2], a01 = cur[i * ld + j2];
-        const float a10 = cur[j * ld + i2], a11 = cur[j * ld + j2];
-        float c, s, c2, s2;
-        jac_rot(cur, ld, i, j, l, c, s);
-        if (k2 == k) { c2 = c; s2 = s; } else { jac_rot(cur, ld, i2, j2, l, c2, s2); }
-        // columns i2, j2 (A J), then rows i, j (J^T A)
-        const float u0 = c2 * a00 - s2 * a01, w0 = s2 * a00 + c2 * a01;
-        const float u1 = c2 * a10 - s2 * a11, w1 = s2 * a10 + c2 * a11;
-        nxt[i * ld + i2] = c * u0 - s * u1;
-        nxt[j * ld + i2] = s * u0 + c * u1;
-        nxt[i * ld + j2] = c * w0 - s * w1;
-        nxt[j * ld + j2] = s * w0 + c * w1;
-        // V <- V J: rows k' and k' + n/2, columns of pair k
+        if (k >= 0) {
+          const float4 r1 = rot4[k], r2 = rot4[k2];
+          const int i = __float_as_int(r1.z), j = __float_as_int(r1.w);
+          const int i2 = __float_as_int(r2.z), j2 = __float_as_int(r2.w);
+          const float c = r1.x, s = r1.y, c2 = r2.x, s2 = r2.y;
+          const float* ri = cur + i * ld;
+          const float* rj = cur + j * ld;
+          const float a00 = ri[i2], a01 = ri[j2], a10 = rj[i2], a11 = rj[j2];
+          // columns i2, j2 (A J), then rows i, j (J^T A)
+          const float u0 = c2 * a00 - s2 * a01, w0 = s2 * a00 + c2 * a01;
+          const float u1 = c2 * a10 - s2 * a11, w1 = s2 * a10 + c2 * a11;
+          float* ni = nxt + i * ld;
+          float* nj = nxt + j * ld;
+          ni[i2] = c * u0 - s * u1; nj[i2] = s * u0 + c * u1;
+          ni[j2] = c * w0 - s * w1; nj[j2] = s * w0 + c * w1;
+          // V <- V J: rows k2 and k2 + n/2, columns of pair k
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int r = k2 + h * npairs;
-          const float vi = V(r, i), vj = V(r, j);
-          V(r, i) = c * vi - s * vj;
-          V(r, j) = s * vi + c * vj;
+          for (int h = 0; h < 2; ++h) {
+            float* vr = Vm + (k2 + h * npairs) * ld;
+            const float vi = vr[i], vj = vr[j];
+            vr[i] = c * vi - s * vj;
+            vr[j] = s * vi + c * vj;
+          }
         }
       }
       __syncthreads();
@@ -1510,8 +1520,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       ea.m_a = m_a; ea.n_a = n_a;
       ea.max_sweeps = 30;
       ea.flags = flags;
-      const int64_t np2 = static_cast<int64_t>((l + 1) / 2) * ((l + 1) / 2);
-      const int jthreads = static_cast<int>(std::min<int64_t>(1024, round_up(np2, 32)));
+      const int jthreads = static_cast<int>(jacobi_threads(l));
       const int nj = (l + 1) & ~1;
       const size_t jsmem = 3 * static_cast<size_t>(nj) * (nj + 1) * sizeof(float);
       k_jacobi<<<B, jthreads, jsmem, s>>>(ea);
