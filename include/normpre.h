@@ -179,7 +179,8 @@ enum normpre_buffer {
                              last step; bf16 in NORMPRE_PREC_BF16 with NORMPRE_G, else fp32 */
   NORMPRE_BUF_T = 1,      /* NormPre-G: Newton-Schulz result T in the stored layout (rows x cols),
                              same dtype as PSI */
-  NORMPRE_BUF_Q = 2,      /* NormPre-L: orthonormal basis Q of the sketch, m_a x l, fp32 */
+  NORMPRE_BUF_Q = 2,      /* NormPre-L: orthonormal basis Q of the sketch, m_a x l, fp32; a column
+                             for a numerically dependent sketch direction (rank(Y) < l) is zero */
   NORMPRE_BUF_RITZ = 3,   /* NormPre-L: all l Ritz values, descending, fp32 (1 x l) */
   NORMPRE_BUF_Z = 4,      /* NormPre-L: Ritz vectors Z (l x l, column j = j-th Ritz value), fp32 */
   NORMPRE_BUF_OMEGA = 5,  /* NormPre-L: sketch matrix Omega of the last step, n_a x l, fp32 */

@@ -748,8 +748,13 @@ __global__ void __launch_bounds__(256) k_gram_fold(const __grid_constant__ GramF
 
 // ---------------------------------------------------------------------------
 // One CholeskyQR pass, fused: every CTA loads the Gram matrix G of Y, factors
-// G = R^T R (upper R, fp32; one diagonal shift when a pivot falls below
-// 1e-6 tr(G)) and then solves q R = y for 256 rows of Y, one row per thread.
+// G = R^T R (upper R, fp32) and then solves q R = y for 256 rows of Y, one
+// row per thread.  A pivot below 1e-6 tr(G) means Y is numerically rank
+// deficient there: the first pass retries with the diagonal shifted by
+// 1e-5 tr(G); the later passes, whose input is already well conditioned
+// wherever it is not rank deficient, drop that column instead (a zero
+// column of q, no elimination with it), so the kept columns stay
+// orthonormal and a dropped one adds a zero Ritz value.
 // The factorization is right-looking over the whole CTA (one pivot per
 // barrier, the trailing square updated by a 16 x 16 thread grid); the solve
 // is column-oriented (x_k final, then every later x_j updated from row k of
@@ -763,6 +768,7 @@ struct CholQRArgs {
   int64_t n;
   int l;
   int vec;       // l % 4 == 0 and 16-byte aligned rows: float4 row loads / stores
+  int drop;      // 0: shifted retry on a small pivot (first pass); 1: drop its column
   int* flags;
 };
 template <int LP>
@@ -796,6 +802,7 @@ __global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRAr
   // for p, q > j (the whole trailing square, so W stays symmetric); row j is
   // final from then on and R[j][i] = W[j][i] / sqrt(W[j][j])
   const int ty = tid >> 4, tx = tid & 15;
+  const float small = 1e-6f * tr;
   bool bad = false;
   for (int attempt = 0; attempt < 2; ++attempt) {
     const float shift = attempt == 0 ? 0.f : 1e-5f * tr;
@@ -807,18 +814,24 @@ __global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRAr
     bad = false;
     for (int j = 0; j < l; ++j) {
       const float d = Wm[j][j];
-      if (!(d > 1e-6f * tr)) bad = true;
-      const float dinv = 1.f / fmaxf(d, 1e-30f * tr);
+      const bool tiny = !(d > small);
+      if (tiny) bad = true;
+      // a dropped column eliminates nothing
+      const float dinv = (tiny && a.drop) ? 0.f : 1.f / fmaxf(d, 1e-30f * tr);
       for (int p = j + 1 + ty; p < l; p += 16) {
         const float wp = Wm[j][p] * dinv;
         for (int c = j + 1 + tx; c < l; c += 16) Wm[p][c] = fmaf(-wp, Wm[j][c], Wm[p][c]);
       }
       __syncthreads();
     }
-    if (!bad) break;     // every thread saw the same pivots
+    if (!bad || a.drop) break;     // every thread saw the same pivots
   }
-  if (tid == 0 && bad && blockIdx.x == 0) raise_flag(a.flags, kFlagNumeric);
-  for (int i = tid; i < LP; i += 256) rinv[i] = (i < l) ? 1.f / sqrtf(fmaxf(Wm[i][i], 1e-30f * tr)) : 0.f;
+  if (tid == 0 && bad && !a.drop && blockIdx.x == 0) raise_flag(a.flags, kFlagNumeric);
+  // W[i][i] is pivot i; a dropped column gets 1 / R_ii = 0 (and so a zero row of R)
+  for (int i = tid; i < LP; i += 256) {
+    const float d = (i < l) ? Wm[i][i] : 0.f;
+    rinv[i] = (i >= l || (a.drop && !(d > small))) ? 0.f : 1.f / sqrtf(fmaxf(d, 1e-30f * tr));
+  }
   __syncthreads();
   for (int e = tid; e < LP * LP; e += 256) {
     const int i = e / LP, j = e % LP;
@@ -1482,8 +1495,9 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       if ((e = contract(ta, g.zt, g.y))) return e;
       ycur = g.y;
     }
-    // Q = qr(Y): three CholeskyQR passes (a pass shifts when its Gram matrix is
-    // numerically singular): y -> q -> zt -> q
+    // Q = qr(Y): three CholeskyQR passes (the first shifts when its Gram matrix
+    // is numerically singular, the others drop numerically dependent
+    // columns): y -> q -> zt -> q
     prof->begin(kProfQR, s);
     {
       const float* src = ycur;
@@ -1497,6 +1511,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
         cq.n = m_a; cq.l = l; cq.flags = flags;
         cq.vec = (l % 4 == 0) && (vbs % 4 == 0) && (reinterpret_cast<uintptr_t>(src) % 16 == 0) &&
                  (reinterpret_cast<uintptr_t>(dst) % 16 == 0);
+        cq.drop = (pass > 0);
         if ((e = launch_cholqr(cq, B, lp, s))) return e;
         src = dst;
       }

@@ -85,6 +85,10 @@ SMALL = S.custom_config("small_mixed", [(128, 384), (128, 128), (128, 512), (512
 RAGGED = S.custom_config("ragged", [(50, 203), (203, 50), (1, 77), (77, 1), (33, 33)],
                          g_dtype="f32", w_dtype="f32", row_sigma=1.0, rank=4, oversample=4)
 SINGLE = S.CONFIGS["single_256x1024"]
+# odd sketch widths (l = 19 and 11): the Jacobi pads a zero row and column,
+# the CholeskyQR rows are not float4-aligned
+ODD = S.custom_config("odd_width", [(96, 160), (160, 96), (19, 300), (250, 11), (45, 45)],
+                      g_dtype="f32", w_dtype="f32", row_sigma=1.0, col_sigma=1.0, rank=13, oversample=6)
 # tall column-active strips: clusters of 4, 8 and 12 CTAs (the last with a
 # partial row block) and one matrix whose column count is not a multiple of 32
 TALL = S.custom_config("tall_cols", [(1000, 40), (4100, 64), (6144, 32), (2056, 24)],
@@ -223,10 +227,48 @@ def _check_l(cs, t, indices=None, w_tol=2e-3):
     return n_checked
 
 
-@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED, ODD], ids=lambda c: c.name)
 @pytest.mark.parametrize("t", [0, 1])
 def test_l_sketch(cfgset, t):
     _check_l(cfgset, t)
+
+
+@pytest.mark.parametrize("t", [0, 1])
+def test_l_rank_deficient_sketch(t):
+    """A rank-2 update with l = 8 (no tangent correction, no prior momentum):
+    the sketch Y has rank 2, so the unshifted Cholesky pivots of its Gram
+    matrix fall below 1e-6 tr and the first CholeskyQR pass takes its shifted
+    retry.  The two selected Ritz directions, their values and the weight
+    update still match the oracle (Householder QR), with no status raised."""
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    shapes = [(64, 96), (96, 64)]
+    cs = S.custom_config("rank2", shapes, g_dtype="f32", w_dtype="f32", rank=4, oversample=4,
+                         prior_momentum=False)
+    mats = [S.make_matrix(cs, i) for i in range(len(shapes))]
+    rng = np.random.default_rng(7)
+    for m in mats:
+        r, c = m["G"].shape
+        m["G"][:] = (rng.standard_normal((r, 2)) @ rng.standard_normal((2, c))).astype(np.float32)
+    W, G, M = to_device(mats, "f32", "f32")
+    opt = _normpre(shapes, ["f32"] * 2, ["f32"] * 2, variant=C.NORMPRE_L, precision=1, rank=4,
+                   oversample=4, seed=1234, tangent=_TANGENT["none"])
+    opt.step(t, LR, W, G, M)
+    torch.cuda.synchronize()
+    assert opt.status() == C.NORMPRE_OK
+    for i in range(len(shapes)):
+        ref = _oracle(mats, i, t, "L", cs, tangent="none")
+        sk = ref["sketch"]
+        st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
+        assert int(st[3]) == sk["n_active"] == 2, (i, st[3], sk["n_active"])
+        ritz = opt.read(i, C.NORMPRE_BUF_RITZ)[0]
+        assert np.max(np.abs(ritz[:2] - sk["ritz"][:2])) <= 1e-4 * sk["ritz"][0], (i, ritz, sk["ritz"])
+        Q = opt.read(i, C.NORMPRE_BUF_Q)
+        Z = opt.read(i, C.NORMPRE_BUF_Z)
+        U = Q.astype(np.float64) @ Z[:, :2].astype(np.float64)
+        assert principal_sine(U, sk["U_C"]) <= 1e-3, i
+        dW = to_host(W[i]).astype(np.float64) - mats[i]["W"]
+        assert rel_fro(dW, ref["W"] - mats[i]["W"]) <= 2e-3, (i, rel_fro(dW, ref["W"] - mats[i]["W"]))
 
 
 @pytest.mark.parametrize("t", [0, 1])
