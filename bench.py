@@ -42,6 +42,7 @@ LR = 0.02
 # (dram__bytes_read.sum + dram__bytes_write.sum), per workload; None until a
 # capture of the current kernel exists (profiles/ keeps the summaries).
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # 80.5 TFLOP/s, for the ALU-bound k_gamma
+L2_BYTES = 129e6                                    # GB300 L2
 
 NCU_TRAFFIC_PER_LAUNCH = {
     "gpt2_small_G": 208.1e6,   # mean of 15 launches: Gram, poly and update of five NS iterations
@@ -300,6 +301,21 @@ def run_ours(args, cfg, variant, rank, world):
     ms_step = ms_total / args.steps
     ms_step = max_over_ranks(ms_step, world, "cuda")
 
+    # ---- per-step distribution: a separate pass with one event pair per step
+    # (row- and column-active steps alternate, so p10 and p90 tell them apart) ----
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    for e_a, e_b in evs:
+        e_a.record(stream)
+        opt.step(t, LR, W, G, M)
+        t += 1
+        e_b.record(stream)
+    torch.cuda.synchronize()
+    per_step = [e_a.elapsed_time(e_b) for e_a, e_b in evs]
+    p10, p50, p90 = (float(v) for v in np.percentile(per_step, [10, 50, 90]))
+    step_dist = {"p10": p10, "p50": p50, "p90": p90, "steps": len(per_step),
+                 "source": "untimed pass after the timed region, one event pair per step"}
+
     # ---- per-kernel-class time of the same workload (events on the launch stream) ----
     C.normpre_profile(h, True)
     for _ in range(args.steps):
@@ -422,11 +438,14 @@ def run_ours(args, cfg, variant, rank, world):
                 "config": {"workload": cfg.name, "variant": variant, "n_mats": cfg.n_mats,
                            "elements": n_el, "ns_steps": cfg.ns_steps if variant == "G" else None,
                            "rank": cfg.rank if variant in ("L", "L_exact") else None,
-                           "l2": "inputs larger than L2 (W, G, M = %.0f MB)" % (h2d / 1e6),
+                           "l2": ("inputs larger than L2 (W, G, M = %.0f MB)" if h2d > L2_BYTES else
+                                  "inputs within L2 (W, G, M = %.0f MB): a latency-scale workload, "
+                                  "not flushed between steps") % (h2d / 1e6),
                            "parallelism": "replicas" if world > 1 else "single"},
                 "e2e": {"value": e2e_ms / world, "unit": "ms", "h2d_bytes_per_step": h2d,
                         "d2h_bytes_per_step": d2h},
                 "gpu_launches": launches,
+                "step_ms": step_dist,
                 "roofline": roof,
                 "normalize": {"achieved": norm_gbs, "peak": hbm, "unit": "GB/s",
                               "frac": (norm_gbs / hbm) if norm_gbs else None,
