@@ -184,7 +184,8 @@ enum normpre_buffer {
   NORMPRE_BUF_RITZ = 3,   /* NormPre-L: all l Ritz values, descending, fp32 (1 x l) */
   NORMPRE_BUF_Z = 4,      /* NormPre-L: Ritz vectors Z (l x l, column j = j-th Ritz value), fp32 */
   NORMPRE_BUF_OMEGA = 5,  /* NormPre-L: sketch matrix Omega of the last step, n_a x l, fp32 */
-  NORMPRE_BUF_STATS = 6,  /* 1 x 8 fp32: [k, m', ||T||_F^2, |C|, l, n_a, m_a, 0] of the last step */
+  NORMPRE_BUF_STATS = 6,  /* 1 x 8 fp32: [k, m', ||T||_F^2, |C|, l, n_a, m_a, s] of the last step,
+                             s = Jacobi sweeps of NormPre-L (0 for NORMPRE_L_EXACT) */
   NORMPRE_BUF_EIGS = 7,   /* NORMPRE_L_EXACT: all m_a eigenvalues of Gamma, descending (1 x m_a) */
   NORMPRE_BUF_DIAG = 8    /* 1 x 8 fp32 diagnostics of the last step: [E_top, E_remain, E_sub,
                              E_global, cos(G, Phi), ||G||_F, ||T||_F, <G, T>].  The spectral
