@@ -233,6 +233,16 @@ def test_l_sketch(cfgset, t):
     _check_l(cfgset, t)
 
 
+@pytest.mark.parametrize("rank,oversample", [(26, 6), (44, 6), (52, 8)], ids=["l32", "l50", "l60"])
+def test_l_sketch_widths(rank, oversample):
+    """Sketch widths between the ones above: l = 32 and 60 take the tensor-core
+    contraction (60: the widest panel, 64 + 64 columns per MMA), l = 50 the
+    SIMT one; the CholeskyQR register widths 32, 56 and 64."""
+    import dataclasses
+    cs = dataclasses.replace(SMALL, rank=rank, oversample=oversample)
+    _check_l(cs, 0)
+
+
 @pytest.mark.parametrize("t", [0, 1])
 def test_l_rank_deficient_sketch(t):
     """A rank-2 update with l = 8 (no tangent correction, no prior momentum):
