@@ -190,16 +190,15 @@ def strict_tangent(Mbar: np.ndarray, Wbar: np.ndarray) -> np.ndarray:
     tangent space of the row direction, which Sec. 3.1 says the relaxed form
     recovers when ||w_i|| = 1 (the "strict tangent" ablation of Table 5a).
     A zero weight row has no direction: x_i = m_i.
-    A momentum row parallel to its weight row has no tangent component; what
-    the subtraction leaves of it is rounding, so a result below 1e-3 of the
-    momentum row's norm is taken as zero (reading; the threshold sits above
-    the fp32 rounding of any row the library accepts, including the
-    cancellation of the column-active closed form ||m||^2 - <m, w>^2 / ||w||^2)."""
+    A momentum row parallel to its weight row has no tangent component, and
+    the fp64 subtraction leaves only rounding of it (about n * 2^-53 of
+    ||m_i|| at most); a result at most 1e-12 of the momentum row's norm is
+    taken as that exact zero (reading: only exact parallelism zeroes a row)."""
     a = np.einsum("ij,ij->i", Mbar, Wbar)
     ww = np.einsum("ij,ij->i", Wbar, Wbar)
     coef = np.divide(a, ww, out=np.zeros_like(a), where=ww > 0)
     X = Mbar - coef[:, None] * Wbar
-    tiny = np.linalg.norm(X, axis=1) <= 1e-3 * np.linalg.norm(Mbar, axis=1)
+    tiny = np.linalg.norm(X, axis=1) <= 1e-12 * np.linalg.norm(Mbar, axis=1)
     X[tiny] = 0.0
     return X
 
@@ -253,16 +252,6 @@ def newton_schulz(Psi: np.ndarray, steps: int = 5, coef=MUON_QUINTIC, eps: float
         B = b * A + c * (A @ A)
         X = a * X + B @ X
     return X.T if tall else X
-
-
-def ns_scalar_map(x: np.ndarray, steps: int = 5, coef=MUON_QUINTIC) -> np.ndarray:
-    """The singular-value map of ``newton_schulz``: p(x) = a x + b x^3 + c x^5,
-    applied ``steps`` times (each iteration acts on every singular value alone)."""
-    a, b, c = (float(v) for v in coef)
-    y = np.asarray(x, dtype=np.float64)
-    for _ in range(steps):
-        y = a * y + b * y ** 3 + c * y ** 5
-    return y
 
 
 def _descending(lam: np.ndarray, vecs: np.ndarray):
@@ -424,7 +413,7 @@ __all__ = [
     "MUON_QUINTIC", "OracleConfig", "philox4x32_10", "philox_uniform", "sketch_omega",
     "momentum_update", "orientation_of", "orient", "relaxed_tangent", "strict_tangent", "tangent_step",
     "diag_gram_normalize", "both_axes_normalize",
-    "newton_schulz", "ns_scalar_map", "interaction_sketch", "exact_interaction_eigs",
+    "newton_schulz", "interaction_sketch", "exact_interaction_eigs",
     "localized_apply", "rms_matched", "weight_update", "normpre_step", "muon_step",
     "spectral_energies", "descent_alignment",
 ]

@@ -510,6 +510,24 @@ def test_strict_tangent_of_a_parallel_row_is_zero():
     assert np.all(X1 == 0.0)
 
 
+def test_strict_tangent_keeps_a_small_tangent_part():
+    """Only exact parallelism zeroes a row: a momentum row whose tangent part is
+    1e-6 or 1e-9 of its norm keeps exactly that part (the projection of Sec. 3.1
+    is linear), and normalizes to the unit tangent direction (Eq. 3)."""
+    rng = _rng(43)
+    w = rng.standard_normal(300)
+    v = rng.standard_normal(300)
+    v -= (v @ w) / (w @ w) * w                 # tangent direction, orthogonal to w
+    v /= np.linalg.norm(v)
+    for eps in (1e-6, 1e-9):
+        m = 2.5 * w / np.linalg.norm(w) + eps * 2.5 * v
+        X = O.strict_tangent(m[None, :], w[None, :])
+        np.testing.assert_allclose(X[0], eps * 2.5 * v, atol=1e-14, rtol=0)
+        Psi, d = O.diag_gram_normalize(X)
+        np.testing.assert_allclose(Psi[0], v, atol=1e-5 if eps == 1e-9 else 1e-8)
+        assert d[0] > 0
+
+
 # --------------------------------------------------------------------------
 # Diagnostics (App. E)
 # --------------------------------------------------------------------------
