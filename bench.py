@@ -1,21 +1,29 @@
 #!/usr/bin/env python
 """Benchmark of one NormPre optimizer step over a synthetic model parameter set.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--config NAME]
+    python bench.py [--steps K] [--warmup W] [--impl ours|reference]
+                    [--config NAME] [--variant G|L|L_exact]
 
 A step is the whole hot path (momentum, relaxed tangent, diagonal-Gram
 normalization, spectral preconditioning, RMS-matched weight update with decay)
-over every matrix of the parameter set.  Default workload: the GPT-2 Small
-hidden matrices under NormPre-G (48 matrices, 84.9 M parameters, bf16
-gradients, fp32 weights and momentum, 5 Newton-Schulz iterations).
+over every matrix of the parameter set.  Default workload: the Qwen3 ~1.7B
+hidden matrices (196 matrices, 1.41 G parameters, bf16 gradients and weights,
+fp32 momentum), the largest parameter set that the paper measures on one
+device's worth of matrices.  The default run measures NormPre-G (5 Newton-
+Schulz iterations, the line's own keys) and NormPre-L (r = 32, o = 8, p = 1,
+under ``variants.L``) on it.
 
 Prints one JSON line: `value` is the device-timed ms per parameter-set step
 (inputs resident in HBM), `e2e` the same step through the C ABI on pinned host
 buffers with the copies inside the timed region, `roofline` the dominant
-kernel class (the Newton-Schulz GEMMs for NormPre-G) against the measured
-peak, `cpu_baseline` the fp64 oracle on the host cores for a bounded sample.
-`--impl reference` times the oracle itself on the same workload.
+kernel class (the Newton-Schulz GEMMs for NormPre-G, the sketch contractions
+for NormPre-L) against the measured peak, `cpu_baseline` the fp64 oracle on
+the host cores for a bounded sample.  `--impl reference` times the oracle
+itself on the same workload.
+
+The library runs on one GPU: the step has no exchange between matrices and
+the workload fixes a single device, so there is no multi-GPU launch path;
+`--impl ours` refuses `--gpus` > 1 or a process group of more than one rank.
 """
 from __future__ import annotations
 
@@ -36,17 +44,17 @@ sys.path.insert(0, ROOT)
 from synth import inputs as S  # noqa: E402
 
 METRIC = "NormPre step ms per model param set; NS TFLOP/s & normalize GB/s vs peak"
-DEFAULT_CONFIG = "gpt2_small_G"
+DEFAULT_CONFIG = "qwen3_1p7b"
 LR = 0.02
-# Traffic of one launch of the dominant kernel class from an ncu capture
-# (dram__bytes_read.sum + dram__bytes_write.sum), per workload; None until a
-# capture of the current kernel exists (profiles/ keeps the summaries).
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # 80.5 TFLOP/s, for the ALU-bound k_gamma
 L2_BYTES = 129e6                                    # GB300 L2
 
+# Traffic of one launch of the dominant kernel class from an ncu capture
+# (dram__bytes_read.sum + dram__bytes_write.sum), per workload and variant;
+# absent until a capture of the current kernel exists (profiles/ keeps the
+# summaries).
 NCU_TRAFFIC_PER_LAUNCH = {
-    "gpt2_small_G": 208.1e6,   # mean of 15 launches: Gram, poly and update of five NS iterations
-    "gpt2_small_L": 108.0e6,   # mean of six k_contract_tc launches (both operand orientations)
+    ("gpt2_small_G", "G"): 208.1e6,   # mean of 15 launches: Gram, poly and update of five NS iterations
 }
 
 
@@ -62,7 +70,7 @@ def measured_peaks():
 
 
 def ns_flops(cfg: S.ParamSetConfig, steps: int) -> float:
-    """Algorithmic Newton-Schulz flops of one step: per iteration and matrix
+    """Nominal Newton-Schulz flops of one step: per iteration and matrix
     2 s^2 big (Gram) + 2 s^3 (A A) + 2 s^2 big (B X), s = min(m, n)."""
     tot = 0.0
     for m in cfg.matrices:
@@ -155,46 +163,65 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(self.rows)}
 
 
-def max_over_ranks(x: float, world: int, device: str) -> float:
-    """The largest value over the ranks of the process group (the job's time
-    is its slowest rank's); x itself when there is one rank."""
-    if world <= 1:
-        return x
-    import torch
-    import torch.distributed as dist
-    tt = torch.tensor([x], dtype=torch.float64, device=device)
-    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-    return float(tt.item())
-
-
-def oracle_sample(cfg: S.ParamSetConfig, variant: str, seconds_budget: float = 20.0):
-    """Times the fp64 oracle on a bounded sample of the workload (one layer's
-    matrices of each distinct shape) and scales to the whole parameter set by
-    matrix counts.  Returns (ms per parameter set, description, cores)."""
-    import oracle as O
-    from synth.inputs import make_matrix
+def sample_combos(cfg: S.ParamSetConfig):
+    """The (shape, orientation) pairs the CPU oracle is timed on: one matrix of
+    each distinct shape, at t = 0 (row-active) and t = 1 (column-active)."""
     shapes = {}
     for i, m in enumerate(cfg.matrices):
         shapes.setdefault((m.rows, m.cols), []).append(i)
+    return [(shp, idx, t) for shp, idx in shapes.items() for t in (0, 1)]
+
+
+def oracle_time(cfg: S.ParamSetConfig, variant: str, combo) -> float:
+    """Wall ms of the fp64 oracle's step on one matrix (one (shape, t) pair)."""
+    import oracle as O
+    from synth.inputs import make_matrix
+    shp, idx, t = combo
     oc = O.OracleConfig(variant=variant, rank=cfg.rank, oversample=0 if variant == "L_exact" else cfg.oversample,
                         power_iters=cfg.power_iters, seed=1234)
-    total_ms = 0.0
-    sampled = []
-    for shp, idx in shapes.items():
-        mats = make_matrix(cfg, idx[0])
-        t0 = time.perf_counter()
-        O.normpre_step(mats["W"], mats["G"], mats["M"], 0, LR, oc, matrix_id=idx[0])
-        dt = (time.perf_counter() - t0) * 1e3
-        total_ms += dt * len(idx)
-        sampled.append("%dx%d" % shp)
+    mats = make_matrix(cfg, idx[0])
+    t0 = time.perf_counter()
+    O.normpre_step(mats["W"], mats["G"], mats["M"], t, LR, oc, matrix_id=idx[0])
+    return (time.perf_counter() - t0) * 1e3
+
+
+def oracle_set_estimate(cfg: S.ParamSetConfig, timed: dict) -> float:
+    """ms of one parameter-set step from per-(shape, t) oracle times: every
+    shape's time averaged over the orientations measured, times the number of
+    matrices of that shape."""
+    tot = 0.0
+    by_shape = {}
+    for (shp, idx, t), ms in timed.items():
+        by_shape.setdefault((shp, len(idx)), []).append(ms)
+    for (shp, count), v in by_shape.items():
+        tot += count * float(np.mean(v))
+    return tot
+
+
+def host_cores() -> int:
     try:
         from threadpoolctl import threadpool_info
-        cores = max([d.get("num_threads", 1) for d in threadpool_info()] + [1])
+        return max([d.get("num_threads", 1) for d in threadpool_info()] + [1])
     except Exception:
-        cores = os.cpu_count() or 1
-    desc = ("oracle (numpy fp64) on one matrix of each distinct shape (%s), scaled by the matrix "
-            "count of each shape to the %d-matrix set" % (", ".join(sampled), cfg.n_mats))
-    return total_ms, desc, cores
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(cfg: S.ParamSetConfig, variant: str):
+    """The oracle as it stands on the host cores: one matrix of each distinct
+    shape at both orientations, extrapolated to the set by matrix counts."""
+    timed = {}
+    t0 = time.perf_counter()
+    for combo in sample_combos(cfg):
+        timed[(combo[0], tuple(combo[1]), combo[2])] = oracle_time(cfg, variant, combo)
+    wall = time.perf_counter() - t0
+    ms = oracle_set_estimate(cfg, timed)
+    shapes = sorted({"%dx%d" % k[0] for k in timed})
+    return {"value": ms, "unit": "ms", "cores": host_cores(), "kind": "oracle",
+            "extrapolated_from_sample": True, "sample_wall_s": wall,
+            "sample": ("numpy fp64 oracle, variant %s, on one matrix of each distinct shape (%s) at t = 0 "
+                       "and t = 1 (%.1f s of CPU work); each shape's time, averaged over the two "
+                       "orientations, times its matrix count in the %d-matrix set"
+                       % (variant, ", ".join(shapes), wall, cfg.n_mats))}
 
 
 # ---------------------------------------------------------------------------
@@ -203,21 +230,31 @@ def oracle_sample(cfg: S.ParamSetConfig, variant: str, seconds_budget: float = 2
 def run_reference(args, cfg, variant, rank, world):
     if rank != 0:
         return
-    for _ in range(args.warmup):
-        oracle_sample(cfg, variant)
-    times = []
-    desc, cores = "", 1
-    for _ in range(args.steps):
-        ms, desc, cores = oracle_sample(cfg, variant)
-        times.append(ms)
-    v = float(np.mean(times))
+    combos = sample_combos(cfg)
+    # every step times one (shape, orientation) pair in rotation; the set
+    # estimate uses each pair's mean over the timed steps
+    for i in range(args.warmup):
+        oracle_time(cfg, variant, combos[i % len(combos)])
+    timed = {}
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        c = combos[i % len(combos)]
+        timed.setdefault((c[0], tuple(c[1]), c[2]), []).append(oracle_time(cfg, variant, c))
+    wall = time.perf_counter() - t0
+    v = oracle_set_estimate(cfg, {k: float(np.mean(x)) for k, x in timed.items()})
+    covered = len(timed)
+    desc = ("numpy fp64 oracle, variant %s: each timed step runs one matrix of one distinct shape at one "
+            "orientation, in rotation over the %d (shape, t) pairs (%d covered, %.1f s of timed CPU work); "
+            "value = each shape's mean time over the orientations measured times its matrix count"
+            % (variant, len(combos), covered, wall))
     line = {"metric": METRIC, "value": v, "unit": "ms", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": v, "higher_is_better": False, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
             "config": {"workload": cfg.name, "variant": variant, "n_mats": cfg.n_mats,
                        "elements": cfg.elements},
-            "cpu_baseline": {"value": v, "unit": "ms", "cores": cores, "kind": "oracle", "sample": desc},
+            "cpu_baseline": {"value": v, "unit": "ms", "cores": host_cores(), "kind": "oracle",
+                             "extrapolated_from_sample": True, "sample_wall_s": wall, "sample": desc},
             "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -225,24 +262,74 @@ def run_reference(args, cfg, variant, rank, world):
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
-def run_ours(args, cfg, variant, rank, world):
-    import torch
-    import torch.distributed as dist
+def _roofline(cfg, variant, prof, steps, clocks):
+    hbm, bf16_burst, bf16_sust, peak_src = measured_peaks()
+    n_el = cfg.elements
+    if variant == "G":
+        fl = ns_flops(cfg, cfg.ns_steps)
+        fl_exec = ns_executed_flops(cfg, cfg.ns_steps)
+        ns_ms = sum(prof[k][0] for k in ("ns_gram", "ns_poly", "ns_update")) / steps
+        ns_launches = sum(prof[k][1] for k in ("ns_gram", "ns_poly", "ns_update")) / steps
+        achieved = fl_exec / (ns_ms * 1e-3) / 1e12
+        # a step that ran into the power cap is held to the sustained matmul rate
+        capped = "sw_power_cap" in clocks.get("reasons", [])
+        peak = bf16_sust if capped else bf16_burst
+        return {"bound": "tensor", "kernel": "k_ns_gemm_tc (Newton-Schulz Gram / poly / update)",
+                "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "peak_source": "%s bf16 %s" % (peak_src, "sustained (sw_power_cap seen in the timed region)"
+                                               if capped else "burst"),
+                "flops_note": "executed flops: padded shapes, only the tiles on or above the diagonal of "
+                              "the two symmetric products (the mirror is copied, not multiplied)",
+                "flops_per_launch": fl_exec / ns_launches, "ms_per_launch": ns_ms / ns_launches,
+                "launches_per_step": ns_launches,
+                "nominal_flops_per_launch": fl / ns_launches,
+                "achieved_nominal": fl / (ns_ms * 1e-3) / 1e12,
+                "frac_nominal": fl / (ns_ms * 1e-3) / 1e12 / peak,
+                "traffic": NCU_TRAFFIC_PER_LAUNCH.get((cfg.name, variant))}
+    if variant == "L_exact":
+        # k_gamma: Gamma = Psi_a Psi_a^T on the fp32 FMA pipes (both triangles,
+        # 2 m_a^2 n_a flops per matrix); the dense eigensolver is a library call
+        gam_ms = prof["gamma"][0] / steps
+        gam_launches = prof["gamma"][1] / steps
+        k_even = sum(2.0 * m.rows * m.rows * m.cols for m in cfg.matrices)
+        k_odd = sum(2.0 * m.cols * m.cols * m.rows for m in cfg.matrices)
+        fl = (k_even + k_odd) / 2.0          # row- and column-active steps alternate
+        achieved = fl / (gam_ms * 1e-3) / 1e12
+        return {"bound": "alu", "kernel": "k_gamma (Gamma = Psi_a Psi_a^T, fp32 FMA)",
+                "achieved": achieved, "peak": FP32_FMA_TFLOPS, "unit": "TFLOP/s",
+                "frac": achieved / FP32_FMA_TFLOPS,
+                "peak_source": "nominal fp32 FMA rate: 152 SMs x 128 lanes x 2 flops x 2.07 GHz",
+                "flops_per_launch": fl / gam_launches, "ms_per_launch": gam_ms / gam_launches,
+                "launches_per_step": gam_launches,
+                "syevd_ms_per_step": prof["syevd"][0] / steps,
+                "traffic": None}
+    con_ms = prof["contract"][0] / steps
+    con_launches = prof["contract"][1] / steps
+    # each contraction streams the fp32 Psi of its group once: Y0 = Psi Omega,
+    # Psi^T Y and Psi Z per power iteration, B = Q^T Psi
+    nbytes = n_el * 4.0 * (2 + 2 * cfg.power_iters)
+    achieved = nbytes / (con_ms * 1e-3) / 1e9
+    return {"bound": "hbm", "kernel": "k_contract_tc (sketch contractions of Psi, tcgen05 TF32 split)",
+            "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+            "peak_source": "%s HBM copy bandwidth" % peak_src,
+            "bytes_per_launch": nbytes / con_launches, "ms_per_launch": con_ms / con_launches,
+            "launches_per_step": con_launches,
+            "traffic": NCU_TRAFFIC_PER_LAUNCH.get((cfg.name, variant))}
 
-    from paper_2609_36692_gb300 import build as B
-    B.build()
+
+def measure_variant(args, cfg, variant, host, dev):
+    """Device-timed steps, per-step spread, per-kernel-class times and the
+    host-buffer (e2e) step of one variant on fresh copies of the inputs."""
+    import torch
+
     from paper_2609_36692_gb300 import normpre as C
     from paper_2609_36692_gb300.optim import NormPre
 
-    dev = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(dev)
+    Wh, Gh, Mh = host
+    W = [x.to("cuda", non_blocking=False) for x in Wh]
+    G = [x.to("cuda", non_blocking=False) for x in Gh]
+    M = [x.to("cuda", non_blocking=False) for x in Mh]
     stream = torch.cuda.current_stream()
-
-    mats = S.make_param_set(cfg, workers=min(16, os.cpu_count() or 1))
-    tdt = {"f32": torch.float32, "bf16": torch.bfloat16}
-    W = [torch.from_numpy(m["W"]).to(tdt[cfg.w_dtype]).cuda() for m in mats]
-    G = [torch.from_numpy(m["G"]).to(tdt[cfg.g_dtype]).cuda() for m in mats]
-    M = [torch.from_numpy(m["M"]).cuda() for m in mats]
     prec = C.NORMPRE_PREC_BF16 if variant == "G" else C.NORMPRE_PREC_F32
     vcode = {"G": C.NORMPRE_G, "L": C.NORMPRE_L, "L_exact": C.NORMPRE_L_EXACT}[variant]
     opt = NormPre([(m.rows, m.cols) for m in cfg.matrices], [cfg.w_dtype] * cfg.n_mats,
@@ -250,24 +337,19 @@ def run_ours(args, cfg, variant, rank, world):
                   precision=prec, rank=cfg.rank, oversample=cfg.oversample,
                   power_iters=cfg.power_iters, ns_steps=cfg.ns_steps, seed=1234)
     h = opt.handle
-
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
+    warm = max(args.warmup, 3)
     sampler = ClockSampler(gpu_index=dev)
     t = 0
-    for _ in range(max(args.warmup, 3)):
+    for _ in range(warm):
         opt.step(t, LR, W, G, M)
         t += 1
     torch.cuda.synchronize()
     opt.status()
-    C.normpre_profile_read(h)           # reset launch counters
+    C.normpre_profile_read(h)           # reset the launch counters
 
     # ---- timed region: K steps, inputs resident in HBM (> L2 in total) ----
     sampler.start()
     time.sleep(0.1)                     # let the sampler's first query land
-    barrier()
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
@@ -276,10 +358,9 @@ def run_ours(args, cfg, variant, rank, world):
         t += 1
     ev1.record(stream)
     torch.cuda.synchronize()
-    barrier()
     ms_total = ev0.elapsed_time(ev1)
     sampler.stop()
-    counts = C.normpre_profile_read(h)
+    counts = C.normpre_profile_read(h)  # launches of the timed region; resets the counters
     launches = int(sum(c for _, c in counts.values()))
     opt.status()
     clocks = sampler.summary()
@@ -299,7 +380,6 @@ def run_ours(args, cfg, variant, rank, world):
         clocks = soak.summary()
         clocks["source"] = "1.5 s soak of the same step right after the timed region (too short to sample)"
     ms_step = ms_total / args.steps
-    ms_step = max_over_ranks(ms_step, world, "cuda")
 
     # ---- per-step distribution: a separate pass with one event pair per step
     # (row- and column-active steps alternate, so p10 and p90 tell them apart) ----
@@ -317,6 +397,7 @@ def run_ours(args, cfg, variant, rank, world):
                  "source": "untimed pass after the timed region, one event pair per step"}
 
     # ---- per-kernel-class time of the same workload (events on the launch stream) ----
+    C.normpre_profile_read(h)           # counters start at zero for the profiled pass
     C.normpre_profile(h, True)
     for _ in range(args.steps):
         opt.step(t, LR, W, G, M)
@@ -325,137 +406,137 @@ def run_ours(args, cfg, variant, rank, world):
     prof = C.normpre_profile_read(h)
     C.normpre_profile(h, False)
 
-    hbm, bf16_burst, bf16_sust, peak_src = measured_peaks()
+    hbm = measured_peaks()[0]
     n_el = cfg.elements
     b_norm, b_apply = bytes_per_elt(cfg, variant)
     norm_ms = prof["normalize"][0] / args.steps
     phases = {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps}
               for k, v in prof.items() if v[1] > 0}
-    if variant == "G":
-        fl = ns_flops(cfg, cfg.ns_steps)
-        fl_exec = ns_executed_flops(cfg, cfg.ns_steps)
-        ns_ms = sum(prof[k][0] for k in ("ns_gram", "ns_poly", "ns_update")) / args.steps
-        ns_launches = sum(prof[k][1] for k in ("ns_gram", "ns_poly", "ns_update")) / args.steps
-        achieved = fl / (ns_ms * 1e-3) / 1e12
-        # a step that ran into the power cap is held to the sustained matmul rate
-        capped = "sw_power_cap" in clocks.get("reasons", [])
-        peak = bf16_sust if capped else bf16_burst
-        roof = {"bound": "tensor", "kernel": "k_ns_gemm_tc (Newton-Schulz Gram / poly / update)",
-                "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak,
-                "peak_source": "%s bf16 %s" % (peak_src, "sustained (sw_power_cap seen in the timed region)"
-                                                if capped else "burst"),
-                "flops_per_launch": fl / ns_launches, "ms_per_launch": ns_ms / ns_launches,
-                "flops_note": "nominal dense flops (full Gram); the kernel computes only the "
-                              "tiles on or above the diagonal of the two symmetric products",
-                "executed_flops_per_launch": fl_exec / ns_launches,
-                "achieved_executed": fl_exec / (ns_ms * 1e-3) / 1e12,
-                "frac_executed": fl_exec / (ns_ms * 1e-3) / 1e12 / peak,
-                "traffic": NCU_TRAFFIC_PER_LAUNCH.get(cfg.name)}
-    elif variant == "L_exact":
-        # k_gamma: Gamma = Psi_a Psi_a^T on the fp32 FMA pipes (both triangles,
-        # 2 m_a^2 n_a flops per matrix); the dense eigensolver is a library call
-        gam_ms = prof["gamma"][0] / args.steps
-        gam_launches = prof["gamma"][1] / args.steps
-        k_even = sum(2.0 * m.rows * m.rows * m.cols for m in cfg.matrices)
-        k_odd = sum(2.0 * m.cols * m.cols * m.rows for m in cfg.matrices)
-        fl = (k_even + k_odd) / 2.0          # row- and column-active steps alternate
-        achieved = fl / (gam_ms * 1e-3) / 1e12
-        fp32_peak = FP32_FMA_TFLOPS
-        roof = {"bound": "alu", "kernel": "k_gamma (Gamma = Psi_a Psi_a^T, fp32 FMA)",
-                "achieved": achieved, "peak": fp32_peak, "unit": "TFLOP/s", "frac": achieved / fp32_peak,
-                "peak_source": "nominal fp32 FMA rate: 152 SMs x 128 lanes x 2 flops x 2.07 GHz",
-                "flops_per_launch": fl / gam_launches, "ms_per_launch": gam_ms / gam_launches,
-                "syevd_ms_per_step": prof["syevd"][0] / args.steps,
-                "traffic": None}
-    else:
-        con_ms = prof["contract"][0] / args.steps
-        con_launches = prof["contract"][1] / args.steps
-        # each contraction streams the fp32 Psi of its group once: Y0 = Psi Omega,
-        # Psi^T Y and Psi Z per power iteration, B = Q^T Psi
-        nbytes = n_el * 4.0 * (2 + 2 * cfg.power_iters)
-        achieved = nbytes / (con_ms * 1e-3) / 1e9
-        roof = {"bound": "hbm", "kernel": "k_contract_tc (sketch contractions of Psi, tcgen05 TF32 split)",
-                "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                "peak_source": "%s HBM copy bandwidth" % peak_src,
-                "bytes_per_launch": nbytes / con_launches, "ms_per_launch": con_ms / con_launches,
-                "traffic": NCU_TRAFFIC_PER_LAUNCH.get(cfg.name)}
+    roof = _roofline(cfg, variant, prof, args.steps, clocks)
     norm_gbs = n_el * b_norm / (norm_ms * 1e-3) / 1e9 if norm_ms > 0 else None
 
     # ---- end to end through the C ABI on pinned host buffers ----
-    Wh = [torch.from_numpy(m["W"]).to(tdt[cfg.w_dtype]).pin_memory() for m in mats]
-    Gh = [torch.from_numpy(m["G"]).to(tdt[cfg.g_dtype]).pin_memory() for m in mats]
-    Mh = [torch.from_numpy(m["M"]).pin_memory() for m in mats]
     h2d = sum(x.numel() * x.element_size() for x in Wh + Gh + Mh)
     d2h = sum(x.numel() * x.element_size() for x in Wh + Mh)
-    opt.step_host(t, LR, Wh, Gh, Mh)
+    del W, G, M
+    torch.cuda.empty_cache()
+    Wh2 = [x.clone().pin_memory() for x in Wh]
+    Mh2 = [x.clone().pin_memory() for x in Mh]
+    opt.step_host(t, LR, Wh2, Gh, Mh2)
     t += 1
-    barrier()
+    torch.cuda.synchronize()
     n_e2e = max(3, min(args.steps, 20))
     t0 = time.perf_counter()
     for _ in range(n_e2e):
-        opt.step_host(t, LR, Wh, Gh, Mh)
+        opt.step_host(t, LR, Wh2, Gh, Mh2)
         t += 1
     e2e_ms = (time.perf_counter() - t0) * 1e3 / n_e2e
-    e2e_ms = max_over_ranks(e2e_ms, world, "cuda")
-
-    # ---- the paper's comparison optimizer (Muon) on the same workload and kernels ----
-    muon = None
-    if not args.no_muon:
-        opt_m = NormPre([(m.rows, m.cols) for m in cfg.matrices], [cfg.w_dtype] * cfg.n_mats,
-                        [cfg.g_dtype] * cfg.n_mats, variant=C.NORMPRE_MUON, precision=C.NORMPRE_PREC_BF16,
-                        ns_steps=cfg.ns_steps)
-        for _ in range(max(args.warmup, 3)):
-            opt_m.step(t, LR, W, G, M)
-            t += 1
-        torch.cuda.synchronize()
-        barrier()
-        ev0.record(stream)
-        for _ in range(args.steps):
-            opt_m.step(t, LR, W, G, M)
-            t += 1
-        ev1.record(stream)
-        torch.cuda.synchronize()
-        ms_muon = ev0.elapsed_time(ev1) / args.steps
-        opt_m.status()
-        opt_m.close()
-        ms_muon = max_over_ranks(ms_muon, world, "cuda")
-        muon = {"ms_per_step": ms_muon, "normpre_vs_muon": ms_step / ms_muon - 1.0,
-                "paper_a100_context": "optimizer latency vs Muon on A100: NormPre-G +5.76 % / +4.37 % / +6.77 %, "
-                                      "NormPre-L -38.12 % / -67.00 % / -57.16 % (GPT-2 Small / LLaMA-1.3B / "
-                                      "Qwen3-1.7B, whole optimizer step incl. AdamW on the other parameters)"}
-
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        ms_cpu, desc, cores = oracle_sample(cfg, variant)
-        cpu = {"value": ms_cpu, "unit": "ms", "cores": cores, "kind": "oracle", "sample": desc}
-
-    if rank == 0:
-        line = {"metric": METRIC, "value": ms_step / world, "unit": "ms", "n_gpus": world,
-                "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_step,
-                "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
-                "dtype": "bf16" if variant == "G" else "f32", "data": "synthetic",
-                "config": {"workload": cfg.name, "variant": variant, "n_mats": cfg.n_mats,
-                           "elements": n_el, "ns_steps": cfg.ns_steps if variant == "G" else None,
-                           "rank": cfg.rank if variant in ("L", "L_exact") else None,
-                           "l2": ("inputs larger than L2 (W, G, M = %.0f MB)" if h2d > L2_BYTES else
-                                  "inputs within L2 (W, G, M = %.0f MB): a latency-scale workload, "
-                                  "not flushed between steps") % (h2d / 1e6),
-                           "parallelism": "replicas" if world > 1 else "single"},
-                "e2e": {"value": e2e_ms / world, "unit": "ms", "h2d_bytes_per_step": h2d,
-                        "d2h_bytes_per_step": d2h},
-                "gpu_launches": launches,
-                "step_ms": step_dist,
-                "roofline": roof,
-                "normalize": {"achieved": norm_gbs, "peak": hbm, "unit": "GB/s",
-                              "frac": (norm_gbs / hbm) if norm_gbs else None,
-                              "bytes_per_element": b_norm},
-                "phases": phases,
-                "muon": muon,
-                "cpu_baseline": cpu,
-                "clocks": clocks}
-        print(json.dumps(line), flush=True)
+    opt.status()
     opt.close()
+    del Wh2, Mh2
+    torch.cuda.empty_cache()
+    return {"ms_per_step": ms_step, "warmup": warm, "launches": launches, "clocks": clocks,
+            "step_ms": step_dist, "roofline": roof,
+            "normalize": {"achieved": norm_gbs, "peak": hbm, "unit": "GB/s",
+                          "frac": (norm_gbs / hbm) if norm_gbs else None, "bytes_per_element": b_norm},
+            "phases": phases,
+            "e2e": {"value": e2e_ms, "unit": "ms", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "steps": n_e2e, "timer": "host wall clock around normpre_step_host (synchronous)"}}
+
+
+def measure_muon(args, cfg, host):
+    """The paper's comparison optimizer on the same matrices and kernels."""
+    import torch
+
+    from paper_2609_36692_gb300 import normpre as C
+    from paper_2609_36692_gb300.optim import NormPre
+
+    Wh, Gh, Mh = host
+    W = [x.to("cuda") for x in Wh]
+    G = [x.to("cuda") for x in Gh]
+    M = [x.to("cuda") for x in Mh]
+    stream = torch.cuda.current_stream()
+    opt = NormPre([(m.rows, m.cols) for m in cfg.matrices], [cfg.w_dtype] * cfg.n_mats,
+                  [cfg.g_dtype] * cfg.n_mats, variant=C.NORMPRE_MUON, precision=C.NORMPRE_PREC_BF16,
+                  ns_steps=cfg.ns_steps)
+    t = 0
+    for _ in range(max(args.warmup, 3)):
+        opt.step(t, LR, W, G, M)
+        t += 1
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        opt.step(t, LR, W, G, M)
+        t += 1
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    opt.status()
+    opt.close()
+    del W, G, M
+    torch.cuda.empty_cache()
+    return ms
+
+
+def run_ours(args, cfg, variants):
+    import torch
+
+    from paper_2609_36692_gb300 import build as B
+    B.build()
+
+    dev = 0
+    torch.cuda.set_device(dev)
+    mats = S.make_param_set(cfg, workers=min(16, os.cpu_count() or 1))
+    tdt = {"f32": torch.float32, "bf16": torch.bfloat16}
+    Wh = [torch.from_numpy(m["W"]).to(tdt[cfg.w_dtype]).pin_memory() for m in mats]
+    Gh = [torch.from_numpy(m["G"]).to(tdt[cfg.g_dtype]).pin_memory() for m in mats]
+    Mh = [torch.from_numpy(m["M"]).pin_memory() for m in mats]
+    del mats
+    host = (Wh, Gh, Mh)
+
+    res = {v: measure_variant(args, cfg, v, host, dev) for v in variants}
+    muon_ms = None if args.no_muon else measure_muon(args, cfg, host)
+    ctx = ("optimizer latency vs Muon on A100: NormPre-G +5.76 % / +4.37 % / +6.77 %, NormPre-L -38.12 % / "
+           "-67.00 % / -57.16 % (GPT-2 Small / LLaMA-1.3B / Qwen3-1.7B, whole optimizer step incl. AdamW "
+           "on the other parameters)")
+    for v, r in res.items():
+        r["muon"] = None if muon_ms is None else {
+            "ms_per_step": muon_ms, "normpre_vs_muon": r["ms_per_step"] / muon_ms - 1.0,
+            "paper_a100_context": ctx}
+        r["cpu_baseline"] = None if args.no_cpu_baseline else cpu_baseline(cfg, v)
+
+    def config_of(v):
+        return {"workload": cfg.name, "variant": v, "n_mats": cfg.n_mats, "elements": cfg.elements,
+                "ns_steps": cfg.ns_steps if v == "G" else None,
+                "rank": cfg.rank if v in ("L", "L_exact") else None,
+                "oversample": cfg.oversample if v == "L" else None,
+                "power_iters": cfg.power_iters if v == "L" else None,
+                "l2": ("inputs larger than L2 (W, G, M = %.0f MB)" if res[v]["e2e"]["h2d_bytes_per_step"] >
+                       L2_BYTES else "inputs within L2 (W, G, M = %.0f MB): a latency-scale workload, not "
+                       "flushed between steps") % (res[v]["e2e"]["h2d_bytes_per_step"] / 1e6),
+                "parallelism": "single GPU"}
+
+    def entry(v):
+        r = res[v]
+        return {"value": r["ms_per_step"], "unit": "ms", "ms_per_step": r["ms_per_step"],
+                "dtype": "bf16" if v == "G" else "f32", "config": config_of(v),
+                "e2e": r["e2e"], "gpu_launches": r["launches"], "step_ms": r["step_ms"],
+                "roofline": r["roofline"], "normalize": r["normalize"], "phases": r["phases"],
+                "muon": r["muon"], "cpu_baseline": r["cpu_baseline"], "clocks": r["clocks"]}
+
+    primary = variants[0]
+    p = entry(primary)
+    line = {"metric": METRIC, "value": p["value"], "unit": "ms", "n_gpus": 1,
+            "steps": args.steps, "warmup": res[primary]["warmup"], "ms_per_step": p["ms_per_step"],
+            "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+            "dtype": p["dtype"], "data": "synthetic", "config": p["config"],
+            "e2e": p["e2e"], "gpu_launches": p["gpu_launches"], "step_ms": p["step_ms"],
+            "roofline": p["roofline"], "normalize": p["normalize"], "phases": p["phases"],
+            "muon": p["muon"], "cpu_baseline": p["cpu_baseline"], "clocks": p["clocks"]}
+    if len(variants) > 1:
+        line["variants"] = {v: entry(v) for v in variants[1:]}
+    print(json.dumps(line), flush=True)
 
 
 def main():
@@ -465,27 +546,31 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(S.CONFIGS))
-    ap.add_argument("--variant", default=None, choices=[None, "G", "L", "L_exact"])
+    ap.add_argument("--variant", default=None, choices=[None, "G", "L", "L_exact"],
+                    help="one variant only (default: every variant the workload names)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-muon", action="store_true", help="skip timing the Muon comparison step")
     args = ap.parse_args()
     cfg = S.CONFIGS[args.config]
-    variant = args.variant or cfg.variants[0]
+    variants = [args.variant] if args.variant else list(cfg.variants)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
-    if world > 1:
-        import torch.distributed as dist
-        if args.impl == "ours":
-            import torch
-            torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
-        dist.init_process_group("nccl" if args.impl == "ours" else "gloo")
     if args.impl == "reference":
-        run_reference(args, cfg, variant, rank, world)
-    else:
-        run_ours(args, cfg, variant, rank, world)
-    if world > 1:
-        import torch.distributed as dist
-        dist.destroy_process_group()
+        # the oracle on the host cores: rank 0 alone works, the other ranks exit
+        if world > 1:
+            import torch.distributed as dist
+            dist.init_process_group("gloo")
+        run_reference(args, cfg, variants[0], rank, world)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+    if args.gpus != 1 or world != 1:
+        sys.stderr.write("bench.py: the NormPre library runs on one GPU only (the per-matrix step has no "
+                         "exchange and the workload fixes a single device); got --gpus %d, WORLD_SIZE %d\n"
+                         % (args.gpus, world))
+        sys.exit(2)
+    run_ours(args, cfg, variants)
 
 
 if __name__ == "__main__":

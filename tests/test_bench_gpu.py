@@ -40,3 +40,27 @@ def test_bench_line_contract(variant):
     st = d["step_ms"]
     assert 0 < st["p10"] <= st["p50"] <= st["p90"] and st["steps"] == 4
     assert "sm_mhz" in d["clocks"] and "reasons" in d["clocks"]
+
+
+def test_bench_line_both_variants():
+    """Without --variant the workload's variants all run: NormPre-G on the
+    line's own keys, NormPre-L under variants.L with its own roofline (the
+    sketch contractions against HBM) and end-to-end number."""
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--steps", "4", "--warmup", "3",
+           "--no-cpu-baseline", "--no-muon", "--config", "single_256x1024"]
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1, r.stdout[-2000:]
+    d = json.loads(lines[0])
+    assert d["config"]["variant"] == "G" and d["roofline"]["bound"] == "tensor"
+    lv = d["variants"]["L"]
+    assert lv["config"]["variant"] == "L" and lv["value"] > 0 and lv["gpu_launches"] > 0
+    assert lv["roofline"]["bound"] == "hbm" and lv["roofline"]["achieved"] > 0
+    assert lv["e2e"]["value"] > 0
+    # the launch counts of the timed region are per step, not doubled by the
+    # untimed passes around it
+    for e in (d, lv):
+        ph = e["phases"]
+        assert ph["normalize"]["launches_per_step"] >= 1
+        assert e["gpu_launches"] == round(sum(v["launches_per_step"] for v in ph.values()) * 4)

@@ -1,31 +1,17 @@
-"""The N > 1 launch path on CPU: world-size-2 gloo process groups.
+"""Launches with more than one rank, on CPU.
 
-NormPre's per-matrix step has no exchange between matrices, so several GPUs
-run replicas (one parameter set each) and the job's time is the slowest
-rank's.  These tests cover that host logic without a GPU: the max-over-ranks
-reduction bench.py uses, and the reference arm launched by
-torch.distributed.run with two ranks (rank 0 alone works and prints one JSON
-line, the other exits 0)."""
+The library runs on one GPU (the per-matrix step has no exchange and the
+workload fixes a single device), so bench.py's own arm refuses any launch of
+more than one GPU or rank.  The reference arm (the fp64 oracle on the host
+cores) may still be started by torch.distributed.run with several ranks:
+rank 0 alone works and prints one JSON line, the other ranks exit 0.  Both
+are checked here with world-size-2 gloo groups and plain subprocesses."""
 import json
 import os
 import subprocess
 import sys
 
-import pytest
-
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-
-
-def _worker(rank, world, port, q):
-    import torch.distributed as dist
-    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
-    sys.path.insert(0, ROOT)
-    import bench
-    dist.init_process_group("gloo", rank=rank, world_size=world)
-    try:
-        q.put((rank, bench.max_over_ranks(1.5 + rank, world, "cpu")))
-    finally:
-        dist.destroy_process_group()
 
 
 def _free_port():
@@ -35,32 +21,11 @@ def _free_port():
         return s.getsockname()[1]
 
 
-def test_max_over_ranks_gloo_world_2():
-    import torch.multiprocessing as mp
-    ctx = mp.get_context("spawn")
-    q = ctx.Queue()
-    port = _free_port()
-    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
-    for p in procs:
-        p.start()
-    for p in procs:
-        p.join(timeout=120)
-        assert p.exitcode == 0
-    got = dict(q.get(timeout=10) for _ in range(2))
-    assert got == {0: 2.5, 1: 2.5}
-
-
-def test_max_over_ranks_single_rank_is_identity():
-    sys.path.insert(0, ROOT)
-    import bench
-    assert bench.max_over_ranks(3.25, 1, "cpu") == 3.25
-
-
 def test_reference_arm_under_torchrun_world_2():
     env = dict(os.environ, PYTHONPATH=ROOT)
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
            "--master-addr", "127.0.0.1", "--master-port", str(_free_port()),
-           os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2", "--steps", "1",
+           os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2", "--steps", "2",
            "--warmup", "0", "--config", "single_256x1024"]
     r = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stderr[-2000:]
@@ -68,4 +33,23 @@ def test_reference_arm_under_torchrun_world_2():
     assert len(lines) == 1, r.stdout[-2000:]
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["unit"] == "ms"
-    assert d["cpu_baseline"]["kind"] == "oracle"
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
+    assert d["config"]["workload"] == "single_256x1024"
+
+
+def test_our_arm_refuses_more_than_one_gpu():
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--gpus", "2", "--steps", "1",
+           "--config", "single_256x1024"]
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 2
+    assert "one GPU only" in r.stderr
+    assert not [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+
+
+def test_our_arm_refuses_a_multi_rank_launch():
+    env = dict(os.environ, WORLD_SIZE="2", RANK="1", LOCAL_RANK="1")
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--steps", "1", "--config", "single_256x1024"]
+    r = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 2
+    assert "WORLD_SIZE 2" in r.stderr
