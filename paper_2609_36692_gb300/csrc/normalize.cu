@@ -19,10 +19,14 @@
 //
 // The tangent step subtracts c_i w_i with c_i = <m_i, w_i> (relaxed, the
 // paper's), <m_i, w_i> / ||w_i||^2 (strict tangent ablation; 0 for a zero
-// weight row) or 0 (no-tangent ablation), Table 5a.  A strict-tangent row
-// below 1e-3 of its momentum row's norm is rounding left by a momentum row
-// parallel to its weight row (or by the cancellation of the column-active
-// closed form), and is taken as zero.
+// weight row) or 0 (no-tangent ablation), Table 5a.  The strict projection
+// of a momentum row parallel to its weight row leaves only rounding, which
+// would normalize to a unit row of noise: with the coefficient from fp32
+// sums that residue is up to ~1e-5 of ||m_i||, so a strict-tangent row
+// whose x_i is at most 1e-3 of ||m_i|| is taken as zero (the kernels'
+// fp32 resolution of the projection).  Column-active strict steps sum
+// ||x_j||^2 from the subtracted values in an extra pass (the closed form
+// ||m||^2 - <m, w>^2 / ||w||^2 cancels for such columns).
 #include <type_traits>
 
 #include "common.cuh"
@@ -253,8 +257,12 @@ __global__ void __launch_bounds__(kColThreads) k_norm_cols_stats(const __grid_co
   }
 }
 
-// column-active fold: per column a_j = <m_j, w_j>, inv_j = 1 / ||x_j||
-__global__ void __launch_bounds__(256) k_norm_cols_final(const __grid_constant__ NormLaunch a, int nrb) {
+// column-active fold: per column a_j = <m_j, w_j>, inv_j = 1 / ||x_j||.
+// stage 0: both from the pass-A sums (relaxed and no-tangent modes).
+// stage 1 (strict): a_j = <m_j, w_j> / ||w_j||^2 only.
+// stage 2 (strict): ||x_j||^2 from the direct sums of k_norm_cols_xsq (slot 1),
+// ||m_j||^2 from pass A (slot 0), a_j kept.
+__global__ void __launch_bounds__(256) k_norm_cols_final(const __grid_constant__ NormLaunch a, int nrb, int stage) {
   __shared__ float red[32];
   const int b = blockIdx.y;
   const int64_t cols = a.cols;
@@ -267,24 +275,93 @@ __global__ void __launch_bounds__(256) k_norm_cols_final(const __grid_constant__
       s0 += p[0]; s1 += p[1]; s2 += p[2];
       p += cols * 3;
     }
-    // relaxed: a = S_mw, ||x||^2 = S_mm - a^2 (2 - S_ww); strict: a = S_mw / S_ww,
-    // ||x||^2 = S_mm - a S_mw; none: a = 0, ||x||^2 = S_mm
-    double aa, d2;
-    if (a.tangent == 0) { aa = s1; d2 = s0 - aa * aa * (2.0 - s2); }
-    else if (a.tangent == 2) {
-      aa = s2 > 0.0 ? s1 / s2 : 0.0;
-      d2 = s0 - aa * s1;
-      if (d2 <= 1e-6 * s0) d2 = 0.0;     // parallel to the weight column: no tangent part
+    float2* out = a.col_coef + static_cast<int64_t>(b) * cols + j;
+    if (stage == 1) {
+      // strict: only the projection coefficient; the norm comes from the direct pass
+      *out = make_float2(s2 > 0.0 ? static_cast<float>(s1 / s2) : 0.f, 0.f);
+    } else {
+      // relaxed: a = S_mw, ||x||^2 = S_mm - a^2 (2 - S_ww); none: a = 0,
+      // ||x||^2 = S_mm; strict (stage 2): S_xx summed directly
+      double aa, d2;
+      if (stage == 2) {
+        aa = out->x;
+        d2 = s1;
+        if (d2 <= 1e-6 * s0) d2 = 0.0;   // parallel to the weight column: no tangent part
+      }
+      else if (a.tangent == 0) { aa = s1; d2 = s0 - aa * aa * (2.0 - s2); }
+      else { aa = 0.0; d2 = s0; }
+      if (!(d2 > 0.0)) d2 = (d2 == d2) ? 0.0 : d2;    // clamp rounding below zero, keep NaN
+      const float inv = d2 > 0.0 ? static_cast<float>(1.0 / sqrt(d2)) : 0.f;
+      *out = make_float2(static_cast<float>(aa), inv);
+      nz = d2 > 0.0 ? 1.f : 0.f;
+      if (!isfinite(d2) || !isfinite(aa)) raise_flag(a.flags, kFlagNonfinite);
     }
-    else { aa = 0.0; d2 = s0; }
-    if (!(d2 > 0.0)) d2 = (d2 == d2) ? 0.0 : d2;    // clamp rounding below zero, keep NaN
-    const float inv = d2 > 0.0 ? static_cast<float>(1.0 / sqrt(d2)) : 0.f;
-    a.col_coef[static_cast<int64_t>(b) * cols + j] = make_float2(static_cast<float>(aa), inv);
-    nz = d2 > 0.0 ? 1.f : 0.f;
-    if (!isfinite(d2) || !isfinite(aa)) raise_flag(a.flags, kFlagNonfinite);
   }
   nz = block_sum(nz, red);
   if (threadIdx.x == 0 && nz > 0.f) atomicAdd(&a.count[a.mat_id[b]], static_cast<int>(nz));
+}
+
+// strict tangent, column-active: ||x_j||^2 of this block's rows summed from
+// x_ij = m_ij - a_j w_ij itself (no cancellation), into slot 1 of the
+// block's partials (the <m, w> sums, already folded into a_j).
+// grid and thread layout as pass A.
+template <typename TW, bool VEC>
+__global__ void __launch_bounds__(kColThreads) k_norm_cols_xsq(const __grid_constant__ NormLaunch a) {
+  __shared__ float part[8][256];
+  const int b = blockIdx.z, rb = blockIdx.y;
+  const int cc = threadIdx.x & 31, rl = threadIdx.x >> 5;
+  const int64_t rows = a.rows, cols = a.cols;
+  const int64_t r0 = static_cast<int64_t>(rb) * kColStatsRB;
+  const int64_t r1 = min(r0 + kColStatsRB, rows);
+  const float* M = a.M[b];
+  const TW* w = static_cast<const TW*>(a.W[b]);
+  const float2* coef = a.col_coef + static_cast<int64_t>(b) * cols;
+  if (VEC) {
+    const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 256 + cc * 8;
+    float sx[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) sx[e] = 0.f;
+    if (j0 < cols) {
+      float ca[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) ca[e] = coef[j0 + e].x;
+      for (int64_t r = r0 + rl; r < r1; r += 8) {
+        float mv[8], wv[8];
+        load8(M + r * cols + j0, mv);
+        load8(w + r * cols + j0, wv);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float x = fmaf(-ca[e], wv[e], mv[e]);
+          sx[e] = fmaf(x, x, sx[e]);
+        }
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) part[rl][cc * 8 + e] = sx[e];
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int64_t j = static_cast<int64_t>(blockIdx.x) * 256 + cc + 32 * e;
+      float sx = 0.f;
+      if (j < cols) {
+        const float cj = coef[j].x;
+        for (int64_t r = r0 + rl; r < r1; r += 8) {
+          const float x = fmaf(-cj, to_f32(w[r * cols + j]), M[r * cols + j]);
+          sx = fmaf(x, x, sx);
+        }
+      }
+      part[rl][cc + 32 * e] = sx;
+    }
+  }
+  __syncthreads();
+  const int col = threadIdx.x;
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * 256 + col;
+  if (j < cols) {
+    double s = 0;
+#pragma unroll
+    for (int l = 0; l < 8; ++l) s += part[l][col];
+    a.col_part[((static_cast<int64_t>(b) * gridDim.y + rb) * cols + j) * 3 + 1] = s;
+  }
 }
 
 // column-active pass B: Psi_ij = (m_ij - a_j w_ij) * inv_j
@@ -439,7 +516,17 @@ cudaError_t launch_normalize_cols(const NormLaunch& a, cudaStream_t s) {
     else k_norm_cols_stats<TG, TW, false><<<grid, kColThreads, 0, s>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_norm_cols_final<<<dim3(grid.x, a.n), 256, 0, s>>>(a, nrb);
+    if (a.tangent == 2) {
+      // strict: the coefficient first, then ||x_j||^2 summed from x itself
+      k_norm_cols_final<<<dim3(grid.x, a.n), 256, 0, s>>>(a, nrb, 1);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      if (vec) k_norm_cols_xsq<TW, true><<<grid, kColThreads, 0, s>>>(a);
+      else k_norm_cols_xsq<TW, false><<<grid, kColThreads, 0, s>>>(a);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      k_norm_cols_final<<<dim3(grid.x, a.n), 256, 0, s>>>(a, nrb, 2);
+    } else {
+      k_norm_cols_final<<<dim3(grid.x, a.n), 256, 0, s>>>(a, nrb, 0);
+    }
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (vec) k_norm_cols_apply<TW, TP, true><<<grid_b, kColThreads, 0, s>>>(a);
