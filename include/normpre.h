@@ -113,13 +113,19 @@ typedef struct normpre_config {
   int diagnostics;        /* 1: every step also accumulates, per matrix, <G, T>, ||G||^2 and
                              ||T||^2 of the raw gradient G and the preconditioned update T (one
                              more read of G and T), for the descent alignment of NORMPRE_BUF_DIAG */
+  int jacobi_max_sweeps;  /* NormPre-L: cap on the Jacobi sweeps of the l x l Ritz problem
+                             (Alg. 2, eig of Gamma_Q); 0 = default 30, else in [1, 1000].  A step
+                             that reaches the cap before converging reports NORMPRE_ERR_NUMERIC */
 } normpre_config;
 
 /* Fills `cfg` with the paper's defaults (NormPre-G, bf16 Newton-Schulz). */
 void normpre_default_config(normpre_config* cfg);
 
 /*
- * Creates a handle for a fixed list of matrices.
+ * Creates a handle for a fixed list of matrices: the weight matrices W in
+ * R^{m x n} that Algorithm 1 updates one by one, with the optimizer's
+ * hyperparameters (Table 4, App. A).  The handle holds no optimizer state of
+ * the paper's (the momentum M is the caller's), only plans and workspaces.
  *   cfg       hyperparameters (copied).
  *   n_mats    number of matrices (>= 1).
  *   rows/cols host arrays[n_mats] of stored shapes (each >= 1, <= 65536).
@@ -208,7 +214,11 @@ int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* row
 /*
  * Synchronizes the device and copies buffer `what` of matrix `mat` into the
  * host array `dst` (row-major, `capacity_bytes` long).  Intended for tests and
- * diagnostics.  Errors: ARG (too small / absent), CUDA.
+ * diagnostics: the intermediates of the last step as the paper defines them,
+ * Psi of Eq. 3, T of Sec. 3.2 (Newton-Schulz), Omega, Q, the Ritz pairs and
+ * the selection of Algorithm 2, the eigenvalues of Gamma of the exact
+ * extraction (Sec. 3.2), the energies and alignment of App. E.
+ * Errors: ARG (too small / absent), CUDA.
  */
 int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capacity_bytes);
 
@@ -225,6 +235,28 @@ int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capaci
  */
 int normpre_newton_schulz(const normpre_config* cfg, int batch, int64_t rows, int64_t cols,
                           const void* X, void* T, void* stream);
+
+/*
+ * The Gaussian sketch matrix of one matrix and step (Algorithm 2, "sample
+ * Omega"), computed by the kernel the NormPre-L step uses, with the random
+ * stream it draws from written out for checking:
+ *   Omega (n_a x l, row-major, fp32, device): element e = i l + j takes word
+ *     e mod 4 of the Philox4x32-10 block (Salmon et al., SC'11) with counter
+ *     (e / 4, matrix_id, t lo 32 bits, t hi 32 bits) and key (seed lo, seed
+ *     hi); each word x gives the uniform u = ((x >> 9) + 0.5) 2^-23 (exact in
+ *     fp32), and the word pairs (0, 1), (2, 3) of a block give two normals by
+ *     Box-Muller (sqrt(-2 ln u_a) cos(2 pi u_b), ... sin ...).
+ *   words    (optional, NULL to skip; device uint32, n_a x l) the word x of
+ *            each element.
+ *   uniforms (optional, NULL to skip; device fp32, n_a x l) its uniform u.
+ * matrix_id is the matrix's index in the list given to normpre_init (the
+ * step's Omega of matrix i at step t equals this call's with matrix_id = i,
+ * the same t and the config's seed).  Outputs 4-byte aligned; n_a * l <= 2^32.
+ * Asynchronous on `stream`; allocates nothing.
+ * Errors (message from normpre_last_error(NULL)): ARG, SHAPE, ALIGN, CUDA.
+ */
+int normpre_sketch_omega(uint64_t seed, int matrix_id, int64_t t, int64_t n_a, int l, float* omega,
+                         uint32_t* words, float* uniforms, void* stream);
 
 /*
  * Per-phase timing of this library's kernels (tests and benchmarks).
@@ -283,7 +315,10 @@ int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* 
  * several host threads on one device) race and give wrong results: order
  * them on one stream.  The first call on each device looks up the array's
  * device address (cudaGetSymbolAddress) with that device current; make that
- * first call before any stream capture.  Asynchronous on `stream`; device-side
+ * first call before any stream capture.  The address is kept for the life of
+ * the process: after cudaDeviceReset (or any other teardown of the device's
+ * primary context) it no longer points at the array, so do not call this
+ * entry point again in a process that has reset the device.  Asynchronous on `stream`; device-side
  * conditions (non-finite input) are not reported by this entry point.
  * Errors (message from normpre_last_error(NULL)): ARG, SHAPE (including sizes
  * beyond the scratch array), DTYPE, ALIGN, CUDA.
@@ -291,7 +326,9 @@ int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* 
 int normpre_normalize_cols_noalloc(int64_t rows, int64_t cols, float mu, const void* G, int g_dtype,
                                    float* M, const void* W, int w_dtype, float* Psi, void* stream);
 
-/* Releases the handle and every device buffer it owns.  NULL is ignored. */
+/* Releases the handle made by normpre_init and every device buffer it owns
+ * (the caller's W, G and M, which carry the optimizer's state across the steps
+ * of Algorithm 1, are untouched).  NULL is ignored. */
 void normpre_free(normpre_handle* h);
 
 /* Message of the last failure of `h` (or of the calling thread when h is NULL). */

@@ -134,6 +134,9 @@ int check_config(const normpre_config* c, std::string* msg) {
       *msg = "need rank >= 1, oversample >= 0 and rank + oversample <= 72"; return NORMPRE_ERR_ARG;
     }
     if (c->power_iters < 0 || c->power_iters > 8) { *msg = "power_iters must be in [0, 8]"; return NORMPRE_ERR_ARG; }
+    if (c->jacobi_max_sweeps < 0 || c->jacobi_max_sweeps > 1000) {
+      *msg = "jacobi_max_sweeps must be 0 (default) or in [1, 1000]"; return NORMPRE_ERR_ARG;
+    }
   }
   return NORMPRE_OK;
 }
@@ -510,6 +513,7 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
     SketchParams p;
     p.rank = c.rank; p.oversample = c.oversample; p.power_iters = c.power_iters;
     p.seed = c.seed; p.t = t; p.k = k;
+    p.max_sweeps = c.jacobi_max_sweeps > 0 ? c.jacobi_max_sweeps : 30;
     p.lr = lr; p.wd = c.weight_decay; p.target = c.target_rms;
     for (int ui = 0; ui < nu; ++ui) {
       if ((rc = normalize(ui))) return rc;

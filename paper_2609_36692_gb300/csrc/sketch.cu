@@ -31,6 +31,7 @@
 #include <string>
 #include <type_traits>
 
+#include "../../include/normpre.h"
 #include "common.cuh"
 #include "internal.h"
 #include "tc.cuh"
@@ -77,15 +78,27 @@ struct OmegaArgs {
   int64_t n_a;
   int l;
   uint32_t key0, key1, t_lo, t_hi;
-  const int* mat_id;     // [batch]
+  const int* mat_id;     // [batch]; null: every matrix is mat_id0
+  int mat_id0 = 0;
+  uint32_t* words = nullptr;   // optional [batch][n_a][l]: the Philox word of each element
+  float* uniforms = nullptr;   // optional [batch][n_a][l]: its uniform in (0, 1)
 };
 __global__ void k_omega(const __grid_constant__ OmegaArgs a) {
   const int b = blockIdx.y;
   const int64_t n = a.n_a * a.l;
   const int64_t blk = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (blk * 4 >= n) return;
-  uint32_t c[4] = {static_cast<uint32_t>(blk), static_cast<uint32_t>(a.mat_id[b]), a.t_lo, a.t_hi};
+  const int mid = a.mat_id ? a.mat_id[b] : a.mat_id0;
+  uint32_t c[4] = {static_cast<uint32_t>(blk), static_cast<uint32_t>(mid), a.t_lo, a.t_hi};
   philox4x32_10(c, a.key0, a.key1);
+  if (a.words != nullptr || a.uniforms != nullptr) {
+#pragma unroll
+    for (int w = 0; w < 4; ++w)
+      if (blk * 4 + w < n) {
+        if (a.words) a.words[b * a.bstride + blk * 4 + w] = c[w];
+        if (a.uniforms) a.uniforms[b * a.bstride + blk * 4 + w] = philox_unit(c[w]);
+      }
+  }
   float z[4];
 #pragma unroll
   for (int p = 0; p < 2; ++p) {
@@ -1533,7 +1546,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       ea.count = count; ea.mat_id = mat_ids;
       ea.l = l; ea.rank = p.rank; ea.k_orient = p.k;
       ea.m_a = m_a; ea.n_a = n_a;
-      ea.max_sweeps = 30;
+      ea.max_sweeps = p.max_sweeps;
       ea.flags = flags;
       const int jthreads = static_cast<int>(jacobi_threads(l));
       const int nj = (l + 1) & ~1;
@@ -1594,3 +1607,37 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
 }
 
 }  // namespace normpre
+
+// ---------------------------------------------------------------------------
+// Stand-alone sketch matrix (normpre_sketch_omega): the kernel the step uses,
+// for one matrix, with its Philox words and uniforms written out as well.
+// ---------------------------------------------------------------------------
+extern "C" int normpre_sketch_omega(uint64_t seed, int matrix_id, int64_t t, int64_t n_a, int l, float* omega,
+                                    uint32_t* words, float* uniforms, void* stream) {
+  using namespace normpre;
+  if (!omega) { set_thread_error("null omega pointer"); return NORMPRE_ERR_ARG; }
+  if (matrix_id < 0) { set_thread_error("matrix_id must be >= 0"); return NORMPRE_ERR_ARG; }
+  if (n_a < 1 || l < 1 || n_a > (int64_t(1) << 24) || l > 4096 || n_a * l > (int64_t(1) << 32)) {
+    set_thread_error("n_a and l must be >= 1 with n_a * l <= 2^32 (the 32-bit block counter)");
+    return NORMPRE_ERR_SHAPE;
+  }
+  auto al4 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 3u) == 0; };
+  if (!al4(omega) || (words && !al4(words)) || (uniforms && !al4(uniforms))) {
+    set_thread_error("outputs must be 4-byte aligned");
+    return NORMPRE_ERR_ALIGN;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  OmegaArgs o;
+  o.omega = omega; o.bstride = n_a * l; o.n_a = n_a; o.l = l;
+  o.key0 = static_cast<uint32_t>(seed); o.key1 = static_cast<uint32_t>(seed >> 32);
+  o.t_lo = static_cast<uint32_t>(static_cast<uint64_t>(t)); o.t_hi = static_cast<uint32_t>(static_cast<uint64_t>(t) >> 32);
+  o.mat_id = nullptr;
+  o.mat_id0 = matrix_id;
+  o.words = words;
+  o.uniforms = uniforms;
+  const int64_t blocks = cdiv(n_a * l, 4);
+  k_omega<<<dim3(static_cast<unsigned>(cdiv(blocks, 256)), 1), 256, 0, s>>>(o);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) { set_thread_error(std::string("launch: ") + cudaGetErrorString(e)); return NORMPRE_ERR_CUDA; }
+  return NORMPRE_OK;
+}

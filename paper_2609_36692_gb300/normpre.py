@@ -46,6 +46,7 @@ class normpre_config(ctypes.Structure):
         ("orientation", ctypes.c_int),
         ("tangent", ctypes.c_int),
         ("diagnostics", ctypes.c_int),
+        ("jacobi_max_sweeps", ctypes.c_int),
     ]
 
 
@@ -96,6 +97,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.normpre_normalize_cols_noalloc.argtypes = [i64, i64, ctypes.c_float, P, ctypes.c_int, P, P,
                                                    ctypes.c_int, P, P]
     lib.normpre_normalize_cols_noalloc.restype = ctypes.c_int
+    lib.normpre_sketch_omega.argtypes = [ctypes.c_uint64, ctypes.c_int, i64, i64, ctypes.c_int, P, P, P, P]
+    lib.normpre_sketch_omega.restype = ctypes.c_int
     lib.normpre_free.argtypes = [P]
     lib.normpre_free.restype = None
     lib.normpre_last_error.argtypes = [P]
@@ -201,6 +204,13 @@ def normpre_normalize_cols_noalloc(rows: int, cols: int, mu: float, G_ptr: int, 
     return _check(load_library().normpre_normalize_cols_noalloc(
         int(rows), int(cols), float(mu), G_ptr, int(g_dtype), M_ptr, W_ptr, int(w_dtype), Psi_ptr,
         stream))
+
+
+def normpre_sketch_omega(seed: int, matrix_id: int, t: int, n_a: int, l: int, omega_ptr: int,
+                         words_ptr: int = 0, uniforms_ptr: int = 0, stream: int = 0) -> int:
+    return _check(load_library().normpre_sketch_omega(int(seed), int(matrix_id), int(t), int(n_a), int(l),
+                                                      omega_ptr, words_ptr or None, uniforms_ptr or None,
+                                                      stream))
 
 
 def normpre_free(handle: int) -> None:

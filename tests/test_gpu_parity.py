@@ -9,8 +9,11 @@ Tolerances (stated by the workload and derived where it is silent):
     subspaces <= 1e-3 (fp32), equal |C| whenever the Ritz values are >= 1e-3
     away from 1 and from the r-th/(r+1)-th cut.
   * weight update: the change W_{t+1} - W_t has relative Frobenius error within
-    the tolerance of T (fp32 weights); bf16 weights are compared elementwise to
-    the oracle's result within 1 bf16 ulp plus the T tolerance share.
+    the tolerance of T (fp32 weights); bf16 weights are compared element by
+    element with the oracle's W_{t+1}: within one bf16 ulp plus the update
+    tolerance times (the element's own update + six times the update's
+    root-mean-square); in aggregate, within the update tolerance plus half an
+    ulp per element.
 """
 import os
 
@@ -117,6 +120,25 @@ def test_normalize_and_momentum(cfgset, t, w_dtype):
         assert int(st[0]) == k and int(st[1]) == int((ref["d"] > 0).sum())
 
 
+def _check_bf16_w(w_gpu, w_ref, dw_ref, tol, where):
+    """bf16 weights: the device stores the bf16 rounding (RNE) of its fp32
+    update.  Element by element, the stored value is within one bf16 ulp of the
+    oracle's exact W_{t+1} plus that element's share of the update tolerance:
+    the tolerance relative to the element's own update (the operand and output
+    roundings of a bf16 product scale with the entry) plus 6 times the
+    root-mean-square share (the error spread over the matrix).  In aggregate,
+    the Frobenius error is within the update tolerance plus the half-ulp
+    rounding of every element."""
+    w_gpu = np.asarray(w_gpu, np.float64)
+    err = np.abs(w_gpu - w_ref)
+    share = tol * (np.abs(dw_ref) + 6.0 * np.sqrt(np.mean(dw_ref ** 2)))
+    bound = bf16_ulp(w_ref) + share
+    worst = int(np.argmax(err - bound))
+    assert np.all(err <= bound), (where, worst, float(err.flat[worst]), float(bound.flat[worst]))
+    assert np.linalg.norm(w_gpu - w_ref) <= tol * np.linalg.norm(dw_ref) + \
+        np.linalg.norm(0.5 * bf16_ulp(w_ref)), where
+
+
 # ---------------------------------------------------------------------------
 # NormPre-G
 # ---------------------------------------------------------------------------
@@ -134,11 +156,7 @@ def _check_g(cs, t, precision, tol_t, indices=None):
         if cs.w_dtype == "f32":
             assert rel_fro(dW, dW_ref) <= tol_t, (cs.name, i)
         else:
-            # bf16 weights: the device result is the bf16 rounding (<= half an ulp
-            # per element) of an update within the T tolerance
-            half_ulp = 0.5 * bf16_ulp(ref["W"])
-            err = np.linalg.norm(W1[i].astype(np.float64) - ref["W"])
-            assert err <= tol_t * np.linalg.norm(dW_ref) + np.linalg.norm(half_ulp), (cs.name, i)
+            _check_bf16_w(W1[i], ref["W"], dW_ref, tol_t, (cs.name, i))
         st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
         assert abs(st[2] - (ref["T"] ** 2).sum()) <= 4 * tol_t * (ref["T"] ** 2).sum()
 
@@ -164,11 +182,13 @@ def test_g_bf16_gpt2_full_size_sampled(t):
 
 
 @pytest.mark.slow
+@pytest.mark.parametrize("t", [0, 1])
 @pytest.mark.parametrize("name,indices", [("llama_1b", [0, 4, 6, 111]), ("qwen3_1p7b", [0, 1, 4, 6, 195])])
-def test_g_bf16_large_sets_sampled(name, indices):
+def test_g_bf16_large_sets_sampled(name, indices, t):
     """LLaMA ~1B (112 matrices) and Qwen3 ~1.7B (196 matrices, bf16 weights),
-    full set on the GPU, one matrix of each shape against the oracle."""
-    _check_g(S.CONFIGS[name], 1, precision=0, tol_t=2e-2, indices=indices)
+    full set on the GPU in the launch configuration the bench times, one matrix
+    of each shape against the oracle, at both orientations."""
+    _check_g(S.CONFIGS[name], t, precision=0, tol_t=2e-2, indices=indices)
 
 
 # ---------------------------------------------------------------------------
@@ -224,7 +244,59 @@ def _check_l(cs, t, indices=None, w_tol=2e-3):
         dW_ref = ref["W"] - mats[i]["W"]
         if cs.w_dtype == "f32":
             assert rel_fro(dW, dW_ref) <= w_tol, (cs.name, i, rel_fro(dW, dW_ref))
+        else:
+            _check_bf16_w(W1[i], ref["W"], dW_ref, w_tol, (cs.name, i))
     return n_checked
+
+
+def _oracle_words(seed, mid, t, n):
+    """The oracle's Philox words of elements 0..n-1 in the counter layout of the
+    sketch (Alg. 2 "sample Omega"): element e takes word e mod 4 of block e / 4."""
+    nblk = (n + 3) // 4
+    blk = np.arange(nblk, dtype=np.uint64)
+    full = lambda v: np.full(nblk, v & 0xFFFFFFFF, dtype=np.uint64)  # noqa: E731
+    x = O.philox4x32_10((blk, full(mid), full(t), full(t >> 32)), (seed & 0xFFFFFFFF, seed >> 32))
+    return np.stack(x, axis=1).reshape(-1)[:n]
+
+
+@pytest.mark.parametrize("seed,mid,t,n_a,l", [(1234, 0, 0, 1024, 24), (0xDEADBEEFCAFE, 7, (1 << 33) + 5, 777, 40),
+                                              (1, 195, 1, 6144, 40), (2 ** 64 - 1, 3, 12, 5, 3)])
+def test_philox_stream_bit_exact(seed, mid, t, n_a, l):
+    """The sketch's random stream on the GPU is the oracle's, bit for bit: the
+    Philox4x32-10 words and their uniforms are compared exactly, the Box-Muller
+    normals within libm rounding."""
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    om = torch.empty((n_a, l), dtype=torch.float32, device="cuda")
+    words = torch.empty((n_a, l), dtype=torch.int32, device="cuda")
+    uni = torch.empty((n_a, l), dtype=torch.float32, device="cuda")
+    C.normpre_sketch_omega(seed, mid, t, n_a, l, om.data_ptr(), words.data_ptr(), uni.data_ptr(),
+                           torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    w_gpu = words.cpu().numpy().view(np.uint32).reshape(-1)
+    w_ref = _oracle_words(seed, mid, t, n_a * l)
+    assert np.array_equal(w_gpu, w_ref)
+    u_ref = O.philox_uniform(w_ref).astype(np.float32)
+    assert np.array_equal(uni.cpu().numpy().reshape(-1).view(np.uint32), u_ref.view(np.uint32))
+    ref = O.sketch_omega(seed, mid, t, n_a, l)
+    assert np.max(np.abs(om.cpu().numpy() - ref)) <= 1e-5 * (1 + np.abs(ref).max())
+
+
+@pytest.mark.parametrize("t", [0, 1])
+def test_step_omega_is_the_stand_alone_stream(t):
+    """The Omega a NormPre-L step draws for matrix i is, bit for bit, the
+    stand-alone sketch matrix for (seed, i, t)."""
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    opt, mats, _, _ = _run(SMALL, t, "L", precision=1)
+    for i in range(SMALL.n_mats):
+        got = opt.read(i, C.NORMPRE_BUF_OMEGA)
+        n_a, l = got.shape
+        om = torch.empty((n_a, l), dtype=torch.float32, device="cuda")
+        C.normpre_sketch_omega(1234, i, t, n_a, l, om.data_ptr(), 0, 0, torch.cuda.current_stream().cuda_stream)
+        torch.cuda.synchronize()
+        assert np.array_equal(got.view(np.uint32), om.cpu().numpy().view(np.uint32)), i
+    opt.close()
 
 
 @pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED, ODD], ids=lambda c: c.name)
@@ -288,11 +360,15 @@ def test_l_gpt2_full_size_sampled(t):
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name,indices", [("llama_1b", [0, 4, 6]), ("qwen3_1p7b", [1, 4, 6])])
-def test_l_large_sets_sampled(name, indices):
+@pytest.mark.parametrize("t", [0, 1])
+@pytest.mark.parametrize("name,indices", [("llama_1b", [0, 4, 6]), ("qwen3_1p7b", [0, 1, 4, 6])])
+def test_l_large_sets_sampled(name, indices, t):
+    """The full LLaMA ~1B and Qwen3 ~1.7B sets under NormPre-L (r = 32, o = 8,
+    p = 1), one matrix of each shape against the oracle at both orientations;
+    Qwen3's bf16 weights are compared element by element."""
     import dataclasses
     cs = dataclasses.replace(S.CONFIGS[name], rank=32, oversample=8)
-    _check_l(cs, 0, indices=indices)
+    _check_l(cs, t, indices=indices)
 
 
 # ---------------------------------------------------------------------------
@@ -309,10 +385,56 @@ def test_tangent_ablation_normalization(cfgset, t, mode):
     for i in range(cfgset.n_mats):
         ref = _oracle(mats, i, t, "L", cfgset, tangent=mode)
         psi = opt.read(i, 0)   # NORMPRE_BUF_PSI, stored layout
-        # per normalized active row psi_i (Eq. 3): the strict projection cancels
-        # most of m, so single small entries carry ~u ||m|| absolute error
         active = psi if ref["k"] == 0 else psi.T
+        if mode == "strict":
+            # every active row is either exactly parallel to its weight row (the
+            # oracle's x_i vanishes to fp64 rounding; the kernels zero it at
+            # their fp32 resolution, 1e-3 of ||m_i||) or keeps a tangent part
+            # far above that resolution, so the comparison is well posed
+            ratio = np.linalg.norm(ref["X"], axis=1) / np.maximum(
+                np.linalg.norm(O.orient(ref["M"], ref["k"]), axis=1), 1e-300)
+            assert np.all((ratio == 0.0) | (ratio > 1e-2)), (cfgset.name, i)
+        # per normalized active row psi_i (Eq. 3): the strict projection cancels
+        # part of m, so single small entries carry ~u ||m|| absolute error
         assert max_row_rel(active, ref["Psi"]) <= 1e-5, (cfgset.name, i, mode)
+
+
+@pytest.mark.parametrize("t", [0, 1])
+def test_strict_tangent_planted_parallel_rows(t):
+    """Momentum rows (t = 0) or columns (t = 1) exactly parallel to their weight
+    rows, over 384 / 1536 entries: the strict projection leaves no tangent part
+    (Sec. 3.1, Table 5a), so those rows of Psi are zero and m' drops by their
+    number; the other rows match the oracle per normalized row."""
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    rows, cols = 1536, 384
+    cs = S.custom_config("planted_parallel", [(rows, cols)], g_dtype="f32", w_dtype="f32",
+                         row_sigma=1.0, col_sigma=1.0, prior_momentum=False, rank=4, oversample=4)
+    m = S.make_matrix(cs, 0)
+    G, W = m["G"].copy(), m["W"].copy()
+    picks = [3, 77, 200] if t == 0 else [5, 131, 383]
+    for p in picks:
+        # w = 2^-6 g (exact in fp32), and M_{t-1} = 0 there: m = g is exactly parallel to w
+        if t == 0:
+            W[p, :] = G[p, :] * np.float32(2.0 ** -6)
+        else:
+            W[:, p] = G[:, p] * np.float32(2.0 ** -6)
+    mats = [{"G": G, "W": W, "M": m["M"]}]
+    Wd, Gd, Md = to_device(mats, "f32", "f32")
+    opt = _normpre([(rows, cols)], ["f32"], ["f32"], variant=C.NORMPRE_L, precision=1, rank=4,
+                   oversample=4, seed=1234, tangent=_TANGENT["strict"])
+    opt.step(t, LR, Wd, Gd, Md)
+    torch.cuda.synchronize()
+    opt.status()
+    ref = _oracle(mats, 0, t, "L", cs, tangent="strict")
+    assert np.all(ref["d"][picks] == 0.0)
+    psi = opt.read(0, C.NORMPRE_BUF_PSI)
+    active = psi if t == 0 else psi.T
+    assert np.all(active[picks] == 0.0)
+    assert max_row_rel(active, ref["Psi"]) <= 1e-5
+    st = opt.read(0, C.NORMPRE_BUF_STATS)[0]
+    assert int(st[1]) == int((ref["d"] > 0).sum()) == active.shape[0] - len(picks)
+    opt.close()
 
 
 @pytest.mark.parametrize("mode", ["none", "strict"])
@@ -537,7 +659,46 @@ def test_host_entry_point_in_units(variant):
 # --------------------------------------------------------------------------
 # NormPre-L with exact eigenspace extraction (Sec. 3.2, App. B)
 # --------------------------------------------------------------------------
-@pytest.mark.parametrize("cfgset", [SMALL, RAGGED], ids=lambda c: c.name)
+# --------------------------------------------------------------------------
+# device-detected conditions reported through the status word
+# --------------------------------------------------------------------------
+def test_jacobi_sweep_cap_reports_numeric():
+    """With a cap of one Jacobi sweep, the 16 x 16 Ritz problems stop before
+    their off-diagonal mass reaches the fp32 floor: the kernel records one
+    sweep, raises the NUMERIC flag and returns (no trap, no hang), and
+    normpre_sync_status reports NORMPRE_ERR_NUMERIC.  The status word is
+    cleared by that read, so a following step with the default cap is clean."""
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    cs = SMALL
+    mats = S.make_param_set(cs)
+    W, G, M = to_device(mats, cs.g_dtype, cs.w_dtype)
+    shapes = [(m.rows, m.cols) for m in cs.matrices]
+    opt = _normpre(shapes, [cs.w_dtype] * cs.n_mats, [cs.g_dtype] * cs.n_mats, variant=C.NORMPRE_L,
+                   precision=1, rank=cs.rank, oversample=cs.oversample, seed=1234, jacobi_max_sweeps=1)
+    opt.step(0, LR, W, G, M)
+    torch.cuda.synchronize()
+    assert opt.status(raise_on_error=False) == C.NORMPRE_ERR_NUMERIC
+    assert "Jacobi" in C.normpre_last_error(opt.handle)
+    for i in range(cs.n_mats):
+        assert int(opt.read(i, C.NORMPRE_BUF_STATS)[0][7]) == 1
+    opt.close()
+    opt = _normpre(shapes, [cs.w_dtype] * cs.n_mats, [cs.g_dtype] * cs.n_mats, variant=C.NORMPRE_L,
+                   precision=1, rank=cs.rank, oversample=cs.oversample, seed=1234)
+    opt.step(1, LR, W, G, M)
+    torch.cuda.synchronize()
+    assert opt.status(raise_on_error=False) == C.NORMPRE_OK
+    assert all(int(opt.read(i, C.NORMPRE_BUF_STATS)[0][7]) > 1 for i in range(cs.n_mats))
+    opt.close()
+
+
+# one GPT-2 Small attention qkv matrix (768 x 2304): Gamma is 768 x 768 at
+# t = 0 and 2304 x 2304 at t = 1
+GPT2_QKV = S.custom_config("gpt2_qkv", [(768, 2304)], g_dtype="bf16", w_dtype="f32",
+                           row_sigma=1.0, col_sigma=1.0, rank=32, oversample=8)
+
+
+@pytest.mark.parametrize("cfgset", [SMALL, RAGGED, GPT2_QKV], ids=lambda c: c.name)
 @pytest.mark.parametrize("t", [0, 1])
 def test_l_exact(cfgset, t):
     """Gamma = Psi_a Psi_a^T, all its eigenvalues, the selected eigenvectors,
@@ -551,8 +712,10 @@ def test_l_exact(cfgset, t):
         lam = ex["lam"]
         eig = opt.read(i, C.NORMPRE_BUF_EIGS)[0].astype(np.float64)
         assert eig.shape == lam.shape, (cfgset.name, i)
-        # fp32 Gamma and eigensolver: errors of a few ulp of lambda_max
-        assert np.max(np.abs(eig - lam)) <= 2e-5 * max(1.0, lam[0]), (cfgset.name, i)
+        # fp32 Gamma and a backward-stable fp32 eigensolver: errors of order
+        # m_a u ||Gamma||_2 (u = 2^-24), a few ulp of lambda_max for small m_a
+        tol = max(2e-5, lam.size * 2.0 ** -24)
+        assert np.max(np.abs(eig - lam)) <= tol * max(1.0, lam[0]), (cfgset.name, i)
         st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
         if ritz_gaps_ok(lam, cfgset.rank):
             nc = int(st[3])

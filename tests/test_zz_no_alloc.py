@@ -4,7 +4,8 @@ allocator or memory-pool callback, frameworks whose allocator must not be
 re-entered, processes whose device memory is reserved in advance).  Its
 scratch is a fixed array inside the library, so these tests check that it
 gives what the handle-based step gives, call after call, and that it refuses
-shapes whose scratch would not fit.
+shapes whose scratch would not fit.  Each call is also checked against the
+fp64 oracle's column-active step (k = 1) on the same inputs.
 
 This file is named to be collected last: a failure here leaves every other
 test already run.
@@ -12,9 +13,10 @@ test already run.
 import numpy as np
 import pytest
 
+import oracle as O
 from synth import inputs as S
 
-from helpers import max_row_rel, to_device, to_host
+from helpers import max_row_rel, oracle_config, to_device, to_host
 
 
 def _lib():
@@ -77,3 +79,10 @@ def test_noalloc_matches_handle_step_on_two_calls_in_a_row():
         assert max_row_rel(out.T, psi_ref.T.astype(np.float64)) <= 1e-5, (rows, cols)
         m = to_host(M[0])
         assert np.all(np.abs(m.astype(np.float64) - m_ref) <= 2.5e-7 * np.abs(m_ref) + 1e-30), (rows, cols)
+        # the oracle's column-active step (t = 1): momentum, relaxed tangent and
+        # normalization of every column (Alg. 1, Eq. 3)
+        ref = O.normpre_step(mats[0]["W"], mats[0]["G"], mats[0]["M"], 1, 0.02,
+                             oracle_config("L", rank=4, oversample=4), matrix_id=0)
+        assert ref["k"] == 1
+        assert max_row_rel(out.T, ref["Psi"]) <= 1e-5, (rows, cols)
+        assert np.all(np.abs(m.astype(np.float64) - ref["M"]) <= 2.5e-7 * np.abs(ref["M"]) + 1e-30), (rows, cols)
