@@ -353,18 +353,18 @@ constexpr uint32_t kCtcTmemA = 256;
 constexpr uint32_t kCtcTmemCols = 512;
 static_assert(kCtcTmemA + 64 * kCtcStages <= kCtcTmemCols, "TMEM budget");
 
-// x rounded to the nearest TF32 value (ties away from zero), as an fp32 bit
-// pattern with the low 13 mantissa bits clear: adding half of the dropped
-// range to the magnitude bits carries into the kept ones exactly when the
-// dropped part is at least half an ulp of TF32.
-__device__ __forceinline__ float tf32_rna(float x) {
-  return __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
-}
+// The three-product split of an fp32 operand: hi = x with the low 13
+// mantissa bits cleared (a TF32 value, so the MMA reads it exactly), lo =
+// x - hi (exact in fp32, |lo| < 2^-10 |x|).  The MMA reads lo at TF32
+// precision, whatever rounding it applies to the dropped bits, which costs at
+// most 2^-10 |lo| < 2^-20 |x|; the dropped lo * lo term is below 2^-20 of the
+// product as well.
+__device__ __forceinline__ float tf32_hi(float x) { return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u); }
 __device__ __forceinline__ void split4(const float4 x, float4& h, float4& l) {
-  h.x = tf32_rna(x.x); l.x = tf32_rna(x.x - h.x);
-  h.y = tf32_rna(x.y); l.y = tf32_rna(x.y - h.y);
-  h.z = tf32_rna(x.z); l.z = tf32_rna(x.z - h.z);
-  h.w = tf32_rna(x.w); l.w = tf32_rna(x.w - h.w);
+  h.x = tf32_hi(x.x); l.x = x.x - h.x;
+  h.y = tf32_hi(x.y); l.y = x.y - h.y;
+  h.z = tf32_hi(x.z); l.z = x.z - h.z;
+  h.w = tf32_hi(x.w); l.w = x.w - h.w;
 }
 // byte offset of 16-byte chunk j of row r in a 128-byte-swizzled tile
 __device__ __forceinline__ uint32_t sw128(int r, int j) { return static_cast<uint32_t>(r * 128 + ((j ^ (r & 7)) << 4)); }
@@ -612,8 +612,8 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
           }
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
-            hi[e] = tf32_rna(x[e]);
-            lo[e] = tf32_rna(x[e] - hi[e]);
+            hi[e] = tf32_hi(x[e]);
+            lo[e] = x[e] - hi[e];
           }
           const uint32_t ta = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + kCtcTmemA + 64u * st + 16u * kh;
           tmem_st16(ta, hi);
@@ -1256,6 +1256,239 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
 }
 
 // ---------------------------------------------------------------------------
+// Fused apply on the tensor cores (l % 4 == 0, l <= 64, no diagnostics).
+// The rank-l product of T = Psi + Lm Rm^T runs as D = Rm_tile Lm_tile^T on
+// tcgen05 kind::tf32 with the three-product split (hi hi + hi lo + lo hi, as
+// the sketch contractions), M = 128 W columns and N = 256 W rows, so that the
+// TMEM lane is the W column and the TMEM column the W row: an epilogue warp
+// reading one TMEM column block then touches Psi and W in 128-byte rows
+// across its 32 lanes, and the kernel is left with the compulsory HBM stream
+// (Psi read, W read and write) instead of l fp32 FMAs per element.
+//
+// Persistent: CTA c takes a contiguous range of units (matrix, row tile,
+// column tile), column tiles fastest, so the Lm tile is split once per row
+// tile.  Warps 0-1 split the panel rows into the shared-memory operands
+// (K-major, 128-byte swizzle, 32-wide K atoms), warp 2 issues the MMAs into
+// one of two TMEM accumulators (256 columns each), warps 3-10 drain an
+// accumulator into the weight update while the next unit's operands and MMAs
+// proceed.
+// ---------------------------------------------------------------------------
+constexpr int kAtcRows = 256;                         // W rows per unit (MMA N)
+constexpr int kAtcCols = 128;                         // W columns per unit (MMA M)
+constexpr int kAtcProd = 2, kAtcEpi = 8;
+constexpr int kAtcThreads = 32 * (kAtcProd + 1 + kAtcEpi);
+constexpr int kAtcAtomA = kAtcCols * 128;             // one 32-wide K atom of the A (Rm) tile
+constexpr int kAtcAtomB = kAtcRows * 128;             // one 32-wide K atom of the B (Lm) tile
+static size_t atc_smem(int natoms) { return 1024 + static_cast<size_t>(natoms) * 2 * (kAtcAtomA + kAtcAtomB) + 256; }
+
+// rows [r0, r0 + R) of a panel (row stride l floats) split into hi / lo
+// swizzled K-major tiles; rows past `nrows` are zero.  Eight 16-byte loads
+// per thread are in flight before the first split.
+template <int R>
+__device__ __forceinline__ void atc_split_rows(const float* panel, int64_t r0, int64_t nrows, int l, uint8_t* hi,
+                                               uint8_t* lo, int atom_bytes, int ptid) {
+  constexpr int NT = 32 * kAtcProd, B = 8;
+  const int l4 = l >> 2;
+  const int n = R * l4;
+  const float* src = panel + r0 * l;
+  const int64_t valid = (nrows - r0) * l4;   // float4s of rows below nrows
+  for (int base = ptid; base < n; base += B * NT) {
+    float4 x[B];
+#pragma unroll
+    for (int k = 0; k < B; ++k) {
+      const int idx = base + k * NT;
+      x[k] = (idx < n && idx < valid) ? __ldg(reinterpret_cast<const float4*>(src) + idx)
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < B; ++k) {
+      const int idx = base + k * NT;
+      if (idx < n) {
+        const int r = idx / l4, c4 = idx - r * l4;
+        float4 h, lw;
+        split4(x[k], h, lw);
+        const int kk = 4 * c4;
+        const uint32_t off = static_cast<uint32_t>((kk >> 5) * atom_bytes) + sw128(r, (kk & 31) >> 2);
+        *reinterpret_cast<float4*>(hi + off) = h;
+        *reinterpret_cast<float4*>(lo + off) = lw;
+      }
+    }
+  }
+}
+
+template <typename TW>
+__global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_constant__ LApplyArgs a, int nmat,
+                                                              int natoms, int* flags) {
+  extern __shared__ uint8_t atc_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(atc_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* a_hi = smem;
+  uint8_t* a_lo = a_hi + natoms * kAtcAtomA;
+  uint8_t* b_hi = a_lo + natoms * kAtcAtomA;
+  uint8_t* b_lo = b_hi + natoms * kAtcAtomB;
+  uint64_t* opfull = reinterpret_cast<uint64_t*>(b_lo + natoms * kAtcAtomB);   // operands written
+  uint64_t* opfree = opfull + 1;                                               // MMAs done with them
+  uint64_t* tfull = opfree + 1;                                                // [2] accumulator ready
+  uint64_t* tempty = tfull + 2;                                                // [2] accumulator drained
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t rt = (a.rows + kAtcRows - 1) / kAtcRows, ct = (a.cols + kAtcCols - 1) / kAtcCols;
+  const int64_t per_mat = rt * ct;
+  const int64_t units = per_mat * nmat;
+  const int64_t u0 = units * blockIdx.x / gridDim.x, u1 = units * (blockIdx.x + 1) / gridDim.x;
+  // column tiles fastest: consecutive units of a CTA share the 256-row Lm tile
+  auto unit_of = [&](int64_t u, int& b, int64_t& i0, int64_t& j0) {
+    b = static_cast<int>(u / per_mat);
+    const int64_t rem = u - b * per_mat;
+    i0 = (rem / ct) * kAtcRows;
+    j0 = (rem % ct) * kAtcCols;
+  };
+  if (threadIdx.x == 0) {
+    tc::mbar_init(opfull, kAtcProd);
+    tc::mbar_init(opfree, 1);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&tfull[i], 1);
+      tc::mbar_init(&tempty[i], kAtcEpi);
+    }
+    *abort_flag = 0;
+    tc::fence_barrier_init();
+  }
+  if (warp == kAtcProd) {
+    tc::tmem_alloc(tmem_slot, 512);
+    tc::tmem_relinquish();
+    tc::fence_before();
+  }
+  // K columns past l up to the next multiple of 8 enter the last MMA K step
+  // and are never written below: zero the operand tiles once
+  for (int i = threadIdx.x; i < natoms * 2 * (kAtcAtomA + kAtcAtomB) / 16; i += blockDim.x)
+    reinterpret_cast<float4*>(smem)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int l = a.l;
+  const int ksteps = (l + 7) / 8;
+
+  if (warp < kAtcProd) {
+    // ---------------- operand split ----------------
+    const int ptid = threadIdx.x;
+    bool ok = true;
+    int64_t b_key = -1;
+    uint32_t it = 0;
+    for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
+      int b;
+      int64_t i0, j0;
+      unit_of(u, b, i0, j0);
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(opfree, (it & 1) ^ 1u, abort_flag));
+      if (!ok) break;
+      // the warps of this role finish the previous unit's writes before any
+      // of them overwrites a tile: the MMAs that read them are done (opfree)
+      const int64_t key = static_cast<int64_t>(b) * rt + i0 / kAtcRows;
+      if (key != b_key)
+        atc_split_rows<kAtcRows>(a.lm + b * a.lm_bs, i0, a.rows, l, b_hi, b_lo, kAtcAtomB, ptid);
+      b_key = key;
+      atc_split_rows<kAtcCols>(a.rm + b * a.rm_bs, j0, a.cols, l, a_hi, a_lo, kAtcAtomA, ptid);
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(opfull);
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
+  } else if (warp == kAtcProd) {
+    // ---------------- MMA issuer ----------------
+    const uint32_t idesc = tc::idesc_tf32(kAtcCols, kAtcRows, 0, 0);
+    bool ok = true;
+    uint32_t it = 0;
+    for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
+      const int acc = it & 1;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(opfull, it & 1, abort_flag));
+      if (!ok) break;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&tempty[acc], ((it >> 1) & 1) ^ 1u, abort_flag));
+      if (!ok) break;
+      tc::fence_after();
+      if (lane == 0) {
+        const uint32_t d = tmem_base + static_cast<uint32_t>(256 * acc);
+        for (int kk = 0; kk < ksteps; ++kk) {
+          const uint32_t off = static_cast<uint32_t>(kk & 3) * 32u;
+          const uint32_t aa = static_cast<uint32_t>(kk >> 2) * kAtcAtomA + off;
+          const uint32_t bb = static_cast<uint32_t>(kk >> 2) * kAtcAtomB + off;
+          const uint64_t dah = tc::sdesc(tc::su32(a_hi) + aa, 16, 1024), dal = tc::sdesc(tc::su32(a_lo) + aa, 16, 1024);
+          const uint64_t dbh = tc::sdesc(tc::su32(b_hi) + bb, 16, 1024), dbl = tc::sdesc(tc::su32(b_lo) + bb, 16, 1024);
+          tc::mma_tf32(d, dah, dbh, idesc, kk > 0 ? 1u : 0u);
+          tc::mma_tf32(d, dah, dbl, idesc, 1u);
+          tc::mma_tf32(d, dal, dbh, idesc, 1u);
+        }
+        tc::mma_commit(opfree);
+        tc::mma_commit(&tfull[acc]);
+      }
+      __syncwarp();
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
+  } else {
+    // ---------------- epilogue: W <- (1 - lr wd) W - lr s (Psi + D) ----------------
+    const int e = warp - kAtcProd - 1;
+    const int q = warp & 3;          // TMEM lane quarter = W columns 32 q .. 32 q + 31 of the tile
+    const int h = e >> 2;            // W rows 128 h .. 128 h + 127 of the tile
+    const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
+    const float cw = 1.f - a.lr * a.wd;
+    bool ok = true;
+    uint32_t it = 0;
+    for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
+      const int acc = it & 1;
+      int b;
+      int64_t i0, j0;
+      unit_of(u, b, i0, j0);
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&tfull[acc], (it >> 1) & 1, abort_flag));
+      if (!ok) break;
+      tc::fence_after();
+      const float nrm2 = a.stats[b * a.stats_bs + 2];
+      const float scale = nrm2 > 0.f ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
+      const float ctt = -a.lr * scale;
+      const int64_t j = j0 + 32 * q + lane;
+      const bool jok = j < a.cols;
+      const float* psi = a.psi + b * a.psi_bs + j;
+      TW* W = static_cast<TW*>(a.W[b]) + j;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        const int64_t r0 = i0 + 128 * h + 32 * c;
+        uint32_t v[32];
+        tc::tmem_ld32(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(256 * acc + 128 * h + 32 * c), v);
+        tc::tmem_ld_wait();
+        const int nr = (r0 < a.rows && jok) ? static_cast<int>(a.rows - r0 < 32 ? a.rows - r0 : 32) : 0;
+        if (nr == 32) {
+          float pv[32], wv[32];
+#pragma unroll
+          for (int rr = 0; rr < 32; ++rr) {
+            pv[rr] = __ldcs(psi + (r0 + rr) * a.psi_ld);
+            wv[rr] = to_f32(W[(r0 + rr) * a.cols]);
+          }
+#pragma unroll
+          for (int rr = 0; rr < 32; ++rr)
+            W[(r0 + rr) * a.cols] = from_f32<TW>(fmaf(cw, wv[rr], ctt * (pv[rr] + __uint_as_float(v[rr]))));
+        } else {
+#pragma unroll
+          for (int rr = 0; rr < 32; ++rr)
+            if (rr < nr) {
+              const float t = psi[(r0 + rr) * a.psi_ld] + __uint_as_float(v[rr]);
+              W[(r0 + rr) * a.cols] = from_f32<TW>(fmaf(cw, to_f32(W[(r0 + rr) * a.cols]), ctt * t));
+            }
+        }
+      }
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
+  }
+  __syncthreads();
+  if (warp == kAtcProd) {
+    __syncwarp();
+    tc::fence_after();
+    tc::tmem_dealloc(tmem_base, 512);
+  }
+}
+
+// ---------------------------------------------------------------------------
 // host orchestration
 // ---------------------------------------------------------------------------
 #define NP_FOR_LP(X) X(8) X(16) X(24) X(32) X(40) X(48) X(56) X(64) X(72)
@@ -1587,6 +1820,27 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     for (int i = 0; i < nb; ++i) {
       la.G[i] = diag ? p.G[c0 + i] : nullptr;
       la.diag[i] = diag ? p.diag + 8 * static_cast<int64_t>(p.mat_ids_host[c0 + i]) : nullptr;
+    }
+    if (!diag && l % 4 == 0 && l <= 64 && la.vec_panels) {
+      // tensor-core apply: one persistent CTA per SM over the launch's units
+      const int natoms = (l + 31) / 32;
+      // the two-atom size for every l: one CTA per SM, so the 512 TMEM
+      // columns of a CTA never wait for another's
+      const size_t smem = atc_smem(2);
+      static bool attr_f = false, attr_b = false;
+      bool& attr = g.w_dtype == 0 ? attr_f : attr_b;
+      if (!attr) {
+        e = g.w_dtype == 0 ? cudaFuncSetAttribute(k_apply_tc<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(atc_smem(2)))
+                           : cudaFuncSetAttribute(k_apply_tc<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(atc_smem(2)));
+        if (e != cudaSuccess) return e;
+        attr = true;
+      }
+      const int64_t units = cdiv(g.rows, kAtcRows) * cdiv(g.cols, kAtcCols) * nb;
+      const unsigned ctas = static_cast<unsigned>(std::min<int64_t>(units, device_sm_count()));
+      if (g.w_dtype == 0) k_apply_tc<float><<<ctas, kAtcThreads, smem, s>>>(la, nb, natoms, flags);
+      else k_apply_tc<bf16><<<ctas, kAtcThreads, smem, s>>>(la, nb, natoms, flags);
+      NP_CHECK();
+      continue;
     }
     const dim3 grid(static_cast<unsigned>(cdiv(g.cols, 64)), static_cast<unsigned>(cdiv(g.rows, 64)), nb);
 #define NP_APPLY_L(TWT, V) \
