@@ -317,14 +317,20 @@ __global__ void __launch_bounds__(kCtThreads) k_contract(const __grid_constant__
 // (N = np) adds into columns 0..np-1.
 //
 // The kernel is persistent: one CTA per SM walks the units (matrix, K split,
-// 128-row tile), carrying its 4-stage ring and accumulators from one unit to
-// the next.  Warp 0 issues the TMA copies, warps 2-9 split, warp 1 issues the
-// MMAs, which free the stage.  The tensor core's fp32 accumulation is biased
-// toward zero by up to an ulp per addition, which over thousands of K steps
-// reaches 1e-4 relative; so every kCtcSeg blocks the MMAs switch to the other
-// of two TMEM accumulators and warps 2-5 (one per TMEM lane quarter) drain the
+// 128-row tile), carrying its rings and accumulators from one unit to the
+// next.  Warp 0 issues the TMA copies into a 6-slot input ring, which the
+// split warps (2-9) free as soon as they have read a slot, so the copies run
+// ahead of the split by up to six blocks; warp 1 issues the MMAs, which free
+// the 4 operand stages (V hi / lo tiles, A hi / lo TMEM columns).  The tensor
+// core's fp32 accumulation is biased toward zero by up to an ulp per
+// addition, which over thousands of K steps reaches 1e-4 relative; so every
+// kCtcSeg blocks the MMAs switch to the other of two TMEM accumulators, and
+// warps 10-13 (one per TMEM lane quarter), which do nothing else, drain the
 // finished one into fp32 registers with round-to-nearest additions (bias
-// bounded by ~32 additions, ~2e-6), and write each unit's result.
+// bounded by ~32 additions, ~2e-6) and write each unit's result.  (Draining
+// from split warps stalled the split for the MMAs' completion every segment;
+// sixteen split warps with eight drain warps measured slower than eight and
+// four.)
 // ---------------------------------------------------------------------------
 struct ContractTcArgs {
   CUtensorMap psi_map;    // {cols, rows, batch} fp32, 128-byte swizzle
@@ -336,17 +342,22 @@ struct ContractTcArgs {
   int ksplit, batch;      // K splits and matrices (the units are tiles x ksplit x batch)
   int* flags;
 };
-// Stage st of the ring: copies of the Psi block and of the V block (TMA),
-// the split V hi / lo tiles in shared memory and the split A hi / lo in TMEM;
-// the MMAs free the stage.
-constexpr int kCtcStages = 4;
+// Two rings.  The input ring holds the TMA copies of the Psi block and of the
+// V block; the split warps free a slot as soon as they have read it, so the
+// copies run up to kCtcIn blocks ahead of the split and the HBM latency is
+// covered by the copies in flight.  The MMA stages hold the split V hi / lo
+// tiles in shared memory and the split A hi / lo in TMEM; the MMAs free them.
+constexpr int kCtcIn = 6;                            // input ring slots
+constexpr int kCtcStages = 4;                        // MMA operand stages
 constexpr int kCtcSeg = 4;                           // K blocks per accumulator segment
 constexpr int kCtcA = 128 * 32 * 4;                  // one A tile (128 rows x 32 K): 16 KB
 constexpr int kCtcV = 64 * 32 * 4;                   // one V tile (64 rows x 32 K): 8 KB
-constexpr int kCtcStage = kCtcA + 3 * kCtcV;         // A copy, V copy, V hi, V lo: 40 KB
+constexpr int kCtcInSlot = kCtcA + kCtcV;            // Psi copy, V copy: 24 KB
+constexpr int kCtcStage = 2 * kCtcV;                 // V hi, V lo: 16 KB
 constexpr int kCtcSplitWarps = 8;
-constexpr int kCtcThreads = 64 + 32 * kCtcSplitWarps; // TMA, MMA, 8 split warps
-constexpr size_t kCtcSmem = 1024 + kCtcStages * kCtcStage + 512;
+constexpr int kCtcDrainWarps = 4;
+constexpr int kCtcThreads = 64 + 32 * (kCtcSplitWarps + kCtcDrainWarps);   // TMA, MMA, split, drain
+constexpr size_t kCtcSmem = 1024 + kCtcIn * kCtcInSlot + kCtcStages * kCtcStage + 512;
 // TMEM columns: two 128-column accumulators, then per stage 32 columns of A
 // hi and 32 of A lo
 constexpr uint32_t kCtcTmemA = 256;
@@ -399,6 +410,15 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float* v) {
       : "memory");
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// 32 TMEM lanes x 16 consecutive 32-bit columns: thread i receives lane (base + i).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
 // D[tmem] (+)= A[tmem] * B[smem]^T, kind::tf32
 __device__ __forceinline__ void mma_tf32_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
                                             uint32_t accumulate) {
@@ -414,17 +434,20 @@ template <bool TRANS>
 __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_constant__ ContractTcArgs a) {
   extern __shared__ uint8_t ctc_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(ctc_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kCtcStages * kCtcStage);   // [kCtcStages] copies landed
-  uint64_t* splitb = full + kCtcStages;      // [kCtcStages] split written
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kCtcIn * kCtcInSlot + kCtcStages * kCtcStage);
+                                             // [kCtcIn] copies landed
+  uint64_t* inempty = full + kCtcIn;         // [kCtcIn] split warps done reading the slot
+  uint64_t* splitb = inempty + kCtcIn;       // [kCtcStages] split written
   uint64_t* empty = splitb + kCtcStages;     // [kCtcStages] MMAs done with the stage
   uint64_t* tfull = empty + kCtcStages;      // [2] accumulator segment complete
   uint64_t* tempty = tfull + 2;              // [2] accumulator drained
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [kCtcStages] last parity + 1
-  // stage layout: A copy | V copy | V hi | V lo
-  auto a_copy = [&](int st) { return smem + st * kCtcStage; };
-  auto v_copy = [&](int st) { return smem + st * kCtcStage + kCtcA; };
+  uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [kCtcIn] last parity + 1
+  // input slot: A copy | V copy; MMA stage: V hi | V lo
+  auto a_copy = [&](int i) { return smem + i * kCtcInSlot; };
+  auto v_copy = [&](int i) { return smem + i * kCtcInSlot + kCtcA; };
+  auto v_split = [&](int st) { return smem + kCtcIn * kCtcInSlot + st * kCtcStage; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nvb = a.np > 32 ? 2 : 1;
@@ -442,15 +465,18 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
     nk = kend > kbeg ? static_cast<int>((kend - kbeg + 31) / 32) : 0;
   };
   if (threadIdx.x == 0) {
+    for (int i = 0; i < kCtcIn; ++i) {
+      tc::mbar_init(&full[i], 1);
+      tc::mbar_init(&inempty[i], kCtcSplitWarps);
+      issued[i] = 0;
+    }
     for (int st = 0; st < kCtcStages; ++st) {
-      tc::mbar_init(&full[st], 1);
       tc::mbar_init(&splitb[st], kCtcSplitWarps);
       tc::mbar_init(&empty[st], 1);
-      issued[st] = 0;
     }
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&tfull[i], 1);
-      tc::mbar_init(&tempty[i], 4);
+      tc::mbar_init(&tempty[i], kCtcDrainWarps);
     }
     *abort_flag = 0;
     tc::fence_barrier_init();
@@ -467,7 +493,7 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
   if (nvb == 1)
     for (int st = 0; st < kCtcStages; ++st)
       for (int i = threadIdx.x; i < 2 * kCtcV / 16; i += blockDim.x)
-        reinterpret_cast<float4*>(v_copy(st) + kCtcV)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        reinterpret_cast<float4*>(v_split(st))[i] = make_float4(0.f, 0.f, 0.f, 0.f);
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   __syncthreads();
   tc::fence_after();
@@ -482,21 +508,21 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
       int64_t p0, kbeg;
       unit_of(u, b, z, p0, kbeg, nk);
       for (int kb = 0; kb < nk && ok; ++kb, ++it) {
-        const int st = it % kCtcStages;
-        const uint32_t ph = (it / kCtcStages) & 1;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[st], ph ^ 1u, abort_flag));
+        const int i = it % kCtcIn;
+        const uint32_t ph = (it / kCtcIn) & 1;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&inempty[i], ph ^ 1u, abort_flag));
         if (!ok) break;
         if (lane == 0) {
-          tc::mbar_expect_tx(&full[st], static_cast<uint32_t>(kCtcA + nvb * 4096));
-          issued[st] = ph + 1;
+          tc::mbar_expect_tx(&full[i], static_cast<uint32_t>(kCtcA + nvb * 4096));
+          issued[i] = ph + 1;
           const int k0 = static_cast<int>(kbeg) + 32 * kb, pr = static_cast<int>(p0);
           if (!TRANS) {
-            tc::tma_load_3d(a_copy(st), &a.psi_map, &full[st], k0, pr, b);
+            tc::tma_load_3d(a_copy(i), &a.psi_map, &full[i], k0, pr, b);
           } else {
 #pragma unroll
-            for (int j = 0; j < 4; ++j) tc::tma_load_3d(a_copy(st) + j * 4096, &a.psi_map, &full[st], pr + 32 * j, k0, b);
+            for (int j = 0; j < 4; ++j) tc::tma_load_3d(a_copy(i) + j * 4096, &a.psi_map, &full[i], pr + 32 * j, k0, b);
           }
-          for (int j = 0; j < nvb; ++j) tc::tma_load_3d(v_copy(st) + j * 4096, &a.v_map, &full[st], 32 * j, k0, b);
+          for (int j = 0; j < nvb; ++j) tc::tma_load_3d(v_copy(i) + j * 4096, &a.v_map, &full[i], 32 * j, k0, b);
         }
         __syncwarp();
       }
@@ -530,7 +556,7 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(128 * acc);
         if (lane == 0) {
           const uint32_t ahi = tmem_base + kCtcTmemA + 64u * st, alo = ahi + 32u;
-          const uint32_t vhi = tc::su32(v_copy(st) + kCtcV);   // V lo follows at row 64
+          const uint32_t vhi = tc::su32(v_split(st));   // V lo follows at row 64
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {       // K step of 8: 8 TMEM columns of A, 32 bytes of a V row
             const uint64_t dv = tc::sdesc(vhi + kk * 32, 16, 1024);
@@ -545,55 +571,30 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
       }
     }
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
-  } else {
-    // ---------------- split (warps 2..9), segment drains and epilogues (warps 2..5) ----------------
+  } else if (warp < 2 + kCtcSplitWarps) {
+    // ---------------- split (warps 2..9) ----------------
     const int w = warp - 2;
-    const bool drainer = w < 4;
     const int q = warp & 3;        // TMEM lane quarter this warp may access
     const int kh = w >> 2;         // half of each 32-deep K block this warp splits
-    float sum[64];
-    // adds the accumulator of segment `seg` into sum (round to nearest) and
-    // hands the accumulator back to the MMA warp
-    auto drain = [&](uint32_t seg) -> bool {
-      const int acc = seg & 1;
-      if (!__all_sync(0xffffffffu, tc::mbar_wait(&tfull[acc], (seg >> 1) & 1, abort_flag))) return false;
-      tc::fence_after();
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        if (32 * h < a.np) {
-          // Ahi Vhi + Alo Vhi in columns 32 h.., Ahi Vlo in 64 + 32 h..
-          uint32_t r[32], v[32];
-          const uint32_t col = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * acc + 32 * h);
-          tc::tmem_ld32(col, r);
-          tc::tmem_ld32(col + 64u, v);
-          tc::tmem_ld_wait();
-#pragma unroll
-          for (int j = 0; j < 32; ++j) sum[32 * h + j] += __uint_as_float(r[j]) + __uint_as_float(v[j]);
-        }
-      }
-      tc::fence_before();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&tempty[acc]);
-      return true;
-    };
     bool ok = true;
-    uint32_t it = 0, gseg = 0;
+    uint32_t it = 0;
     for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
       int b, z, nk;
       int64_t p0, kbeg;
       unit_of(u, b, z, p0, kbeg, nk);
-#pragma unroll
-      for (int j = 0; j < 64; ++j) sum[j] = 0.f;
       for (int kb = 0; kb < nk && ok; ++kb, ++it) {
         const int st = it % kCtcStages;
         const uint32_t ph = (it / kCtcStages) & 1;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(&full[st], ph, abort_flag));
+        const int in = it % kCtcIn;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&full[in], (it / kCtcIn) & 1, abort_flag));
         if (!ok) break;
-        // this stage's TMEM columns were last read by MMAs whose completion
-        // reached here through the empty -> TMA -> full chain
+        // the MMAs are done with this stage's TMEM columns and V tiles
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&empty[st], ph ^ 1u, abort_flag));
+        if (!ok) break;
         tc::fence_after();
-        const uint8_t* ac = a_copy(st);
-        uint8_t* vc = v_copy(st);
+        const uint8_t* ac = a_copy(in);
+        const uint8_t* vc = v_copy(in);
+        uint8_t* vs = v_split(st);
         // A row r = 32 q + lane (the warp's TMEM lane quarter), K half kh
         {
           const int r = 32 * q + lane;
@@ -621,29 +622,60 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
         }
         // V (box w / 4, chunk pair w % 4 of two boxes, or box 0, chunk w of
         // one) while the TMEM stores drain
-        if (nvb == 2) split_transpose<2>(vc + (w >> 2) * 4096, vc + kCtcV, vc + 2 * kCtcV, 32 * (w >> 2), lane, 2 * (w & 3));
-        else split_transpose<1>(vc, vc + kCtcV, vc + 2 * kCtcV, 0, lane, w);
+        if (nvb == 2) split_transpose<2>(vc + (w >> 2) * 4096, vs, vs + kCtcV, 32 * (w >> 2), lane, 2 * (w & 3));
+        else split_transpose<1>(vc, vs, vs + kCtcV, 0, lane, w);
+        // every read of the input slot has returned: hand it back to the copies
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&inempty[in]);
         tmem_st_wait();
         // the MMAs read V through the async proxy and A from TMEM
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         tc::fence_before();
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&splitb[st]);
-        // the previous segment of this unit ends with the block before this
-        // one: drain it while the MMAs of this segment start
-        if (kb % kCtcSeg == 0 && kb > 0) {
-          if (drainer) ok = drain(gseg);
-          ++gseg;
+      }
+    }
+    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(a.flags, kFlagTimeout); }
+  } else {
+    // ---------------- accumulator drains and unit results (warps 10..13) ----------------
+    const int q = warp & 3;        // TMEM lane quarter: rows 32 q .. 32 q + 31 of the unit
+    float sum[64];
+    bool ok = true;
+    uint32_t gseg = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      int b, z, nk;
+      int64_t p0, kbeg;
+      unit_of(u, b, z, p0, kbeg, nk);
+#pragma unroll
+      for (int j = 0; j < 64; ++j) sum[j] = 0.f;
+      // segments of kCtcSeg K blocks, as the MMA warp closes them
+      const int nseg = (nk + kCtcSeg - 1) / kCtcSeg;
+      for (int sg = 0; sg < nseg && ok; ++sg, ++gseg) {
+        const int acc = gseg & 1;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(&tfull[acc], (gseg >> 1) & 1, abort_flag));
+        if (!ok) break;
+        tc::fence_after();
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          if (16 * h < a.np) {
+            // Ahi Vhi + Alo Vhi in columns 16 h.., Ahi Vlo in 64 + 16 h..
+            uint32_t r[16], v[16];
+            const uint32_t col = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * acc + 16 * h);
+            tmem_ld16(col, r);
+            tmem_ld16(col + 64u, v);
+            tc::tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 16; ++j) sum[16 * h + j] += __uint_as_float(r[j]) + __uint_as_float(v[j]);
+          }
         }
+        tc::fence_before();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&tempty[acc]);
       }
       if (!ok) break;
-      if (nk > 0) {
-        if (drainer) ok = drain(gseg);
-        ++gseg;
-      }
       const int64_t row = p0 + 32 * q + lane;
       float* out = a.out + b * a.out_bs + static_cast<int64_t>(z) * a.P * a.l;
-      if (drainer && ok && row < a.P) {
+      if (row < a.P) {
 #pragma unroll
         for (int j = 0; j < 64; ++j)
           if (j < a.l) out[row * a.l + j] = sum[j];
@@ -655,8 +687,8 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
   if (threadIdx.x == 0 && *abort_flag) {
     // let every TMA copy still in flight land before the CTA exits
     volatile int never = 0;
-    for (int st = 0; st < kCtcStages; ++st)
-      if (issued[st]) tc::mbar_wait(&full[st], issued[st] - 1, &never);
+    for (int i = 0; i < kCtcIn; ++i)
+      if (issued[i]) tc::mbar_wait(&full[i], issued[i] - 1, &never);
   }
   __syncthreads();
   if (warp == 1) {
