@@ -39,7 +39,7 @@
 namespace normpre {
 
 constexpr int kLmax = 72;        // largest supported sketch width l (r = 64 with o = 8)
-constexpr int kGramRows = 64;    // rows per fp32 chunk of the split Gram sums
+constexpr int kGramRows = 128;   // rows per fp32 chunk of the split Gram sums
 constexpr int kMaxKSplit = 8;    // split-K factor bound of the contractions
 
 // Kahan-compensated accumulator
@@ -725,23 +725,78 @@ struct GramArgs {
   int l;
   int nsplit;
 };
+// One CTA per chunk.  The chunk is staged in shared memory; each thread
+// accumulates a 4 x 4 block of the l x l sum over its share of the rows in
+// registers (two 16-byte shared loads per 16 FMAs); when the blocks do not
+// fill the CTA the rows are split into 2 or 4 groups whose sums are added in
+// a fixed order.
 __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramArgs a) {
-  __shared__ float ys[kGramRows][kLmax + 1];
-  const int b = blockIdx.y, s = blockIdx.x, l = a.l;
+  constexpr int LD = kLmax + 4;                  // 16-byte rows
+  __shared__ __align__(16) float ys[kGramRows * LD];
+  const int b = blockIdx.y, s = blockIdx.x, l = a.l, tid = threadIdx.x;
+  const int l4 = (l + 3) >> 2, lp = 4 * l4;
   const int64_t i0 = static_cast<int64_t>(s) * kGramRows;
-  const float* y = a.y + b * a.y_bs;
-  for (int e = threadIdx.x; e < kGramRows * l; e += blockDim.x) {
+  const int64_t nval = (a.n - i0 < kGramRows ? a.n - i0 : static_cast<int64_t>(kGramRows)) * l;   // valid floats of the chunk
+  const float* y = a.y + b * a.y_bs + i0 * l;    // the chunk's rows are contiguous
+  for (int e = tid; e < kGramRows * l; e += blockDim.x) {
     const int i = e / l, j = e - i * l;
-    ys[i][j] = (i0 + i < a.n) ? y[(i0 + i) * l + j] : 0.f;
+    ys[i * LD + j] = e < nval ? __ldg(y + e) : 0.f;
+  }
+  for (int e = tid; e < kGramRows * (lp - l); e += blockDim.x) {
+    const int i = e / (lp - l), j = l + (e - i * (lp - l));
+    ys[i * LD + j] = 0.f;
   }
   __syncthreads();
+  const int tiles = l4 * l4;
+  const int groups = tiles <= 64 ? 4 : (tiles <= 128 ? 2 : 1);
+  const int rows_g = kGramRows / groups;
   float* out = a.part + b * a.part_bs + static_cast<int64_t>(s) * l * l;
-  for (int e = threadIdx.x; e < l * l; e += blockDim.x) {
+  float acc[4][4];
+  int my_tile = -1, my_group = 0;
+  for (int t = tid; t < tiles * groups; t += blockDim.x) {
+    const int tile = t % tiles, g = t / tiles;
+    const int p0 = 4 * (tile / l4), q0 = 4 * (tile % l4);
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+    const float* yb = ys + g * rows_g * LD;
+#pragma unroll 4
+    for (int i = 0; i < rows_g; ++i) {
+      const float4 pv = *reinterpret_cast<const float4*>(yb + i * LD + p0);
+      const float4 qv = *reinterpret_cast<const float4*>(yb + i * LD + q0);
+      const float pa[4] = {pv.x, pv.y, pv.z, pv.w}, qa[4] = {qv.x, qv.y, qv.z, qv.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(pa[r], qa[c], acc[r][c]);
+    }
+    if (groups == 1) {
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          if (p0 + r < l && q0 + c < l) out[(p0 + r) * l + q0 + c] = acc[r][c];
+    } else {
+      my_tile = tile;     // one (tile, group) per thread when groups > 1
+      my_group = g;
+    }
+  }
+  if (groups == 1) return;
+  __syncthreads();                                // every read of ys is done: reuse it
+  if (my_tile >= 0) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) ys[(my_group * tiles + my_tile) * 16 + 4 * r + c] = acc[r][c];
+  }
+  __syncthreads();
+  for (int e = tid; e < l * l; e += blockDim.x) {
     const int p = e / l, q = e - p * l;
-    float acc = 0.f;
-#pragma unroll 8
-    for (int i = 0; i < kGramRows; ++i) acc = fmaf(ys[i][p], ys[i][q], acc);
-    out[e] = acc;
+    const int tile = (p >> 2) * l4 + (q >> 2), k = 4 * (p & 3) + (q & 3);
+    float v = 0.f;
+    for (int g = 0; g < groups; ++g) v += ys[(g * tiles + tile) * 16 + k];
+    out[e] = v;
   }
 }
 
@@ -928,20 +983,38 @@ struct RowMulArgs {
   int64_t n;
   int l;
 };
+// One thread per (row, 8 consecutive columns): the row's entries are
+// broadcast loads shared by its threads, S's rows 16-byte shared loads.
 __global__ void __launch_bounds__(256) k_rowmul(const __grid_constant__ RowMulArgs a) {
-  __shared__ float S[kLmax * kLmax];
+  __shared__ __align__(16) float S[kLmax * (kLmax + 8)];
   const int b = blockIdx.y, l = a.l;
+  const int lp = (l + 7) & ~7, ld = lp;          // S rows padded with zeros to 8 columns
   const float* s = a.s + b * a.s_bs;
-  for (int e = threadIdx.x; e < l * l; e += blockDim.x) S[e] = s[e];
+  for (int e = threadIdx.x; e < l * lp; e += blockDim.x) {
+    const int k = e / lp, j = e - k * lp;
+    S[k * ld + j] = j < l ? s[k * l + j] : 0.f;
+  }
   __syncthreads();
-  const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (e >= a.n * l) return;
-  const int64_t i = e / l;
-  const int j = static_cast<int>(e - i * l);
+  const int cg = lp >> 3;                        // column groups per row
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (t >= a.n * cg) return;
+  const int64_t i = t / cg;
+  const int j0 = 8 * static_cast<int>(t - i * cg);
   const float* y = a.y + b * a.y_bs + i * l;
-  float acc = 0.f;
-  for (int k = 0; k < l; ++k) acc = fmaf(y[k], S[k * l + j], acc);
-  a.out[b * a.out_bs + e] = acc;
+  float acc[8] = {};
+  for (int k = 0; k < l; ++k) {
+    const float yk = __ldg(y + k);
+    const float4 s0 = *reinterpret_cast<const float4*>(S + k * ld + j0);
+    const float4 s1 = *reinterpret_cast<const float4*>(S + k * ld + j0 + 4);
+    acc[0] = fmaf(yk, s0.x, acc[0]); acc[1] = fmaf(yk, s0.y, acc[1]);
+    acc[2] = fmaf(yk, s0.z, acc[2]); acc[3] = fmaf(yk, s0.w, acc[3]);
+    acc[4] = fmaf(yk, s1.x, acc[4]); acc[5] = fmaf(yk, s1.y, acc[5]);
+    acc[6] = fmaf(yk, s1.z, acc[6]); acc[7] = fmaf(yk, s1.w, acc[7]);
+  }
+  float* o = a.out + b * a.out_bs + i * l + j0;
+#pragma unroll
+  for (int c = 0; c < 8; ++c)
+    if (j0 + c < l) o[c] = acc[c];
 }
 
 // ---------------------------------------------------------------------------
@@ -1825,7 +1898,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     RowMulArgs rm;
     rm.y = g.q; rm.y_bs = vbs; rm.s = g.kmat; rm.s_bs = sq;
     rm.out = g.qk; rm.out_bs = vbs; rm.n = m_a; rm.l = l;
-    k_rowmul<<<dim3(static_cast<unsigned>(cdiv(m_a * l, 256)), B), 256, 0, s>>>(rm);
+    k_rowmul<<<dim3(static_cast<unsigned>(cdiv(m_a * ((l + 7) / 8), 256)), B), 256, 0, s>>>(rm);
     NP_CHECK();
   }
   prof->end(kProfEig, s, (p.exact ? 1 : 3) + n_fold);
