@@ -243,6 +243,7 @@ struct SketchGroup {
   float* ritz = nullptr;        // [l]
   float* zvec = nullptr;        // [l][l]
   float* stats = nullptr;       // [8] per matrix
+  float* rfac = nullptr;        // CholeskyQR factor of one pass, per matrix
   int lmax = 0;
   int max_part = 0;
   // NORMPRE_L_EXACT: Gamma of one matrix (then its eigenvectors), its

@@ -847,9 +847,10 @@ __global__ void __launch_bounds__(256) k_gram_fold(const __grid_constant__ GramF
 }
 
 // ---------------------------------------------------------------------------
-// One CholeskyQR pass, fused: every CTA loads the Gram matrix G of Y, factors
-// G = R^T R (upper R, fp32) and then solves q R = y for 256 rows of Y, one
-// row per thread.  A pivot below 1e-6 tr(G) means Y is numerically rank
+// One CholeskyQR pass: one CTA per matrix folds the Gram matrix G of Y and
+// factors G = R^T R (upper R, fp32); then every CTA of the solve reads R and
+// solves q R = y for 256 rows of Y, one row per thread.  A pivot below
+// 1e-6 tr(G) means Y is numerically rank
 // deficient there: the first pass retries with the diagonal shifted by
 // 1e-5 tr(G); the later passes, whose input is already well conditioned
 // wherever it is not rank deficient, drop that column instead (a zero
@@ -858,9 +859,9 @@ __global__ void __launch_bounds__(256) k_gram_fold(const __grid_constant__ GramF
 // The factorization is right-looking over the whole CTA (one pivot per
 // barrier, the trailing square updated by a 16 x 16 thread grid); the solve
 // is column-oriented (x_k final, then every later x_j updated from row k of
-// R), so its dependent chain is l steps long, not l^2 / 2.  The
-// factorization is repeated by each CTA of a matrix: it is tiny next to the
-// row solves.
+// R), so its dependent chain is l steps long, not l^2 / 2.  (Repeating the
+// factorization in every solve CTA cost 1344 factorizations a pass on the
+// 56 Qwen3 MLP matrices of 6144 rows.)
 // ---------------------------------------------------------------------------
 struct CholQRArgs {
   const float* part; int64_t part_bs; int nsplit;
@@ -871,15 +872,22 @@ struct CholQRArgs {
   int drop;      // 0: shifted retry on a small pivot (first pass); 1: drop its column
   int* flags;
 };
+// Per matrix [R (LP x LP, strictly upper, rows scaled by 1 / R_ii) | 1 / R_ii
+// (LP) | zero-panel flag]: the factorization of one CholeskyQR pass, made
+// once per matrix by k_chol_factor and read by every CTA of k_chol_solve.
+constexpr int kRfacStride = kLmax * kLmax + kLmax + 8;
+
+// One CTA per matrix: fold the Gram partials of the panel, factor G (+ shift)
+// = R^T R right-looking (one pivot per barrier), write R and 1 / R_ii.
 template <int LP>
-__global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRArgs a) {
-  // G (row stride LP + 1) until the factorization ends, then R strictly above
-  // the diagonal and zero elsewhere (row stride LP, 16-byte rows)
+__global__ void __launch_bounds__(256) k_chol_factor(const __grid_constant__ CholQRArgs a, float* rfac) {
+  // G (row stride LP + 1) until the factorization ends
   __shared__ __align__(16) float GR[LP * (LP + 1)];
   __shared__ float Wm[LP][LP + 1];             // G + shift I, reduced in place
   __shared__ float rinv[LP];                   // 1 / R_jj (zero past l)
   __shared__ float tr;
-  const int b = blockIdx.y, l = a.l, tid = threadIdx.x;
+  const int b = blockIdx.x, l = a.l, tid = threadIdx.x;
+  float* out = rfac + static_cast<int64_t>(b) * kRfacStride;
   fold_partials(a.part + b * a.part_bs, a.nsplit, l, GR, LP + 1);
   __syncthreads();
   if (tid < 32) {
@@ -889,13 +897,9 @@ __global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRAr
     if (tid == 0) tr = t;
   }
   __syncthreads();
-  const int64_t row = static_cast<int64_t>(blockIdx.x) * 256 + tid;
-  const float* y = a.y + b * a.v_bs + row * l;
-  float* q = a.q + b * a.v_bs + row * l;
   if (!(tr > 0.f)) {
     // Y = 0 (a zero normalized update): Q = 0, nothing is selected downstream
-    if (row < a.n)
-      for (int j = 0; j < l; ++j) q[j] = 0.f;
+    if (tid == 0) out[LP * LP + LP] = 1.f;
     return;
   }
   // right-looking Cholesky: at pivot j, W[p][q] -= W[j][p] W[j][q] / W[j][j]
@@ -926,7 +930,7 @@ __global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRAr
     }
     if (!bad || a.drop) break;     // every thread saw the same pivots
   }
-  if (tid == 0 && bad && !a.drop && blockIdx.x == 0) raise_flag(a.flags, kFlagNumeric);
+  if (tid == 0 && bad && !a.drop) raise_flag(a.flags, kFlagNumeric);
   // W[i][i] is pivot i; a dropped column gets 1 / R_ii = 0 (and so a zero row of R)
   for (int i = tid; i < LP; i += 256) {
     const float d = (i < l) ? Wm[i][i] : 0.f;
@@ -935,8 +939,31 @@ __global__ void __launch_bounds__(256) k_cholqr(const __grid_constant__ CholQRAr
   __syncthreads();
   for (int e = tid; e < LP * LP; e += 256) {
     const int i = e / LP, j = e % LP;
-    GR[e] = (i < l && j < l && j > i) ? Wm[i][j] * rinv[i] : 0.f;
+    out[e] = (i < l && j < l && j > i) ? Wm[i][j] * rinv[i] : 0.f;
   }
+  for (int i = tid; i < LP; i += 256) out[LP * LP + i] = rinv[i];
+  if (tid == 0) out[LP * LP + LP] = 0.f;
+}
+
+// The rows of Q: q R = y, one row per thread, with R from k_chol_factor.
+template <int LP>
+__global__ void __launch_bounds__(256) k_chol_solve(const __grid_constant__ CholQRArgs a, const float* rfac) {
+  __shared__ __align__(16) float GR[LP * LP];  // R strictly above the diagonal, 16-byte rows
+  __shared__ float rinv[LP];
+  const int b = blockIdx.y, l = a.l, tid = threadIdx.x;
+  const float* in = rfac + static_cast<int64_t>(b) * kRfacStride;
+  const bool zero = in[LP * LP + LP] != 0.f;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * 256 + tid;
+  const float* y = a.y + b * a.v_bs + row * l;
+  float* q = a.q + b * a.v_bs + row * l;
+  if (zero) {
+    if (row < a.n)
+      for (int j = 0; j < l; ++j) q[j] = 0.f;
+    return;
+  }
+  for (int e = tid; e < LP * LP / 4; e += 256)
+    reinterpret_cast<float4*>(GR)[e] = __ldg(reinterpret_cast<const float4*>(in) + e);
+  for (int i = tid; i < LP; i += 256) rinv[i] = in[LP * LP + i];
   __syncthreads();
   if (row >= a.n) return;
   float x[LP];
@@ -1625,10 +1652,10 @@ static void contract_attrs() {
 #undef NP_CT
 }
 
-static cudaError_t launch_cholqr(const CholQRArgs& c, int batch, int lp, cudaStream_t s) {
+static cudaError_t launch_cholqr(const CholQRArgs& c, float* rfac, int batch, int lp, cudaStream_t s) {
   const dim3 grid(static_cast<unsigned>(cdiv(c.n, 256)), static_cast<unsigned>(batch));
   switch (lp) {
-#define NP_CQ(N) case N: k_cholqr<N><<<grid, 256, 0, s>>>(c); break;
+#define NP_CQ(N) case N: k_chol_factor<N><<<batch, 256, 0, s>>>(c, rfac); k_chol_solve<N><<<grid, 256, 0, s>>>(c, rfac); break;
     NP_FOR_LP(NP_CQ)
 #undef NP_CQ
     default:
@@ -1662,6 +1689,7 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
   if ((e = alloc((void**)&g.ritz, static_cast<size_t>(g.batch) * g.lmax * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.zvec, sq * sizeof(float)))) return e;
   if ((e = alloc((void**)&g.stats, static_cast<size_t>(g.batch) * 8 * sizeof(float)))) return e;
+  if ((e = alloc((void**)&g.rfac, static_cast<size_t>(g.batch) * kRfacStride * sizeof(float)))) return e;
   contract_attrs<false>();
   contract_attrs<true>();
   // tensor-core contractions: Psi as a 3-D tensor {cols, rows, batch}; the
@@ -1701,6 +1729,7 @@ cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup
   s.zvec = g.zvec + b0 * sq;
   s.ritz = g.ritz + static_cast<int64_t>(b0) * g.lmax;
   s.stats = g.stats + static_cast<int64_t>(b0) * 8;
+  s.rfac = g.rfac + static_cast<int64_t>(b0) * kRfacStride;
   if (g.eig_all) s.eig_all = g.eig_all + b0 * std::max(g.rows, g.cols);
   if (g.tc) {
     const uint64_t dims[3] = {static_cast<uint64_t>(g.cols), static_cast<uint64_t>(g.rows),
@@ -1863,11 +1892,11 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
         cq.vec = (l % 4 == 0) && (vbs % 4 == 0) && (reinterpret_cast<uintptr_t>(src) % 16 == 0) &&
                  (reinterpret_cast<uintptr_t>(dst) % 16 == 0);
         cq.drop = (pass > 0);
-        if ((e = launch_cholqr(cq, B, lp, s))) return e;
+        if ((e = launch_cholqr(cq, g.rfac, B, lp, s))) return e;
         src = dst;
       }
     }
-    prof->end(kProfQR, s, 6 + n_fold);
+    prof->end(kProfQR, s, 9 + n_fold);
     n_fold = 0;
     // B^T = Psi_a^T Q  [n_a x l];  Gamma_Q = B B^T
     if ((e = contract(tb, g.q, g.bt))) return e;
