@@ -46,7 +46,7 @@ from synth import inputs as S  # noqa: E402
 METRIC = "NormPre step ms per model param set; NS TFLOP/s & normalize GB/s vs peak"
 DEFAULT_CONFIG = "qwen3_1p7b"
 LR = 0.02
-FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # 80.5 TFLOP/s, for the ALU-bound k_gamma
+FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # 80.5 TFLOP/s, for the fp32 exact-variant sweeps
 L2_BYTES = 129e6                                    # GB300 L2
 
 # Traffic of one launch of the dominant kernel class from an ncu capture
@@ -262,7 +262,7 @@ def run_reference(args, cfg, variant, rank, world):
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
-def _roofline(cfg, variant, prof, steps, clocks):
+def _roofline(cfg, variant, prof, steps, clocks, exact_sweeps=None):
     hbm, bf16_burst, bf16_sust, peak_src = measured_peaks()
     n_el = cfg.elements
     if variant == "G":
@@ -287,21 +287,31 @@ def _roofline(cfg, variant, prof, steps, clocks):
                 "frac_nominal": fl / (ns_ms * 1e-3) / 1e12 / peak,
                 "traffic": NCU_TRAFFIC_PER_LAUNCH.get((cfg.name, variant))}
     if variant == "L_exact":
-        # k_gamma: Gamma = Psi_a Psi_a^T on the fp32 FMA pipes (both triangles,
-        # 2 m_a^2 n_a flops per matrix); the dense eigensolver is a library call
-        gam_ms = prof["gamma"][0] / steps
-        gam_launches = prof["gamma"][1] / steps
-        k_even = sum(2.0 * m.rows * m.rows * m.cols for m in cfg.matrices)
-        k_odd = sum(2.0 * m.cols * m.cols * m.rows for m in cfg.matrices)
-        fl = (k_even + k_odd) / 2.0          # row- and column-active steps alternate
-        achieved = fl / (gam_ms * 1e-3) / 1e12
-        return {"bound": "alu", "kernel": "k_gamma (Gamma = Psi_a Psi_a^T, fp32 FMA)",
+        # the one-sided block Jacobi sweeps over Psi on the fp32 FMA pipes: per
+        # sweep of a matrix, (nb - 1) rounds of nb / 2 column-block pairs, each
+        # a 64-column Gram matrix and a rotation of the 64 columns (2 * 2 lp 64^2
+        # flops, lp = the long side padded to 64); counted for every pair of the
+        # sweeps that rotated (a pair found orthogonal skips its rotation, so
+        # this is an upper bound of the work)
+        sw_ms = prof["exact_sweeps"][0] / steps
+        sw_launches = prof["exact_sweeps"][1] / steps
+        fl = 0.0
+        for m, sweeps in zip(cfg.matrices, exact_sweeps or []):
+            s_pad = -(-min(m.rows, m.cols) // 64) * 64
+            lp = -(-max(m.rows, m.cols) // 64) * 64
+            nb = s_pad // 32
+            fl += sweeps * (nb - 1) * (nb // 2) * 4.0 * lp * 64 * 64
+        achieved = fl / (sw_ms * 1e-3) / 1e12
+        return {"bound": "alu", "kernel": "k_oj_round (one-sided block Jacobi of Psi, fp32 FMA)",
                 "achieved": achieved, "peak": FP32_FMA_TFLOPS, "unit": "TFLOP/s",
                 "frac": achieved / FP32_FMA_TFLOPS,
                 "peak_source": "nominal fp32 FMA rate: 152 SMs x 128 lanes x 2 flops x 2.07 GHz",
-                "flops_per_launch": fl / gam_launches, "ms_per_launch": gam_ms / gam_launches,
-                "launches_per_step": gam_launches,
-                "syevd_ms_per_step": prof["syevd"][0] / steps,
+                "flops_note": "Gram and rotation flops of every column-block pair in the sweeps that rotated "
+                              "(the last step's sweep counts); an upper bound of the executed work",
+                "flops_per_launch": fl / max(sw_launches, 1), "ms_per_launch": sw_ms / max(sw_launches, 1),
+                "launches_per_step": sw_launches,
+                "select_ms_per_step": prof["exact_select"][0] / steps,
+                "sweeps_per_matrix": exact_sweeps,
                 "traffic": None}
     con_ms = prof["contract"][0] / steps
     con_launches = prof["contract"][1] / steps
@@ -412,7 +422,10 @@ def measure_variant(args, cfg, variant, host, dev):
     norm_ms = prof["normalize"][0] / args.steps
     phases = {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps}
               for k, v in prof.items() if v[1] > 0}
-    roof = _roofline(cfg, variant, prof, args.steps, clocks)
+    exact_sweeps = None
+    if variant == "L_exact":
+        exact_sweeps = [int(opt.read(i, C.NORMPRE_BUF_STATS)[0][7]) for i in range(cfg.n_mats)]
+    roof = _roofline(cfg, variant, prof, args.steps, clocks, exact_sweeps)
     norm_gbs = n_el * b_norm / (norm_ms * 1e-3) / 1e9 if norm_ms > 0 else None
 
     # ---- end to end through the C ABI on pinned host buffers ----

@@ -51,13 +51,14 @@ enum normpre_variant {
                       i.e. Newton-Schulz applied to the momentum itself, with no orientation,
                       tangent or normalization step, and the same RMS-matched update; it
                       shares the Newton-Schulz kernels and serves the latency comparison */
-  NORMPRE_L_EXACT = 3 /* localized with exact eigenspace extraction (Sec. 3.2, App. B): the
-                      interaction matrix Gamma = Psi_a Psi_a^T (m_a x m_a) formed on the GPU, its
-                      full symmetric eigendecomposition, the up to r largest eigenvalues above
-                      one.  Costs O(m_a^2 n_a + m_a^3) per matrix: the reference for the sketch
-                      and the source of the spectral diagnostics, not a fast path.  The dense
-                      eigensolver is cuSOLVER's syevd, loaded at run time (NORMPRE_ERR_UNAVAILABLE
-                      when it cannot be loaded) */
+  NORMPRE_L_EXACT = 3 /* localized with exact eigenspace extraction (Sec. 3.2, App. B): the full
+                      symmetric eigendecomposition of the interaction matrix Gamma = Psi_a Psi_a^T
+                      (m_a x m_a), the up to r largest eigenvalues above one.  Computed without
+                      forming Gamma, by a one-sided block Jacobi SVD of Psi (this library's
+                      kernels; Gamma's eigenvalues are Psi's squared singular values).  Costs
+                      O(sweeps min(m,n)^2 max(m,n)) per matrix: the reference for the sketch and
+                      the source of the spectral diagnostics, not a fast path.  The statistics'
+                      last slot holds the Jacobi sweeps that still rotated */
 };
 
 /* Storage dtypes of caller tensors. */
@@ -77,7 +78,7 @@ enum normpre_status {
   NORMPRE_ERR_NONFINITE = 6,  /* NaN or Inf met in the momentum or weights (device flag) */
   NORMPRE_ERR_NUMERIC = 7,    /* CholeskyQR breakdown or Jacobi sweep cap reached (device flag) */
   NORMPRE_ERR_TIMEOUT = 8,    /* a bounded device-side wait gave up (device flag) */
-  NORMPRE_ERR_UNAVAILABLE = 9 /* NORMPRE_L_EXACT: the cuSOLVER library could not be loaded */
+  NORMPRE_ERR_UNAVAILABLE = 9 /* reserved: no call returns it (NORMPRE_L_EXACT needs no library) */
 };
 
 /* Which precision the spectral stage computes in. */
@@ -191,7 +192,8 @@ enum normpre_buffer {
   NORMPRE_BUF_Z = 4,      /* NormPre-L: Ritz vectors Z (l x l, column j = j-th Ritz value), fp32 */
   NORMPRE_BUF_OMEGA = 5,  /* NormPre-L: sketch matrix Omega of the last step, n_a x l, fp32 */
   NORMPRE_BUF_STATS = 6,  /* 1 x 8 fp32: [k, m', ||T||_F^2, |C|, l, n_a, m_a, s] of the last step,
-                             s = Jacobi sweeps of NormPre-L (0 for NORMPRE_L_EXACT) */
+                             s = Jacobi sweeps of the Ritz problem (NormPre-L) or outer Jacobi
+                             sweeps that rotated a column pair (NORMPRE_L_EXACT) */
   NORMPRE_BUF_EIGS = 7,   /* NORMPRE_L_EXACT: all m_a eigenvalues of Gamma, descending (1 x m_a) */
   NORMPRE_BUF_DIAG = 8    /* 1 x 8 fp32 diagnostics of the last step: [E_top, E_remain, E_sub,
                              E_global, cos(G, Phi), ||G||_F, ||T||_F, <G, T>].  The spectral
@@ -279,8 +281,9 @@ enum normpre_profile_class {
   NORMPRE_PROF_EIG = 8,        /* Rayleigh-Ritz Gram, Jacobi eigensolver, Q K */
   NORMPRE_PROF_APPLY_L = 9,    /* NormPre-L projector apply + weight update */
   NORMPRE_PROF_PRESCALE = 10,  /* Newton-Schulz input scale 1/(sqrt(m') + eps) */
-  NORMPRE_PROF_GAMMA = 11,     /* NORMPRE_L_EXACT: Gamma = Psi_a Psi_a^T */
-  NORMPRE_PROF_SYEVD = 12,     /* NORMPRE_L_EXACT: dense eigensolver and the selection */
+  NORMPRE_PROF_EXACT_SWEEPS = 11,  /* NORMPRE_L_EXACT: the one-sided block Jacobi sweeps over Psi */
+  NORMPRE_PROF_EXACT_SELECT = 12,  /* NORMPRE_L_EXACT: eigenvalues, their order, the selection and the
+                                      eigenvectors */
   NORMPRE_PROF_CLASSES = 13
 };
 

@@ -72,6 +72,12 @@ __device__ __forceinline__ double warp_sum(double v) {
   return v;
 }
 
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
 // Sum over the whole block; every thread gets the result.  `red` must hold
 // blockDim.x / 32 entries.  Deterministic (fixed tree order).
 template <typename T>

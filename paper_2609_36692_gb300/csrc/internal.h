@@ -24,7 +24,7 @@ inline int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 enum ProfClass {
   kProfNormalize = 0, kProfNsGram = 1, kProfNsPoly = 2, kProfNsUpdate = 3, kProfApplyG = 4,
   kProfOmega = 5, kProfContract = 6, kProfQR = 7, kProfEig = 8, kProfApplyL = 9,
-  kProfPrescale = 10, kProfGamma = 11, kProfSyevd = 12, kProfClasses = 13
+  kProfPrescale = 10, kProfExactSweeps = 11, kProfExactSelect = 12, kProfClasses = 13
 };
 
 // Counts kernel launches and, when enabled, brackets launch groups with CUDA
@@ -246,16 +246,17 @@ struct SketchGroup {
   float* rfac = nullptr;        // CholeskyQR factor of one pass, per matrix
   int lmax = 0;
   int max_part = 0;
-  // NORMPRE_L_EXACT: Gamma of one matrix (then its eigenvectors), its
-  // eigenvalues, all eigenvalues of every matrix (descending), the eigensolver
-  // workspace and status, and the cuSOLVER handle
-  float* gamma = nullptr;
-  float* eig_w = nullptr;
+  // NORMPRE_L_EXACT (exact.cu): the one-sided block Jacobi work matrix Z
+  // [batch][oj_s_pad][oj_lp] (columns contiguous), its column norms, the
+  // per-sweep rotation flags, the selected columns and eigenvalues, and all
+  // eigenvalues of every matrix (descending)
+  float* oj_z = nullptr;
+  float* oj_lam = nullptr;      // [batch][oj_s_pad]
+  int* oj_flag = nullptr;       // [(sweeps + 1) per matrix]
+  int* oj_sel = nullptr;        // [batch][lmax]
+  float* oj_sel_lam = nullptr;  // [batch][lmax]
+  int64_t oj_s_pad = 0, oj_lp = 0;
   float* eig_all = nullptr;     // [batch][max(rows, cols)]
-  float* eig_work = nullptr;
-  int* eig_info = nullptr;
-  int eig_lwork = 0;
-  void* solver = nullptr;
   // tensor-core contractions: TMA maps of Psi as the K-major (box 32 x 128)
   // and MN-major (box 32 x 32) A operand; tc = false keeps the SIMT kernel
   CUtensorMap psi_map_k, psi_map_mn;
@@ -277,15 +278,14 @@ struct SketchParams {
 };
 
 cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::vector<void*>& allocs);
-// NORMPRE_L_EXACT (exact.cu): whether cuSOLVER could be loaded; the Gamma and
-// eigensolver workspaces of a group (one matrix at a time); the solver handle's
-// release; and the exact eigenpairs of every matrix of g into q, ritz, zvec,
-// kmat, stats (and the spectral energies into diag).
-int exact_available(std::string* why);
-cudaError_t exact_group_alloc(SketchGroup& g, std::vector<void*>& allocs, std::string* why);
-void exact_group_free(SketchGroup& g);
-cudaError_t exact_eigs(SketchGroup& g, const SketchParams& p, int l, const int* mat_ids_host, const int* count,
-                       double* diag, int* flags, cudaStream_t s, ProfileHook* prof);
+// NORMPRE_L_EXACT (exact.cu): the eigensolver workspaces of a group; and the
+// exact eigenpairs of every matrix of g into ritz, zvec, kmat, stats, the
+// spectral energies (diag) and either q (the eigenvectors) or, when
+// *needs_projection is set, the panel y0 whose product Psi_a y0 is q.
+cudaError_t exact_group_alloc(SketchGroup& g, std::vector<void*>& allocs);
+constexpr int kExactFlagRows = 25;   // per-matrix share of oj_flag (one entry per sweep, and one more)
+cudaError_t exact_eigs(SketchGroup& g, const SketchParams& p, int l, const int* mat_ids, const int* count,
+                       double* diag, int* flags, cudaStream_t s, ProfileHook* prof, bool* needs_projection);
 // Matrices [b0, b1) of a group as a group of their own: the same workspaces
 // from its first matrix on, and tensor maps of Psi over those matrices only.
 cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup* out);

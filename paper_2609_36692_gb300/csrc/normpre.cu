@@ -109,7 +109,7 @@ struct StepHooks {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 // Newton-Schulz preconditioning (NormPre-G, Muon) or the localized one (L, L exact)
 bool uses_ns(int variant) { return variant == NORMPRE_G || variant == NORMPRE_MUON; }
-constexpr int64_t kExactMaxDim = 16384;   // Gamma of one matrix is the L-exact workspace
+constexpr int64_t kExactMaxDim = 16384;   // the L-exact selection sorts up to this many eigenvalues in one CTA
 
 int check_config(const normpre_config* c, std::string* msg) {
   if (c->variant != NORMPRE_G && c->variant != NORMPRE_L && c->variant != NORMPRE_MUON &&
@@ -191,7 +191,6 @@ void normpre_free(normpre_handle* h) {
   cudaSetDevice(h->device);
   cudaDeviceSynchronize();
   h->ns.reset();
-  for (Group& g : h->groups) exact_group_free(g.sk);
   for (cudaStream_t st : h->side) cudaStreamDestroy(st);
   for (cudaEvent_t ev : h->side_done) cudaEventDestroy(ev);
   for (cudaEvent_t ev : h->side_fork) cudaEventDestroy(ev);
@@ -288,14 +287,7 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
       e = sketch_group_alloc(g.sk, cfg->rank, exact ? 0 : cfg->oversample, h->allocs);
       if (e != cudaSuccess) return cuda_fail(nullptr, e, "sketch workspace");
       if (exact) {
-        std::string why;
-        e = exact_group_alloc(g.sk, h->allocs, &why);
-        if (e == cudaErrorNotSupported) {
-          for (Group& gg : h->groups) exact_group_free(gg.sk);
-          for (void* p : h->allocs) cudaFree(p);
-          h->allocs.clear();
-          return fail(nullptr, NORMPRE_ERR_UNAVAILABLE, "NORMPRE_L_EXACT: " + why);
-        }
+        e = exact_group_alloc(g.sk, h->allocs);
         if (e != cudaSuccess) return cuda_fail(nullptr, e, "exact eigensolver workspace");
       }
     }

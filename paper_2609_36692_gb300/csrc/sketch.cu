@@ -1731,6 +1731,13 @@ cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup
   s.stats = g.stats + static_cast<int64_t>(b0) * 8;
   s.rfac = g.rfac + static_cast<int64_t>(b0) * kRfacStride;
   if (g.eig_all) s.eig_all = g.eig_all + b0 * std::max(g.rows, g.cols);
+  if (g.oj_z) {
+    s.oj_z = g.oj_z + b0 * g.oj_s_pad * g.oj_lp;
+    s.oj_lam = g.oj_lam + b0 * g.oj_s_pad;
+    s.oj_flag = g.oj_flag + b0 * static_cast<int64_t>(kExactFlagRows);
+    s.oj_sel = g.oj_sel + static_cast<int64_t>(b0) * g.lmax;
+    s.oj_sel_lam = g.oj_sel_lam + static_cast<int64_t>(b0) * g.lmax;
+  }
   if (g.tc) {
     const uint64_t dims[3] = {static_cast<uint64_t>(g.cols), static_cast<uint64_t>(g.rows),
                               static_cast<uint64_t>(s.batch)};
@@ -1862,8 +1869,11 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     return GramOut{g.gram, sq, 1};
   };
   if (p.exact) {
-    // exact eigenpairs of Gamma = Psi_a Psi_a^T (exact.cu), then B^T = Psi_a^T Q
-    if ((e = exact_eigs(g, p, l, p.mat_ids_host, count, p.diag, flags, s, prof))) return e;
+    // exact eigenpairs of Gamma = Psi_a Psi_a^T (exact.cu): Q directly, or
+    // Q = Psi_a P from the panel P it leaves in y0; then B^T = Psi_a^T Q
+    bool project = false;
+    if ((e = exact_eigs(g, p, l, mat_ids, count, p.diag, flags, s, prof, &project))) return e;
+    if (project && (e = contract(ta, g.y0, g.q))) return e;
     if ((e = contract(tb, g.q, g.bt))) return e;
     prof->begin(kProfEig, s);   // Q K below
   } else {

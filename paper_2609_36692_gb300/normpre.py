@@ -183,7 +183,7 @@ def normpre_newton_schulz(cfg: normpre_config, batch: int, rows: int, cols: int,
 
 
 PROFILE_CLASSES = ["normalize", "ns_gram", "ns_poly", "ns_update", "apply_g", "omega", "contract",
-                   "qr", "eig", "apply_l", "prescale", "gamma", "syevd"]
+                   "qr", "eig", "apply_l", "prescale", "exact_sweeps", "exact_select"]
 
 
 def normpre_profile(handle: int, enable: bool) -> int:
