@@ -117,6 +117,11 @@ typedef struct normpre_config {
   int jacobi_max_sweeps;  /* NormPre-L: cap on the Jacobi sweeps of the l x l Ritz problem
                              (Alg. 2, eig of Gamma_Q); 0 = default 30, else in [1, 1000].  A step
                              that reaches the cap before converging reports NORMPRE_ERR_NUMERIC */
+  int test_stall;         /* tests only, 0 otherwise.  1: in a NormPre-L step, one CTA of the first
+                             sketch contraction does not issue its first copy, so its bounded waits
+                             give up after about two seconds and the step reports
+                             NORMPRE_ERR_TIMEOUT (that step's results are not meaningful; the
+                             context stays usable).  It exercises the device-side timeout path */
 } normpre_config;
 
 /* Fills `cfg` with the paper's defaults (NormPre-G, bf16 Newton-Schulz). */
@@ -175,8 +180,9 @@ int normpre_step_host(normpre_handle* h, int64_t t, float lr, void* const* W_hos
 
 /*
  * Synchronizes `stream`, then reports and clears the device-side flags set
- * since the last call: NONFINITE, NUMERIC or TIMEOUT (the first one found, in
- * that order), else OK.
+ * since the last call: TIMEOUT, NONFINITE or NUMERIC (the first one found, in
+ * that order: a wait that gave up leaves the rest of the step without
+ * meaning), else OK.
  */
 int normpre_sync_status(normpre_handle* h, void* stream);
 

@@ -266,6 +266,7 @@ struct SketchGroup {
 struct SketchParams {
   int rank = 32, oversample = 8, power_iters = 1;
   int max_sweeps = 30;          // Jacobi sweep cap of the Ritz problem
+  int test_stall = 0;           // tests: one CTA of the first contraction skips its first copy
   uint64_t seed = 0;
   int64_t t = 0;
   int k = 0;                    // orientation of this step

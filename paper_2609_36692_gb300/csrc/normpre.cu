@@ -117,6 +117,7 @@ int check_config(const normpre_config* c, std::string* msg) {
     *msg = "variant must be NORMPRE_G, NORMPRE_L, NORMPRE_MUON or NORMPRE_L_EXACT"; return NORMPRE_ERR_ARG;
   }
   if (c->diagnostics != 0 && c->diagnostics != 1) { *msg = "diagnostics must be 0 or 1"; return NORMPRE_ERR_ARG; }
+  if (c->test_stall != 0 && c->test_stall != 1) { *msg = "test_stall must be 0 or 1"; return NORMPRE_ERR_ARG; }
   if (!std::isfinite(c->momentum) || !std::isfinite(c->weight_decay) || !std::isfinite(c->target_rms)) {
     *msg = "momentum, weight_decay and target_rms must be finite"; return NORMPRE_ERR_ARG;
   }
@@ -506,6 +507,7 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
     p.rank = c.rank; p.oversample = c.oversample; p.power_iters = c.power_iters;
     p.seed = c.seed; p.t = t; p.k = k;
     p.max_sweeps = c.jacobi_max_sweeps > 0 ? c.jacobi_max_sweeps : 30;
+    p.test_stall = c.test_stall;
     p.lr = lr; p.wd = c.weight_decay; p.target = c.target_rms;
     for (int ui = 0; ui < nu; ++ui) {
       if ((rc = normalize(ui))) return rc;
@@ -582,9 +584,10 @@ int normpre_sync_status(normpre_handle* h, void* stream) {
     e = cudaMemset(h->flags, 0, sizeof(int));
     if (e) return cuda_fail(h, e, "cudaMemset");
   }
+  // a wait that gave up leaves the rest of the step without meaning: first
+  if (flags & kFlagTimeout) return fail(h, NORMPRE_ERR_TIMEOUT, "a bounded device wait gave up");
   if (flags & kFlagNonfinite) return fail(h, NORMPRE_ERR_NONFINITE, "non-finite value in the momentum or the weights");
   if (flags & kFlagNumeric) return fail(h, NORMPRE_ERR_NUMERIC, "CholeskyQR breakdown or Jacobi sweep cap reached");
-  if (flags & kFlagTimeout) return fail(h, NORMPRE_ERR_TIMEOUT, "a bounded device wait gave up");
   return NORMPRE_OK;
 }
 

@@ -341,6 +341,7 @@ struct ContractTcArgs {
   int64_t kchunk;         // K range of one split (multiple of 32)
   int ksplit, batch;      // K splits and matrices (the units are tiles x ksplit x batch)
   int* flags;
+  int stall_first_copy;   // tests: CTA 0 does not issue its first copy (its waits then give up)
 };
 // Two rings.  The input ring holds the TMA copies of the Psi block and of the
 // V block; the split warps free a slot as soon as they have read it, so the
@@ -512,7 +513,7 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
         const uint32_t ph = (it / kCtcIn) & 1;
         ok = __all_sync(0xffffffffu, tc::mbar_wait(&inempty[i], ph ^ 1u, abort_flag));
         if (!ok) break;
-        if (lane == 0) {
+        if (lane == 0 && !(a.stall_first_copy && blockIdx.x == 0 && it == 0)) {
           tc::mbar_expect_tx(&full[i], static_cast<uint32_t>(kCtcA + nvb * 4096));
           issued[i] = ph + 1;
           const int k0 = static_cast<int>(kbeg) + 32 * kb, pr = static_cast<int>(p0);
@@ -1786,6 +1787,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   // the tensor-core form needs 16-byte rows of the l-wide operand and 16-byte
   // aligned per-matrix strides (TMA)
   const bool use_tc = g.tc && (l % 4 == 0) && (vbs % 4 == 0) && l <= 64;
+  bool stall_pending = p.test_stall != 0;   // the first tensor-core contraction of the step
   auto contract = [&](bool trans, const float* v, float* out) -> cudaError_t {
     prof->begin(kProfContract, s);
     const int64_t P = trans ? g.cols : g.rows, K = trans ? g.rows : g.cols;
@@ -1822,6 +1824,8 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       ct.kchunk = c.kchunk;
       ct.flags = flags;
       ct.ksplit = ks; ct.batch = B;
+      ct.stall_first_copy = stall_pending ? 1 : 0;
+      stall_pending = false;
       // persistent: one CTA per SM (shared memory and TMEM admit one)
       const int64_t units = cdiv(P, 128) * ks * B;
       const unsigned grid = static_cast<unsigned>(std::min<int64_t>(units, device_sm_count()));

@@ -47,6 +47,7 @@ class normpre_config(ctypes.Structure):
         ("tangent", ctypes.c_int),
         ("diagnostics", ctypes.c_int),
         ("jacobi_max_sweeps", ctypes.c_int),
+        ("test_stall", ctypes.c_int),
     ]
 
 

@@ -93,6 +93,11 @@ def test_host_side_argument_errors(lib):
             C.normpre_init(bad, [(4, 5)], [0], [0])
         assert e.value.status == C.NORMPRE_ERR_ARG and "jacobi_max_sweeps" in C.normpre_last_error()
     assert C.normpre_default_config().jacobi_max_sweeps == 0
+    bad = C.normpre_default_config(test_stall=2)
+    with pytest.raises(C.NormPreError) as e:
+        C.normpre_init(bad, [(4, 5)], [0], [0])
+    assert e.value.status == C.NORMPRE_ERR_ARG and "test_stall" in C.normpre_last_error()
+    assert C.normpre_default_config().test_stall == 0
     # exact eigenspace extraction: rank budget and the Gamma workspace limit
     bad = C.normpre_default_config(variant=C.NORMPRE_L_EXACT, rank=73)
     with pytest.raises(C.NormPreError) as e:

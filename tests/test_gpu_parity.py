@@ -692,6 +692,36 @@ def test_jacobi_sweep_cap_reports_numeric():
     opt.close()
 
 
+def test_bounded_wait_timeout_reports_and_recovers():
+    """The device-side timeout path of the tensor-core kernels: with test_stall,
+    one CTA of each group's first sketch contraction never gets its first copy;
+    its split warps give up after the bounded wait (about two seconds) and set
+    the CTA's abort flag, every other role of that CTA leaves its loop at its
+    next wait, thread 0 waits for the copies the CTA did issue, the tensor
+    memory is freed and the kernel exits; the step reports
+    NORMPRE_ERR_TIMEOUT.  No trap and no hang: the context stays usable, and a
+    following step on a new handle matches the oracle."""
+    import time
+
+    import torch
+    from paper_2609_36692_gb300 import normpre as C
+    cs = SMALL
+    mats = S.make_param_set(cs)
+    W, G, M = to_device(mats, cs.g_dtype, cs.w_dtype)
+    shapes = [(m.rows, m.cols) for m in cs.matrices]
+    opt = _normpre(shapes, [cs.w_dtype] * cs.n_mats, [cs.g_dtype] * cs.n_mats, variant=C.NORMPRE_L,
+                   precision=1, rank=cs.rank, oversample=cs.oversample, seed=1234, test_stall=1)
+    t0 = time.perf_counter()
+    opt.step(0, LR, W, G, M)
+    torch.cuda.synchronize()
+    waited = time.perf_counter() - t0
+    assert opt.status(raise_on_error=False) == C.NORMPRE_ERR_TIMEOUT
+    assert "gave up" in C.normpre_last_error(opt.handle)
+    assert 1.0 < waited < 60.0, waited
+    opt.close()
+    _check_l(cs, 1)
+
+
 # one GPT-2 Small attention qkv matrix (768 x 2304): Gamma is 768 x 768 at
 # t = 0 and 2304 x 2304 at t = 1
 GPT2_QKV = S.custom_config("gpt2_qkv", [(768, 2304)], g_dtype="bf16", w_dtype="f32",
