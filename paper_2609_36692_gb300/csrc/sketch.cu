@@ -872,6 +872,7 @@ struct CholQRArgs {
   int vec;       // l % 4 == 0 and 16-byte aligned rows: float4 row loads / stores
   int drop;      // 0: shifted retry on a small pivot (first pass); 1: drop its column
   int* flags;
+  float* gram_out; int64_t gram_bs;   // optional: per solve CTA, the l x l Gram sum of its rows
 };
 // Per matrix [R (LP x LP, strictly upper, rows scaled by 1 / R_ii) | 1 / R_ii
 // (LP) | zero-panel flag]: the factorization of one CholeskyQR pass, made
@@ -1000,6 +1001,127 @@ __global__ void __launch_bounds__(256) k_chol_solve(const __grid_constant__ Chol
 #pragma unroll
     for (int j = 0; j < LP; ++j)
       if (j < l) q[j] = x[j];
+  }
+}
+
+// The solve of a pass whose result feeds another pass also sums the Gram
+// matrix of its 256 rows (the next factorization folds one partial per solve
+// CTA): the rows go through shared memory, 4 x 4 blocks of the l x l sum in
+// registers per thread, rows split into groups when the blocks do not fill
+// the CTA (summed in a fixed order).
+template <int LP>
+__global__ void __launch_bounds__(256) k_chol_solve_gram(const __grid_constant__ CholQRArgs a, const float* rfac) {
+  extern __shared__ float4 sg_smem4[];
+  float* X = reinterpret_cast<float*>(sg_smem4);          // [256][LP + 4]
+  constexpr int LDX = LP + 4;
+  __shared__ __align__(16) float GR[LP * LP];
+  __shared__ float rinv[LP];
+  const int b = blockIdx.y, l = a.l, tid = threadIdx.x;
+  const float* in = rfac + static_cast<int64_t>(b) * kRfacStride;
+  const bool zero = in[LP * LP + LP] != 0.f;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * 256 + tid;
+  const float* y = a.y + b * a.v_bs + row * l;
+  float* q = a.q + b * a.v_bs + row * l;
+  float x[LP];
+#pragma unroll
+  for (int j = 0; j < LP; ++j) x[j] = 0.f;
+  if (!zero) {
+    for (int e = tid; e < LP * LP / 4; e += 256)
+      reinterpret_cast<float4*>(GR)[e] = __ldg(reinterpret_cast<const float4*>(in) + e);
+    for (int i = tid; i < LP; i += 256) rinv[i] = in[LP * LP + i];
+  }
+  __syncthreads();
+  if (row < a.n && !zero) {
+    if (a.vec) {
+#pragma unroll
+      for (int j = 0; j < LP; j += 4) {
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (j < l) v = *reinterpret_cast<const float4*>(y + j);
+        x[j] = v.x; x[j + 1] = v.y; x[j + 2] = v.z; x[j + 3] = v.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < LP; ++j) x[j] = (j < l) ? y[j] : 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < LP; ++k) {
+      x[k] *= rinv[k];
+#pragma unroll
+      for (int j4 = ((k + 1) / 4) * 4; j4 < LP; j4 += 4) {
+        const float4 r = *reinterpret_cast<const float4*>(&GR[k * LP + j4]);
+        if (j4 + 0 > k) x[j4 + 0] = fmaf(-x[k], r.x, x[j4 + 0]);
+        if (j4 + 1 > k) x[j4 + 1] = fmaf(-x[k], r.y, x[j4 + 1]);
+        if (j4 + 2 > k) x[j4 + 2] = fmaf(-x[k], r.z, x[j4 + 2]);
+        if (j4 + 3 > k) x[j4 + 3] = fmaf(-x[k], r.w, x[j4 + 3]);
+      }
+    }
+  }
+  if (row < a.n) {
+    if (a.vec) {
+#pragma unroll
+      for (int j = 0; j < LP; j += 4)
+        if (j < l) *reinterpret_cast<float4*>(q + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < LP; ++j)
+        if (j < l) q[j] = x[j];
+    }
+  }
+  // rows past n and columns past l are zero
+#pragma unroll
+  for (int j = 0; j < LP; j += 4)
+    *reinterpret_cast<float4*>(X + tid * LDX + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
+  __syncthreads();
+  constexpr int L4 = LP / 4, TILES = L4 * L4;
+  constexpr int GROUPS = TILES <= 64 ? 4 : (TILES <= 128 ? 2 : 1);
+  constexpr int ROWS_G = 256 / GROUPS;
+  float* out = a.gram_out + b * a.gram_bs + static_cast<int64_t>(blockIdx.x) * l * l;
+  float acc[4][4];
+  int my_tile = -1, my_group = 0;
+  for (int t = tid; t < TILES * GROUPS; t += 256) {
+    const int tile = t % TILES, g = t / TILES;
+    const int p0 = 4 * (tile / L4), q0 = 4 * (tile % L4);
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+    const float* xb = X + g * ROWS_G * LDX;
+#pragma unroll 4
+    for (int i = 0; i < ROWS_G; ++i) {
+      const float4 pv = *reinterpret_cast<const float4*>(xb + i * LDX + p0);
+      const float4 qv = *reinterpret_cast<const float4*>(xb + i * LDX + q0);
+      const float pa[4] = {pv.x, pv.y, pv.z, pv.w}, qa[4] = {qv.x, qv.y, qv.z, qv.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(pa[r], qa[c], acc[r][c]);
+    }
+    if (GROUPS == 1) {
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          if (p0 + r < l && q0 + c < l) out[(p0 + r) * l + q0 + c] = acc[r][c];
+    } else {
+      my_tile = tile;
+      my_group = g;
+    }
+  }
+  if (GROUPS == 1) return;
+  __syncthreads();                                // X is read: reuse it for the group sums
+  if (my_tile >= 0) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) X[(my_group * TILES + my_tile) * 16 + 4 * r + c] = acc[r][c];
+  }
+  __syncthreads();
+  for (int e = tid; e < l * l; e += 256) {
+    const int p = e / l, qq = e - p * l;
+    const int tile = (p >> 2) * L4 + (qq >> 2), k = 4 * (p & 3) + (qq & 3);
+    float v = 0.f;
+    for (int g = 0; g < GROUPS; ++g) v += X[(g * TILES + tile) * 16 + k];
+    out[e] = v;
   }
 }
 
@@ -1656,7 +1778,22 @@ static void contract_attrs() {
 static cudaError_t launch_cholqr(const CholQRArgs& c, float* rfac, int batch, int lp, cudaStream_t s) {
   const dim3 grid(static_cast<unsigned>(cdiv(c.n, 256)), static_cast<unsigned>(batch));
   switch (lp) {
-#define NP_CQ(N) case N: k_chol_factor<N><<<batch, 256, 0, s>>>(c, rfac); k_chol_solve<N><<<grid, 256, 0, s>>>(c, rfac); break;
+#define NP_CQ(N)                                                                                        \
+  case N:                                                                                               \
+    k_chol_factor<N><<<batch, 256, 0, s>>>(c, rfac);                                                    \
+    if (c.gram_out) {                                                                                   \
+      const size_t sm = sizeof(float) * 256 * (N + 4);                                                  \
+      static bool attr = false;                                                                         \
+      if (!attr) {                                                                                      \
+        cudaFuncSetAttribute(k_chol_solve_gram<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,         \
+                             static_cast<int>(sm));                                                     \
+        attr = true;                                                                                    \
+      }                                                                                                 \
+      k_chol_solve_gram<N><<<grid, 256, sm, s>>>(c, rfac);                                              \
+    } else {                                                                                            \
+      k_chol_solve<N><<<grid, 256, 0, s>>>(c, rfac);                                                    \
+    }                                                                                                   \
+    break;
     NP_FOR_LP(NP_CQ)
 #undef NP_CQ
     default:
@@ -1895,12 +2032,23 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     prof->begin(kProfQR, s);
     {
       const float* src = ycur;
+      // the first pass's Gram partials by k_gram_part (128-row chunks); the
+      // next passes' from the previous solve (256-row chunks); each factor
+      // folds its partials itself
+      GramArgs ga;
+      ga.y = src; ga.y_bs = vbs; ga.part = g.part;
+      ga.part_bs = static_cast<int64_t>(g.max_part) * sq;
+      ga.n = m_a; ga.l = l;
+      ga.nsplit = static_cast<int>(cdiv(m_a, kGramRows));
+      k_gram_part<<<dim3(ga.nsplit, B), 256, 0, s>>>(ga);
+      NP_CHECK();
+      int nsplit = ga.nsplit;
       for (int pass = 0; pass < 3; ++pass) {
-        const GramOut go = gram(src, m_a);
-        NP_CHECK();
         float* dst = (pass == 1) ? g.zt : g.q;
         CholQRArgs cq;
-        cq.part = go.p; cq.part_bs = go.bs; cq.nsplit = go.n;
+        cq.part = g.part; cq.part_bs = ga.part_bs; cq.nsplit = nsplit;
+        cq.gram_out = pass < 2 ? g.part : nullptr;
+        cq.gram_bs = ga.part_bs;
         cq.y = src; cq.q = dst; cq.v_bs = vbs;
         cq.n = m_a; cq.l = l; cq.flags = flags;
         cq.vec = (l % 4 == 0) && (vbs % 4 == 0) && (reinterpret_cast<uintptr_t>(src) % 16 == 0) &&
@@ -1908,9 +2056,10 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
         cq.drop = (pass > 0);
         if ((e = launch_cholqr(cq, g.rfac, B, lp, s))) return e;
         src = dst;
+        nsplit = static_cast<int>(cdiv(m_a, 256));
       }
     }
-    prof->end(kProfQR, s, 9 + n_fold);
+    prof->end(kProfQR, s, 7);
     n_fold = 0;
     // B^T = Psi_a^T Q  [n_a x l];  Gamma_Q = B B^T
     if ((e = contract(tb, g.q, g.bt))) return e;
