@@ -14,18 +14,23 @@ namespace normpre {
 template <typename TW, typename TT, bool VEC>
 __global__ void __launch_bounds__(256) k_apply_g(const __grid_constant__ ApplyLaunch a) {
   __shared__ double red[32];
+  __shared__ float scale_s;
   const int b = blockIdx.y;
   double s = 0;
   for (int i = threadIdx.x; i < a.n_part; i += blockDim.x) s += a.sq_part[b][i];
   s = block_sum(s, red);
-  const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
-  const float scale = s > 0 ? static_cast<float>(a.target * sqrt(mn / s)) : 0.f;
-  if (blockIdx.x == 0 && threadIdx.x == 0 && a.stats[b]) {
-    a.stats[b][0] = static_cast<float>(a.k);
-    a.stats[b][1] = a.count ? static_cast<float>(a.count[a.mat_id[b]]) : 0.f;
-    a.stats[b][2] = static_cast<float>(s);
+  if (threadIdx.x == 0) {
+    // formed by one thread: fp64 throughput is low on this part
+    const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
+    scale_s = s > 0 ? static_cast<float>(a.target * sqrt(mn / s)) : 0.f;
+    if (blockIdx.x == 0 && a.stats[b]) {
+      a.stats[b][0] = static_cast<float>(a.k);
+      a.stats[b][1] = a.count ? static_cast<float>(a.count[a.mat_id[b]]) : 0.f;
+      a.stats[b][2] = static_cast<float>(s);
+    }
   }
-  const float cw = 1.f - a.lr * a.wd, ct = -a.lr * scale;
+  __syncthreads();
+  const float cw = 1.f - a.lr * a.wd, ct = -a.lr * scale_s;
   TW* W = static_cast<TW*>(a.W[b]);
   const TT* T = static_cast<const TT*>(a.T[b]);
   if (VEC) {

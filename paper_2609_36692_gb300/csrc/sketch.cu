@@ -1439,6 +1439,13 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
       for (int p = half; p < l; p += 2) dst[p][i] = ok ? src[p] : 0.f;
     }
   }
+  // the matrix's scale formed once (fp64 throughput is low on this part)
+  __shared__ float scale_s;
+  if (tid == 0) {
+    const float nrm2 = a.stats[b * a.stats_bs + 2];
+    const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
+    scale_s = nrm2 > 0.f ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
+  }
   __syncthreads();
   float acc[4][4] = {};
 #pragma unroll 4
@@ -1451,11 +1458,7 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
 #pragma unroll
       for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(la[r], ra[c], acc[r][c]);
   }
-  const float* st = a.stats + b * a.stats_bs;
-  const float nrm2 = st[2];
-  const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
-  const float scale = nrm2 > 0.f ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
-  const float cw = 1.f - a.lr * a.wd, ct = -a.lr * scale;
+  const float cw = 1.f - a.lr * a.wd, ct = -a.lr * scale_s;
   const float* psi = a.psi + b * a.psi_bs;
   TW* W = static_cast<TW*>(a.W[b]);
   const int64_t j0 = c0 + tx * 4;
@@ -1531,6 +1534,7 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
 constexpr int kAtcRows = 256;                         // W rows per unit (MMA N)
 constexpr int kAtcCols = 128;                         // W columns per unit (MMA M)
 constexpr int kAtcProd = 2, kAtcEpi = 8;
+constexpr int kAtcChunk = 16, kAtcSlots = 3;       // epilogue: rows per chunk, register ring slots
 constexpr int kAtcThreads = 32 * (kAtcProd + 1 + kAtcEpi);
 constexpr int kAtcAtomA = kAtcCols * 128;             // one 32-wide K atom of the A (Rm) tile
 constexpr int kAtcAtomB = kAtcRows * 128;             // one 32-wide K atom of the B (Lm) tile
@@ -1681,57 +1685,111 @@ __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_consta
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
   } else {
     // ---------------- epilogue: W <- (1 - lr wd) W - lr s (Psi + D) ----------------
+    // A stream of 16-row chunks (8 per unit: W rows 128 h .. 128 h + 127 of
+    // the tile, W columns 32 q + lane): the Psi and W loads of a chunk do not
+    // depend on the accumulator, so they are issued kAtcSlots - 1 chunks ahead
+    // into a register ring and stay in flight while earlier chunks wait for
+    // their MMAs and are combined.
     const int e = warp - kAtcProd - 1;
     const int q = warp & 3;          // TMEM lane quarter = W columns 32 q .. 32 q + 31 of the tile
     const int h = e >> 2;            // W rows 128 h .. 128 h + 127 of the tile
     const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
     const float cw = 1.f - a.lr * a.wd;
-    bool ok = true;
-    uint32_t it = 0;
-    for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
-      const int acc = it & 1;
-      int b;
-      int64_t i0, j0;
-      unit_of(u, b, i0, j0);
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&tfull[acc], (it >> 1) & 1, abort_flag));
-      if (!ok) break;
-      tc::fence_after();
-      const float nrm2 = a.stats[b * a.stats_bs + 2];
-      const float scale = nrm2 > 0.f ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
-      const float ctt = -a.lr * scale;
-      const int64_t j = j0 + 32 * q + lane;
-      const bool jok = j < a.cols;
-      const float* psi = a.psi + b * a.psi_bs + j;
-      TW* W = static_cast<TW*>(a.W[b]) + j;
-#pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
-        const int64_t r0 = i0 + 128 * h + 32 * c;
-        uint32_t v[32];
-        tc::tmem_ld32(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(256 * acc + 128 * h + 32 * c), v);
-        tc::tmem_ld_wait();
-        const int nr = (r0 < a.rows && jok) ? static_cast<int>(a.rows - r0 < 32 ? a.rows - r0 : 32) : 0;
-        if (nr == 32) {
-          float pv[32], wv[32];
-#pragma unroll
-          for (int rr = 0; rr < 32; ++rr) {
-            pv[rr] = __ldcs(psi + (r0 + rr) * a.psi_ld);
-            wv[rr] = to_f32(W[(r0 + rr) * a.cols]);
+    constexpr int CH = kAtcChunk, NCH = 128 / kAtcChunk, S = kAtcSlots;
+    const int64_t nck = (u1 - u0) * NCH;
+    // issue cursor: the unit (matrix b, row tile i0, column tile j0) and chunk
+    int ib;
+    int64_t ii0, ij0;
+    unit_of(u0, ib, ii0, ij0);
+    int icc = 0;
+    int cur_b = -1;
+    float cur_ct = 0.f;
+    float pv[S][CH];
+    TW wv[S][CH];
+    TW* wp[S];
+    int nr[S];
+    float ctt[S];
+    auto issue = [&](int64_t k, float* P, TW* Wv, TW*& wptr, int& nrows, float& ct) {
+      if (k < nck) {
+        const int64_t j = ij0 + 32 * q + lane;
+        const int64_t r0 = ii0 + 128 * h + CH * icc;
+        if (ib != cur_b) {
+          // fp64 throughput is low on this part: one lane per warp forms the
+          // scale of a new matrix and broadcasts it
+          float scale = 0.f;
+          if (lane == 0) {
+            const float nrm2 = a.stats[ib * a.stats_bs + 2];
+            scale = nrm2 > 0.f ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
           }
+          cur_ct = -a.lr * __shfl_sync(0xffffffffu, scale, 0);
+          cur_b = ib;
+        }
+        ct = cur_ct;
+        const float* pptr = a.psi + ib * a.psi_bs + r0 * a.psi_ld + j;
+        wptr = static_cast<TW*>(a.W[ib]) + r0 * a.cols + j;
+        nrows = (r0 < a.rows && j < a.cols) ? static_cast<int>(a.rows - r0 < CH ? a.rows - r0 : CH) : 0;
+        if (nrows == CH) {
 #pragma unroll
-          for (int rr = 0; rr < 32; ++rr)
-            W[(r0 + rr) * a.cols] = from_f32<TW>(fmaf(cw, wv[rr], ctt * (pv[rr] + __uint_as_float(v[rr]))));
+          for (int rr = 0; rr < CH; ++rr) {
+            P[rr] = __ldcs(pptr + rr * a.psi_ld);
+            Wv[rr] = wptr[rr * a.cols];
+          }
         } else {
 #pragma unroll
-          for (int rr = 0; rr < 32; ++rr)
-            if (rr < nr) {
-              const float t = psi[(r0 + rr) * a.psi_ld] + __uint_as_float(v[rr]);
-              W[(r0 + rr) * a.cols] = from_f32<TW>(fmaf(cw, to_f32(W[(r0 + rr) * a.cols]), ctt * t));
-            }
+          for (int rr = 0; rr < CH; ++rr) {
+            P[rr] = rr < nrows ? pptr[rr * a.psi_ld] : 0.f;
+            Wv[rr] = rr < nrows ? wptr[rr * a.cols] : from_f32<TW>(0.f);
+          }
+        }
+        if (++icc == NCH) {
+          icc = 0;
+          ij0 += kAtcCols;
+          if (ij0 >= a.cols) {
+            ij0 = 0;
+            ii0 += kAtcRows;
+            if (ii0 >= a.rows) { ii0 = 0; ++ib; }
+          }
         }
       }
-      tc::fence_before();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+    };
+#pragma unroll
+    for (int sl = 0; sl < S; ++sl) issue(sl, pv[sl], wv[sl], wp[sl], nr[sl], ctt[sl]);
+    bool ok = true;
+    for (int64_t k0 = 0; k0 < nck && ok; k0 += S) {
+#pragma unroll
+      for (int sl = 0; sl < S; ++sl) {
+        const int64_t k = k0 + sl;
+        if (k >= nck) break;
+        const int64_t it = k / NCH;            // unit of this chunk, counted from u0
+        const int c = static_cast<int>(k - it * NCH);
+        const int acc = static_cast<int>(it & 1);
+        if (c == 0) {
+          ok = __all_sync(0xffffffffu, tc::mbar_wait(&tfull[acc], static_cast<uint32_t>((it >> 1) & 1), abort_flag));
+          if (!ok) break;
+          tc::fence_after();
+        }
+        uint32_t v[CH];
+        tmem_ld16(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(256 * acc + 128 * h + CH * c), v);
+        tc::tmem_ld_wait();
+        if (c == NCH - 1) {
+          // the accumulator is read: the MMAs of unit it + 2 may overwrite it
+          tc::fence_before();
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+        }
+        TW* W = wp[sl];
+        if (nr[sl] == CH) {
+#pragma unroll
+          for (int rr = 0; rr < CH; ++rr)
+            W[rr * a.cols] = from_f32<TW>(fmaf(cw, to_f32(wv[sl][rr]), ctt[sl] * (pv[sl][rr] + __uint_as_float(v[rr]))));
+        } else {
+#pragma unroll
+          for (int rr = 0; rr < CH; ++rr)
+            if (rr < nr[sl])
+              W[rr * a.cols] = from_f32<TW>(fmaf(cw, to_f32(wv[sl][rr]), ctt[sl] * (pv[sl][rr] + __uint_as_float(v[rr]))));
+        }
+        issue(k + S, pv[sl], wv[sl], wp[sl], nr[sl], ctt[sl]);
+      }
     }
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
   }
