@@ -47,6 +47,11 @@ Readings taken where the paper is silent:
 * "Row+Column/Step" (Table 5b): rows of the row-active tangent momentum
   normalized, then the columns of the result; preconditioning and the update
   in the row orientation.
+* Pure-bf16 storage (App. A: the Qwen3 runs train in pure BF16): with
+  ``psi_storage="bf16"`` the normalized Psi is rounded to bf16 (round to
+  nearest, ties to even) once, before the spectral stage, and both the
+  spectral stage and the update use the rounded Psi.  The default keeps Psi
+  exact.
 * Muon baseline (the comparison optimizer of Sec. 4 and App. A): the same
   momentum, the Newton-Schulz iteration applied to the momentum itself (no
   orientation, tangent or normalization step, Sec. 2.1), and the update
@@ -82,6 +87,20 @@ class OracleConfig:
     orientation: int = 0            # 0 alternate (paper), 1 row only, 2 column only,
                                     # 3 rows then columns every step (Table 5b "Row+Column/Step")
     tangent: str = "relaxed"        # "relaxed" (paper), "strict" or "none" (Table 5a ablations)
+    psi_storage: str = "exact"      # "exact", or "bf16": Psi rounded to bf16 (pure-bf16 training, App. A)
+
+
+def round_to_bf16(x: np.ndarray) -> np.ndarray:
+    """x rounded to the nearest bf16 value (8 significant bits, the fp32
+    exponent range with its subnormals), ties to even, returned as float64.
+    The spacing of bf16 numbers at |x| in [2^e, 2^(e+1)) is 2^(e-7), and
+    2^-133 below the smallest normal 2^-126; dividing by it is exact, so
+    numpy's half-to-even rounding of the quotient is the rounding itself."""
+    x = np.asarray(x, dtype=np.float64)
+    ax = np.abs(x)
+    e = np.floor(np.log2(np.where(ax > 0, ax, 1.0)))
+    spacing = np.exp2(np.maximum(e, -126.0) - 7.0)
+    return np.where(ax > 0, np.round(x / spacing) * spacing, x)
 
 
 # --------------------------------------------------------------------------
@@ -339,6 +358,10 @@ def normpre_step(W: np.ndarray, G: np.ndarray, M_prev: np.ndarray, t: int, lr: f
         Psi, d = both_axes_normalize(X)
     else:
         Psi, d = diag_gram_normalize(X)
+    if cfg.psi_storage == "bf16":
+        Psi = round_to_bf16(Psi)
+    elif cfg.psi_storage != "exact":
+        raise ValueError(cfg.psi_storage)
     out = {"M": M, "k": k, "X": X, "Psi": Psi, "d": d}
     if cfg.variant == "G":
         T = newton_schulz(Psi, cfg.ns_steps, cfg.ns_coef, cfg.ns_eps)
@@ -410,7 +433,7 @@ def descent_alignment(G: np.ndarray, Phi: np.ndarray) -> float:
 
 
 __all__ = [
-    "MUON_QUINTIC", "OracleConfig", "philox4x32_10", "philox_uniform", "sketch_omega",
+    "MUON_QUINTIC", "OracleConfig", "round_to_bf16", "philox4x32_10", "philox_uniform", "sketch_omega",
     "momentum_update", "orientation_of", "orient", "relaxed_tangent", "strict_tangent", "tangent_step",
     "diag_gram_normalize", "both_axes_normalize",
     "newton_schulz", "interaction_sketch", "exact_interaction_eigs",

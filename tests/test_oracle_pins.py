@@ -615,3 +615,50 @@ def test_orientation_3_step_uses_rows():
         out = O.normpre_step(W, G, M, t, 0.01, O.OracleConfig(variant="G", orientation=3))
         assert out["k"] == 0
         assert np.allclose(np.linalg.norm(out["Psi"], axis=0), 1.0)
+
+
+# ---------------------------------------------------------------------------
+# Pure-bf16 storage of Psi (App. A: the Qwen3 runs train in pure BF16)
+# ---------------------------------------------------------------------------
+def test_round_to_bf16_hand_values():
+    """Round to nearest, ties to even, on 8 significant bits (bf16 spacing
+    2^-7 in [1, 2)), the fp32 exponent range with subnormals of 2^-133."""
+    x = np.array([1.0, 1 + 2.0 ** -8, 1 + 3 * 2.0 ** -8, -(1 + 2.0 ** -8 + 2.0 ** -20), 1 + 2.0 ** -7 - 2.0 ** -30,
+                  0.0, -0.0, 2.0 ** -130, 3 * 2.0 ** -134, 255.5 * 2.0 ** -7, 0.1])
+    want = np.array([1.0, 1.0, 1 + 2.0 ** -6, -(1 + 2.0 ** -7), 1 + 2.0 ** -7,
+                     0.0, -0.0, 2.0 ** -130, 2.0 ** -132, 2.0, 0.10009765625])
+    got = O.round_to_bf16(x)
+    assert np.array_equal(got, want)
+    assert np.signbit(got[6])
+
+
+def test_round_to_bf16_matches_the_library_conversion():
+    """On fp32 inputs the rounding is torch's float32 -> bfloat16 conversion
+    (round to nearest even), ties included."""
+    torch = pytest.importorskip("torch")
+    rng = _rng(77)
+    bits = rng.integers(0, 2 ** 32, size=20000, dtype=np.uint64).astype(np.uint32)
+    bits[:5000] = (bits[:5000] & np.uint32(0xFFFF0000)) | np.uint32(0x8000)   # exact ties
+    bits[5000:6000] &= np.uint32(0x807FFFFF)                                   # subnormals
+    x = bits.view(np.float32)
+    x = x[np.isfinite(x) & (np.abs(x) < 3.0e38)]
+    want = torch.from_numpy(x.copy()).to(torch.bfloat16).to(torch.float64).numpy()
+    assert np.array_equal(O.round_to_bf16(x.astype(np.float64)), want)
+
+
+def test_bf16_psi_storage_step():
+    """With Psi stored in bf16 every Psi entry is a bf16 value within half a
+    bf16 spacing of the exact Psi, and the update keeps its RMS of 0.2."""
+    rng = _rng(31)
+    for variant in ("G", "L"):
+        for t in (0, 1):
+            W = rng.standard_normal((24, 40)) * 0.02
+            G = rng.standard_normal((24, 40))
+            ex = O.normpre_step(W, G, np.zeros_like(W), t, 0.1, O.OracleConfig(variant=variant, rank=4, oversample=4))
+            bf = O.normpre_step(W, G, np.zeros_like(W), t, 0.1,
+                                O.OracleConfig(variant=variant, rank=4, oversample=4, psi_storage="bf16"))
+            assert np.array_equal(O.round_to_bf16(bf["Psi"]), bf["Psi"])
+            half = np.exp2(np.floor(np.log2(np.maximum(np.abs(ex["Psi"]), 2.0 ** -126))) - 8)
+            assert np.all(np.abs(bf["Psi"] - ex["Psi"]) <= half)
+            dW = (W - bf["W"]) / 0.1 - 0.1 * W
+            assert abs(np.sqrt((dW * dW).mean()) - 0.2) < 1e-12
