@@ -100,10 +100,22 @@ def ns_executed_flops(cfg: S.ParamSetConfig, steps: int) -> float:
     return tot
 
 
+def l_psi_bf16(cfg: S.ParamSetConfig) -> bool:
+    """NormPre-L keeps Psi in bf16 on the pure-bf16 workloads (bf16 weights:
+    the paper's Qwen3 runs, App. A) and in fp32 where the parameters are fp32
+    (GPT-2, LLaMA)."""
+    return cfg.w_dtype == "bf16"
+
+
+def psi_bytes(cfg: S.ParamSetConfig, variant: str) -> int:
+    """bf16 Newton-Schulz input (G); bf16 or fp32 sketch input (L); fp32 for L-exact."""
+    return 2 if variant == "G" or (variant == "L" and l_psi_bf16(cfg)) else 4
+
+
 def bytes_per_elt(cfg: S.ParamSetConfig, variant: str):
     g = 2 if cfg.g_dtype == "bf16" else 4
     w = 2 if cfg.w_dtype == "bf16" else 4
-    psi = 2 if variant == "G" else 4        # bf16 Newton-Schulz input, fp32 for the L variants
+    psi = psi_bytes(cfg, variant)
     normalize = g + 4 + 4 + w + psi          # read G, M, W; write M, Psi
     apply = psi + 2 * w                      # read T (or Psi), read/write W
     return normalize, apply
@@ -178,7 +190,8 @@ def oracle_time(cfg: S.ParamSetConfig, variant: str, combo) -> float:
     from synth.inputs import make_matrix
     shp, idx, t = combo
     oc = O.OracleConfig(variant=variant, rank=cfg.rank, oversample=0 if variant == "L_exact" else cfg.oversample,
-                        power_iters=cfg.power_iters, seed=1234)
+                        power_iters=cfg.power_iters, seed=1234,
+                        psi_storage="bf16" if variant == "L" and l_psi_bf16(cfg) else "exact")
     mats = make_matrix(cfg, idx[0])
     t0 = time.perf_counter()
     O.normpre_step(mats["W"], mats["G"], mats["M"], t, LR, oc, matrix_id=idx[0])
@@ -313,18 +326,41 @@ def _roofline(cfg, variant, prof, steps, clocks, exact_sweeps=None):
                 "select_ms_per_step": prof["exact_select"][0] / steps,
                 "sweeps_per_matrix": exact_sweeps,
                 "traffic": None}
-    con_ms = prof["contract"][0] / steps
-    con_launches = prof["contract"][1] / steps
-    # each contraction streams the fp32 Psi of its group once: Y0 = Psi Omega,
-    # Psi^T Y and Psi Z per power iteration, B = Q^T Psi
-    nbytes = n_el * 4.0 * (2 + 2 * cfg.power_iters)
-    achieved = nbytes / (con_ms * 1e-3) / 1e9
-    return {"bound": "hbm", "kernel": "k_contract_tc (sketch contractions of Psi, tcgen05 TF32 split)",
-            "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+    # NormPre-L: the three HBM-bound kernel classes, algorithmic bytes per step;
+    # the roofline line is the one that takes the most time
+    psi = psi_bytes(cfg, variant)
+    b_norm, b_apply = bytes_per_elt(cfg, variant)
+    bf = psi == 2
+    classes = {
+        # each contraction streams Psi once: Y0 = Psi Omega, Psi^T Y and Psi Z
+        # per power iteration, B = Q^T Psi
+        "contract": (n_el * psi * (2.0 + 2 * cfg.power_iters),
+                     "k_contract_bf (sketch contractions of the bf16 Psi, tcgen05 kind::f16, V split hi + lo)" if bf
+                     else "k_contract_tc (sketch contractions of the fp32 Psi, tcgen05 TF32 split)"),
+        # G, M, W read once, M and Psi written once (the column-active steps
+        # read M and W a second time: counted against the kernel)
+        "normalize": (n_el * b_norm, "k_norm_rows_* / k_norm_cols_* (momentum, tangent, normalization)"),
+        # Psi and W read, W written
+        "apply_l": (n_el * b_apply, "k_apply_tc (Psi + Lm Rm^T and the weight update, tcgen05 TF32 split)"),
+    }
+    kern = {}
+    for name, (nbytes, label) in classes.items():
+        ms = prof[name][0] / steps
+        nl = prof[name][1] / steps
+        if ms <= 0 or nl <= 0:
+            continue
+        ach = nbytes / (ms * 1e-3) / 1e9
+        kern[name] = {"kernel": label, "achieved": ach, "frac": ach / hbm, "ms_per_step": ms,
+                      "bytes_per_launch": nbytes / nl, "ms_per_launch": ms / nl, "launches_per_step": nl}
+    top = max(kern, key=lambda k: kern[k]["ms_per_step"])
+    d = kern[top]
+    return {"bound": "hbm", "kernel": d["kernel"], "class": top,
+            "achieved": d["achieved"], "peak": hbm, "unit": "GB/s", "frac": d["frac"],
             "peak_source": "%s HBM copy bandwidth" % peak_src,
-            "bytes_per_launch": nbytes / con_launches, "ms_per_launch": con_ms / con_launches,
-            "launches_per_step": con_launches,
-            "traffic": NCU_TRAFFIC_PER_LAUNCH.get((cfg.name, variant))}
+            "bytes_per_launch": d["bytes_per_launch"], "ms_per_launch": d["ms_per_launch"],
+            "launches_per_step": d["launches_per_step"],
+            "traffic": NCU_TRAFFIC_PER_LAUNCH.get((cfg.name, variant, top)),
+            "classes": {k: {kk: v for kk, v in x.items() if kk != "kernel"} for k, x in kern.items()}}
 
 
 def measure_variant(args, cfg, variant, host, dev):
@@ -340,7 +376,7 @@ def measure_variant(args, cfg, variant, host, dev):
     G = [x.to("cuda", non_blocking=False) for x in Gh]
     M = [x.to("cuda", non_blocking=False) for x in Mh]
     stream = torch.cuda.current_stream()
-    prec = C.NORMPRE_PREC_BF16 if variant == "G" else C.NORMPRE_PREC_F32
+    prec = C.NORMPRE_PREC_BF16 if psi_bytes(cfg, variant) == 2 else C.NORMPRE_PREC_F32
     vcode = {"G": C.NORMPRE_G, "L": C.NORMPRE_L, "L_exact": C.NORMPRE_L_EXACT}[variant]
     opt = NormPre([(m.rows, m.cols) for m in cfg.matrices], [cfg.w_dtype] * cfg.n_mats,
                   [cfg.g_dtype] * cfg.n_mats, variant=vcode,
@@ -449,6 +485,7 @@ def measure_variant(args, cfg, variant, host, dev):
     del Wh2, Mh2
     torch.cuda.empty_cache()
     return {"ms_per_step": ms_step, "warmup": warm, "launches": launches, "clocks": clocks,
+            "psi_dtype": "bf16" if prec == C.NORMPRE_PREC_BF16 else "f32",
             "step_ms": step_dist, "roofline": roof,
             "normalize": {"achieved": norm_gbs, "peak": hbm, "unit": "GB/s",
                           "frac": (norm_gbs / hbm) if norm_gbs else None, "bytes_per_element": b_norm},
@@ -525,6 +562,7 @@ def run_ours(args, cfg, variants):
                 "rank": cfg.rank if v in ("L", "L_exact") else None,
                 "oversample": cfg.oversample if v == "L" else None,
                 "power_iters": cfg.power_iters if v == "L" else None,
+                "psi_dtype": res[v]["psi_dtype"],
                 "l2": ("inputs larger than L2 (W, G, M = %.0f MB)" if res[v]["e2e"]["h2d_bytes_per_step"] >
                        L2_BYTES else "inputs within L2 (W, G, M = %.0f MB): a latency-scale workload, not "
                        "flushed between steps") % (res[v]["e2e"]["h2d_bytes_per_step"] / 1e6),
@@ -533,7 +571,7 @@ def run_ours(args, cfg, variants):
     def entry(v):
         r = res[v]
         return {"value": r["ms_per_step"], "unit": "ms", "ms_per_step": r["ms_per_step"],
-                "dtype": "bf16" if v == "G" else "f32", "config": config_of(v),
+                "dtype": "bf16" if res[v]["psi_dtype"] == "bf16" else "f32", "config": config_of(v),
                 "e2e": r["e2e"], "gpu_launches": r["launches"], "step_ms": r["step_ms"],
                 "roofline": r["roofline"], "normalize": r["normalize"], "phases": r["phases"],
                 "muon": r["muon"], "cpu_baseline": r["cpu_baseline"], "clocks": r["clocks"]}

@@ -84,7 +84,13 @@ enum normpre_status {
 /* Which precision the spectral stage computes in. */
 enum normpre_precision {
   NORMPRE_PREC_BF16 = 0,   /* NormPre-G: Psi and the Newton-Schulz operands in bf16 with fp32
-                              accumulation on the tensor cores; normalization in fp32 */
+                              accumulation on the tensor cores; normalization in fp32.
+                              NormPre-L (the sketch; the pure-bf16 setting of the paper's Qwen3
+                              runs, App. A): Psi stored in bf16 (rounded once from the fp32
+                              normalization), contracted against the bf16 hi + lo split of the
+                              fp32 panels with fp32 accumulation; the panels, CholeskyQR,
+                              Rayleigh-Ritz and the update stay fp32.  A group with l > 64 keeps
+                              an fp32 Psi.  NORMPRE_L_EXACT ignores it (fp32). */
   NORMPRE_PREC_F32 = 1     /* everything in fp32 (parity mode) */
 };
 
@@ -189,7 +195,8 @@ int normpre_sync_status(normpre_handle* h, void* stream);
 /* What normpre_read / normpre_buffer_info can return for one matrix. */
 enum normpre_buffer {
   NORMPRE_BUF_PSI = 0,    /* Psi in the stored layout (rows x cols): the normalized update of the
-                             last step; bf16 in NORMPRE_PREC_BF16 with NORMPRE_G, else fp32 */
+                             last step; bf16 in NORMPRE_PREC_BF16 with NORMPRE_G or NORMPRE_L
+                             (l <= 64), else fp32 */
   NORMPRE_BUF_T = 1,      /* NormPre-G: Newton-Schulz result T in the stored layout (rows x cols),
                              same dtype as PSI */
   NORMPRE_BUF_Q = 2,      /* NormPre-L: orthonormal basis Q of the sketch, m_a x l, fp32; a column

@@ -261,6 +261,13 @@ struct SketchGroup {
   // and MN-major (box 32 x 32) A operand; tc = false keeps the SIMT kernel
   CUtensorMap psi_map_k, psi_map_mn;
   bool tc = false;
+  // NORMPRE_L in NORMPRE_PREC_BF16: Psi stored in bf16 ([rows][ld] bf16 in the
+  // same buffer), contracted by contract_bf16.cu (TMA map psi_map_bf, box
+  // 64 x 64) against the bf16 hi / lo split of V in vb [batch][vb_bs]
+  bool psi_bf16 = false;
+  CUtensorMap psi_map_bf;
+  void* vb = nullptr;
+  int64_t vb_bs = 0;
 };
 
 struct SketchParams {
@@ -293,6 +300,27 @@ cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup
 cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* mat_ids,
                              const int* count, void* const* W, int* flags, cudaStream_t s,
                              ProfileHook* prof);
+
+// bf16-Psi sketch contraction (contract_bf16.cu): out = op(Psi) V, op(Psi) =
+// Psi (trans = false, K = cols) or Psi^T (trans = true, K = rows), V fp32
+// [K][l] (l <= 64), vb the bf16 split scratch (vb_bs elements per matrix,
+// at least 2 * round_up(l, 16) * round_up(K, 64)).  With ksplit > 1, out
+// receives per-split partials [ksplit][P][l] per matrix (stride out_bs).
+struct ContractBf16Launch {
+  const CUtensorMap* psi_map;
+  bool trans;
+  const float* v; int64_t v_bs;
+  void* vb; int64_t vb_bs;
+  float* out; int64_t out_bs;
+  int64_t P, K;
+  int l;
+  int64_t kchunk;          // multiple of 64
+  int ksplit, batch;
+  int* flags;
+  int stall_first_copy;
+};
+bool contract_bf16_map(CUtensorMap* map, const void* psi, int64_t rows, int64_t cols, int64_t ld, int batch);
+cudaError_t launch_contract_bf16(const ContractBf16Launch& c, cudaStream_t s);
 
 // Records the message returned by normpre_last_error(NULL) on this thread.
 void set_thread_error(const std::string& msg);

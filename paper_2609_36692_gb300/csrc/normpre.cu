@@ -285,6 +285,9 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
       g.sk.rows = g.rows; g.sk.cols = g.cols; g.sk.w_dtype = g.w_dtype;
       g.sk.ld = round_up(g.cols, 8);
       const bool exact = cfg->variant == NORMPRE_L_EXACT;
+      // the sketch keeps Psi in bf16 in the bf16 precision mode (where its
+      // contraction kernel applies: sketch_group_alloc may clear the flag)
+      g.sk.psi_bf16 = !exact && cfg->precision == NORMPRE_PREC_BF16;
       e = sketch_group_alloc(g.sk, cfg->rank, exact ? 0 : cfg->oversample, h->allocs);
       if (e != cudaSuccess) return cuda_fail(nullptr, e, "sketch workspace");
       if (exact) {
@@ -369,7 +372,7 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
     } else {
       psi_base = reinterpret_cast<char*>(g.sk.psi);
       psi_ld = g.sk.ld;
-      psi_bs = g.rows * g.sk.ld * static_cast<int64_t>(sizeof(float));
+      psi_bs = g.rows * g.sk.ld * static_cast<int64_t>(g.sk.psi_bf16 ? 2 : 4);
     }
     cudaError_t e;
     if ((e = hk.before_normalize(ui, s))) return cuda_fail(h, e, "stream wait");
@@ -379,7 +382,8 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
       NormLaunch a;
       a.n = std::min(kMaxBatch, u.b1 - c0);
       a.rows = g.rows; a.cols = g.cols;
-      a.g_dtype = g.g_dtype; a.w_dtype = g.w_dtype; a.psi_dtype = psi_bf16 ? 1 : 0;
+      a.g_dtype = g.g_dtype; a.w_dtype = g.w_dtype;
+      a.psi_dtype = (is_g ? psi_bf16 : g.sk.psi_bf16) ? 1 : 0;
       for (int i = 0; i < a.n; ++i) {
         const int mid = g.mats[c0 + i];
         a.G[i] = G[mid]; a.M[i] = static_cast<float*>(M[mid]); a.W[i] = W[mid];
@@ -735,7 +739,8 @@ int normpre_buffer_info(const normpre_handle* h, int mat, int what, int64_t* row
   switch (what) {
     case NORMPRE_BUF_PSI:
       r = m.rows; c = m.cols;
-      dt = (is_g && h->cfg.precision == NORMPRE_PREC_BF16) ? NORMPRE_BF16 : NORMPRE_F32;
+      dt = ((is_g && h->cfg.precision == NORMPRE_PREC_BF16) || (!is_g && h->groups[m.group].sk.psi_bf16))
+               ? NORMPRE_BF16 : NORMPRE_F32;
       break;
     case NORMPRE_BUF_T:
       if (!is_g) return fail(hh, NORMPRE_ERR_ARG, "T is kept only for NormPre-G");
@@ -814,7 +819,9 @@ int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capaci
       src = static_cast<char*>(nb.X[idx]) + static_cast<int64_t>(m.slot) * nb.rows_pad * nb.cols_pad * nb.elem;
       src_ld = nb.cols_pad;
     } else {
-      src = g.sk.psi + static_cast<int64_t>(m.slot) * g.rows * g.sk.ld;
+      src = g.sk.psi_bf16 ? static_cast<const void*>(reinterpret_cast<const uint16_t*>(g.sk.psi) +
+                                                      static_cast<int64_t>(m.slot) * g.rows * g.sk.ld)
+                          : static_cast<const void*>(g.sk.psi + static_cast<int64_t>(m.slot) * g.rows * g.sk.ld);
       src_ld = g.sk.ld;
     }
   } else if (what == NORMPRE_BUF_STATS) {

@@ -411,15 +411,6 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float* v) {
       : "memory");
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-// 32 TMEM lanes x 16 consecutive 32-bit columns: thread i receives lane (base + i).
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-}
 // D[tmem] (+)= A[tmem] * B[smem]^T, kind::tf32
 __device__ __forceinline__ void mma_tf32_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
                                             uint32_t accumulate) {
@@ -662,8 +653,8 @@ __global__ void __launch_bounds__(kCtcThreads, 1) k_contract_tc(const __grid_con
             // Ahi Vhi + Alo Vhi in columns 16 h.., Ahi Vlo in 64 + 16 h..
             uint32_t r[16], v[16];
             const uint32_t col = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * acc + 16 * h);
-            tmem_ld16(col, r);
-            tmem_ld16(col + 64u, v);
+            tc::tmem_ld16(col, r);
+            tc::tmem_ld16(col + 64u, v);
             tc::tmem_ld_wait();
 #pragma unroll
             for (int j = 0; j < 16; ++j) sum[16 * h + j] += __uint_as_float(r[j]) + __uint_as_float(v[j]);
@@ -1382,7 +1373,8 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
 // 64 x 64 tiles, thread = 4 x 4 block of consecutive rows / columns.
 // ---------------------------------------------------------------------------
 struct LApplyArgs {
-  const float* psi; int64_t psi_bs, psi_ld;
+  const void* psi; int64_t psi_bs, psi_ld;   // fp32, or bf16 when psi_bf16 (strides in elements)
+  int psi_bf16;
   const float* lm; int64_t lm_bs;
   const float* rm; int64_t rm_bs;
   const float* stats; int64_t stats_bs;
@@ -1459,7 +1451,8 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
       for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(la[r], ra[c], acc[r][c]);
   }
   const float cw = 1.f - a.lr * a.wd, ct = -a.lr * scale_s;
-  const float* psi = a.psi + b * a.psi_bs;
+  const float* psi = static_cast<const float*>(a.psi) + b * a.psi_bs;
+  const bf16* psib = static_cast<const bf16*>(a.psi) + b * a.psi_bs;
   TW* W = static_cast<TW*>(a.W[b]);
   const int64_t j0 = c0 + tx * 4;
 #pragma unroll
@@ -1467,8 +1460,14 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
     const int64_t i = r0 + ty * 4 + r;
     if (i >= a.rows) continue;
     if (VEC && j0 + 4 <= a.cols) {
-      const float4 pv = *reinterpret_cast<const float4*>(psi + i * a.psi_ld + j0);
-      const float ps[4] = {pv.x, pv.y, pv.z, pv.w};
+      float ps[4];
+      if (a.psi_bf16) {
+        const uint2 pv = *reinterpret_cast<const uint2*>(psib + i * a.psi_ld + j0);
+        ps[0] = bf16lo(pv.x); ps[1] = bf16hi(pv.x); ps[2] = bf16lo(pv.y); ps[3] = bf16hi(pv.y);
+      } else {
+        const float4 pv = *reinterpret_cast<const float4*>(psi + i * a.psi_ld + j0);
+        ps[0] = pv.x; ps[1] = pv.y; ps[2] = pv.z; ps[3] = pv.w;
+      }
       float w[4];
       if (std::is_same<TW, float>::value) {
         const float4 wv = *reinterpret_cast<const float4*>(reinterpret_cast<float*>(W) + i * a.cols + j0);
@@ -1493,7 +1492,7 @@ __global__ void __launch_bounds__(256) k_apply_l(const __grid_constant__ LApplyA
       for (int c = 0; c < 4; ++c) {
         const int64_t j = j0 + c;
         if (j >= a.cols) continue;
-        const float t = psi[i * a.psi_ld + j] + acc[r][c];
+        const float t = (a.psi_bf16 ? to_f32(psib[i * a.psi_ld + j]) : psi[i * a.psi_ld + j]) + acc[r][c];
         const float w = to_f32(W[i * a.cols + j]);
         W[i * a.cols + j] = from_f32<TW>(fmaf(cw, w, ct * t));
         diag_add(i * a.cols + j, t);
@@ -1575,7 +1574,7 @@ __device__ __forceinline__ void atc_split_rows(const float* panel, int64_t r0, i
   }
 }
 
-template <typename TW>
+template <typename TW, typename TP>
 __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_constant__ LApplyArgs a, int nmat,
                                                               int natoms, int* flags) {
   extern __shared__ uint8_t atc_raw[];
@@ -1704,12 +1703,12 @@ __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_consta
     int icc = 0;
     int cur_b = -1;
     float cur_ct = 0.f;
-    float pv[S][CH];
+    TP pv[S][CH];
     TW wv[S][CH];
     TW* wp[S];
     int nr[S];
     float ctt[S];
-    auto issue = [&](int64_t k, float* P, TW* Wv, TW*& wptr, int& nrows, float& ct) {
+    auto issue = [&](int64_t k, TP* P, TW* Wv, TW*& wptr, int& nrows, float& ct) {
       if (k < nck) {
         const int64_t j = ij0 + 32 * q + lane;
         const int64_t r0 = ii0 + 128 * h + CH * icc;
@@ -1725,7 +1724,7 @@ __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_consta
           cur_b = ib;
         }
         ct = cur_ct;
-        const float* pptr = a.psi + ib * a.psi_bs + r0 * a.psi_ld + j;
+        const TP* pptr = static_cast<const TP*>(a.psi) + ib * a.psi_bs + r0 * a.psi_ld + j;
         wptr = static_cast<TW*>(a.W[ib]) + r0 * a.cols + j;
         nrows = (r0 < a.rows && j < a.cols) ? static_cast<int>(a.rows - r0 < CH ? a.rows - r0 : CH) : 0;
         if (nrows == CH) {
@@ -1737,7 +1736,7 @@ __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_consta
         } else {
 #pragma unroll
           for (int rr = 0; rr < CH; ++rr) {
-            P[rr] = rr < nrows ? pptr[rr * a.psi_ld] : 0.f;
+            P[rr] = rr < nrows ? pptr[rr * a.psi_ld] : from_f32<TP>(0.f);
             Wv[rr] = rr < nrows ? wptr[rr * a.cols] : from_f32<TW>(0.f);
           }
         }
@@ -1769,7 +1768,7 @@ __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_consta
           tc::fence_after();
         }
         uint32_t v[CH];
-        tmem_ld16(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(256 * acc + 128 * h + CH * c), v);
+        tc::tmem_ld16(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(256 * acc + 128 * h + CH * c), v);
         tc::tmem_ld_wait();
         if (c == NCH - 1) {
           // the accumulator is read: the MMAs of unit it + 2 may overwrite it
@@ -1781,12 +1780,12 @@ __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_consta
         if (nr[sl] == CH) {
 #pragma unroll
           for (int rr = 0; rr < CH; ++rr)
-            W[rr * a.cols] = from_f32<TW>(fmaf(cw, to_f32(wv[sl][rr]), ctt[sl] * (pv[sl][rr] + __uint_as_float(v[rr]))));
+            W[rr * a.cols] = from_f32<TW>(fmaf(cw, to_f32(wv[sl][rr]), ctt[sl] * (to_f32(pv[sl][rr]) + __uint_as_float(v[rr]))));
         } else {
 #pragma unroll
           for (int rr = 0; rr < CH; ++rr)
             if (rr < nr[sl])
-              W[rr * a.cols] = from_f32<TW>(fmaf(cw, to_f32(wv[sl][rr]), ctt[sl] * (pv[sl][rr] + __uint_as_float(v[rr]))));
+              W[rr * a.cols] = from_f32<TW>(fmaf(cw, to_f32(wv[sl][rr]), ctt[sl] * (to_f32(pv[sl][rr]) + __uint_as_float(v[rr]))));
         }
         issue(k + S, pv[sl], wv[sl], wp[sl], nr[sl], ctt[sl]);
       }
@@ -1903,6 +1902,13 @@ cudaError_t sketch_group_alloc(SketchGroup& g, int rank, int oversample, std::ve
       cudaFuncSetAttribute(k_contract_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kCtcSmem));
     }
   }
+  // bf16 Psi (set by the caller for NORMPRE_L in NORMPRE_PREC_BF16): kept only
+  // where the bf16 contraction applies (l <= 64, 16-byte Psi rows)
+  if (g.psi_bf16) {
+    g.vb_bs = 2 * round_up(g.lmax, 16) * round_up(big, 64);
+    g.psi_bf16 = g.lmax <= 64 && contract_bf16_map(&g.psi_map_bf, g.psi, g.rows, g.cols, g.ld, g.batch);
+    if (g.psi_bf16 && (e = alloc(&g.vb, static_cast<size_t>(g.batch) * g.vb_bs * sizeof(uint16_t)))) return e;
+  }
   // the largest Jacobi footprint, so that groups of any width can share the kernel
   cudaFuncSetAttribute(k_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kJacSmem));
   return cudaGetLastError();
@@ -1915,7 +1921,12 @@ cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup
   const int64_t sq = static_cast<int64_t>(g.lmax) * g.lmax;
   s.batch = b1 - b0;
   s.plan_batch = g.plan_batch ? g.plan_batch : g.batch;
-  s.psi = g.psi + b0 * g.rows * g.ld;
+  s.psi = g.psi_bf16 ? reinterpret_cast<float*>(reinterpret_cast<uint16_t*>(g.psi) + b0 * g.rows * g.ld)
+                     : g.psi + b0 * g.rows * g.ld;
+  if (g.psi_bf16) {
+    s.vb = static_cast<uint16_t*>(g.vb) + b0 * g.vb_bs;
+    if (!contract_bf16_map(&s.psi_map_bf, s.psi, g.rows, g.cols, g.ld, s.batch)) return cudaErrorInvalidValue;
+  }
   float** vbufs[] = {&s.omega, &s.y0, &s.zt, &s.y, &s.q, &s.bt, &s.qk};
   for (float** v : vbufs) *v += b0 * vbs;
   s.kpart = g.kpart + b0 * vbs * kMaxKSplit;
@@ -1934,7 +1945,7 @@ cudaError_t sketch_group_slice(const SketchGroup& g, int b0, int b1, SketchGroup
     s.oj_sel = g.oj_sel + static_cast<int64_t>(b0) * g.lmax;
     s.oj_sel_lam = g.oj_sel_lam + static_cast<int64_t>(b0) * g.lmax;
   }
-  if (g.tc) {
+  if (g.tc && !g.psi_bf16) {
     const uint64_t dims[3] = {static_cast<uint64_t>(g.cols), static_cast<uint64_t>(g.rows),
                               static_cast<uint64_t>(s.batch)};
     const uint64_t strides[2] = {static_cast<uint64_t>(g.ld) * 4, static_cast<uint64_t>(g.rows * g.ld) * 4};
@@ -1981,7 +1992,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   // rows.  K is split when the tiles alone would leave SMs idle (fixed-order reduce).
   // the tensor-core form needs 16-byte rows of the l-wide operand and 16-byte
   // aligned per-matrix strides (TMA)
-  const bool use_tc = g.tc && (l % 4 == 0) && (vbs % 4 == 0) && l <= 64;
+  const bool use_tc = g.psi_bf16 || (g.tc && (l % 4 == 0) && (vbs % 4 == 0) && l <= 64);
   bool stall_pending = p.test_stall != 0;   // the first tensor-core contraction of the step
   auto contract = [&](bool trans, const float* v, float* out) -> cudaError_t {
     prof->begin(kProfContract, s);
@@ -2002,7 +2013,20 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       c.out = g.kpart; c.out_bs = vbs * kMaxKSplit;
     }
     cudaError_t err;
-    if (use_tc) {
+    if (g.psi_bf16) {
+      ContractBf16Launch cb;
+      cb.psi_map = &g.psi_map_bf; cb.trans = trans;
+      cb.v = v; cb.v_bs = vbs;
+      cb.vb = g.vb; cb.vb_bs = g.vb_bs;
+      cb.out = c.out; cb.out_bs = c.out_bs;
+      cb.P = P; cb.K = K; cb.l = l;
+      cb.kchunk = round_up(cdiv(K, ks), 64);
+      cb.ksplit = ks; cb.batch = B;
+      cb.flags = flags;
+      cb.stall_first_copy = stall_pending ? 1 : 0;
+      stall_pending = false;
+      err = launch_contract_bf16(cb, s);
+    } else if (use_tc) {
       const int np = static_cast<int>(round_up(l, 16));
       ContractTcArgs ct;
       std::memset(static_cast<void*>(&ct), 0, sizeof(ct));
@@ -2031,7 +2055,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       err = trans ? launch_contract<true>(c, B, cpt, s) : launch_contract<false>(c, B, cpt, s);
     }
     if (err) return err;
-    int n_l = 1;
+    int n_l = g.psi_bf16 ? 2 : 1;   // the bf16 path splits V in a launch of its own
     if (ks > 1) {
       SplitReduceArgs r;
       r.part = g.kpart; r.part_bs = vbs * kMaxKSplit;
@@ -2161,7 +2185,9 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     const int nb = std::min(kMaxBatch, B - c0);
     ++n_apply;
     LApplyArgs la;
-    la.psi = g.psi + c0 * psi_bs; la.psi_bs = psi_bs; la.psi_ld = g.ld;
+    la.psi = g.psi_bf16 ? static_cast<const void*>(reinterpret_cast<const bf16*>(g.psi) + c0 * psi_bs)
+                        : static_cast<const void*>(g.psi + c0 * psi_bs);
+    la.psi_bs = psi_bs; la.psi_ld = g.ld; la.psi_bf16 = g.psi_bf16 ? 1 : 0;
     la.lm = (rows_active ? g.qk : g.bt) + c0 * vbs; la.lm_bs = vbs;
     la.rm = (rows_active ? g.bt : g.qk) + c0 * vbs; la.rm_bs = vbs;
     la.stats = g.stats + c0 * 8; la.stats_bs = 8;
@@ -2182,18 +2208,29 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       // the two-atom size for every l: one CTA per SM, so the 512 TMEM
       // columns of a CTA never wait for another's
       const size_t smem = atc_smem(2);
-      static bool attr_f = false, attr_b = false;
-      bool& attr = g.w_dtype == 0 ? attr_f : attr_b;
-      if (!attr) {
-        e = g.w_dtype == 0 ? cudaFuncSetAttribute(k_apply_tc<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(atc_smem(2)))
-                           : cudaFuncSetAttribute(k_apply_tc<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(atc_smem(2)));
-        if (e != cudaSuccess) return e;
-        attr = true;
+      static bool attr_set[4] = {false, false, false, false};
+      const int kind = 2 * (g.w_dtype != 0) + (g.psi_bf16 ? 1 : 0);
+      auto go = [&](auto* tw, auto* tp) -> cudaError_t {
+        using TWT = std::remove_pointer_t<decltype(tw)>;
+        using TPT = std::remove_pointer_t<decltype(tp)>;
+        if (!attr_set[kind]) {
+          const cudaError_t ea = cudaFuncSetAttribute(k_apply_tc<TWT, TPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      static_cast<int>(smem));
+          if (ea != cudaSuccess) return ea;
+          attr_set[kind] = true;
+        }
+        const int64_t units = cdiv(g.rows, kAtcRows) * cdiv(g.cols, kAtcCols) * nb;
+        const unsigned ctas = static_cast<unsigned>(std::min<int64_t>(units, device_sm_count()));
+        k_apply_tc<TWT, TPT><<<ctas, kAtcThreads, smem, s>>>(la, nb, natoms, flags);
+        return cudaGetLastError();
+      };
+      switch (kind) {
+        case 0: e = go((float*)nullptr, (float*)nullptr); break;
+        case 1: e = go((float*)nullptr, (bf16*)nullptr); break;
+        case 2: e = go((bf16*)nullptr, (float*)nullptr); break;
+        default: e = go((bf16*)nullptr, (bf16*)nullptr); break;
       }
-      const int64_t units = cdiv(g.rows, kAtcRows) * cdiv(g.cols, kAtcCols) * nb;
-      const unsigned ctas = static_cast<unsigned>(std::min<int64_t>(units, device_sm_count()));
-      if (g.w_dtype == 0) k_apply_tc<float><<<ctas, kAtcThreads, smem, s>>>(la, nb, natoms, flags);
-      else k_apply_tc<bf16><<<ctas, kAtcThreads, smem, s>>>(la, nb, natoms, flags);
+      if (e != cudaSuccess) return e;
       NP_CHECK();
       continue;
     }

@@ -120,7 +120,7 @@ def test_normalize_and_momentum(cfgset, t, w_dtype):
         assert int(st[0]) == k and int(st[1]) == int((ref["d"] > 0).sum())
 
 
-def _check_bf16_w(w_gpu, w_ref, dw_ref, tol, where):
+def _check_bf16_w(w_gpu, w_ref, dw_ref, tol, where, elem_tol=None):
     """bf16 weights: the device stores the bf16 rounding (RNE) of its fp32
     update.  Element by element, the stored value is within one bf16 ulp of the
     oracle's exact W_{t+1} plus that element's share of the update tolerance:
@@ -128,10 +128,12 @@ def _check_bf16_w(w_gpu, w_ref, dw_ref, tol, where):
     roundings of a bf16 product scale with the entry) plus 6 times the
     root-mean-square share (the error spread over the matrix).  In aggregate,
     the Frobenius error is within the update tolerance plus the half-ulp
-    rounding of every element."""
+    rounding of every element.  `elem_tol` (default `tol`) replaces the
+    tolerance in the element-wise share."""
     w_gpu = np.asarray(w_gpu, np.float64)
     err = np.abs(w_gpu - w_ref)
-    share = tol * (np.abs(dw_ref) + 6.0 * np.sqrt(np.mean(dw_ref ** 2)))
+    et = tol if elem_tol is None else elem_tol
+    share = et * (np.abs(dw_ref) + 6.0 * np.sqrt(np.mean(dw_ref ** 2)))
     bound = bf16_ulp(w_ref) + share
     worst = int(np.argmax(err - bound))
     assert np.all(err <= bound), (where, worst, float(err.flat[worst]), float(bound.flat[worst]))
@@ -369,6 +371,71 @@ def test_l_large_sets_sampled(name, indices, t):
     import dataclasses
     cs = dataclasses.replace(S.CONFIGS[name], rank=32, oversample=8)
     _check_l(cs, t, indices=indices)
+
+
+# ---------------------------------------------------------------------------
+# NormPre-L with Psi stored in bf16 (NORMPRE_PREC_BF16: the pure-bf16 setting
+# of the paper's Qwen3 runs, App. A), against the oracle that rounds its exact
+# Psi to bf16 once.  The library rounds its fp32 normalization (within 1e-5 of
+# the line norm) once, so the two bf16 Psi agree except where the fp32 value
+# fell across a rounding boundary: there they are one bf16 spacing apart.
+# Those few one-spacing differences (~1% of the entries) perturb Psi by
+# ~1e-4 of its norm, hence the looser sketch tolerances: Ritz values within
+# 1e-3 of max(1, lam_1), subspaces within a principal-angle sine of 1e-2 where
+# the selection is separated by 1e-2, the update within 3e-3 in aggregate.
+# Element by element, a Psi entry one spacing off moves its entry of T by up to
+# 2^-7 of itself, so bf16 weights take 2^-7 + 3e-3 as their element-wise share.
+# ---------------------------------------------------------------------------
+def _check_l_bf16(cs, t, indices=None, w_tol=3e-3):
+    from paper_2609_36692_gb300 import normpre as C
+    opt, mats, W1, _ = _run(cs, t, "L", precision=0)
+    idx = range(cs.n_mats) if indices is None else indices
+    for i in idx:
+        ref = _oracle(mats, i, t, "L", cs, psi_storage="bf16")
+        k = ref["k"]
+        assert C.normpre_buffer_info(opt.handle, i, C.NORMPRE_BUF_PSI)[2] == C.NORMPRE_BF16
+        psi = opt.read(i, C.NORMPRE_BUF_PSI).astype(np.float64)
+        ref_psi = _stored(ref["Psi"], k)
+        line = np.linalg.norm(ref_psi, axis=1 - k, keepdims=True)
+        diff = np.abs(psi - ref_psi)
+        assert np.all(diff <= bf16_ulp(ref_psi) + 1e-5 * line), (cs.name, i)
+        assert np.mean(diff > 0) <= 0.05, (cs.name, i, np.mean(diff > 0))
+        sk = ref["sketch"]
+        ritz = opt.read(i, C.NORMPRE_BUF_RITZ)[0]
+        lam = sk["ritz"]
+        assert np.max(np.abs(ritz - lam)) <= 1e-3 * max(1.0, lam[0]), (cs.name, i)
+        st = opt.read(i, C.NORMPRE_BUF_STATS)[0]
+        if ritz_gaps_ok(lam, cs.rank, tol=1e-2 * max(1.0, lam[0])):
+            nc = int(st[3])
+            assert nc == sk["n_active"], (cs.name, i, nc, sk["n_active"])
+            Q = opt.read(i, C.NORMPRE_BUF_Q)
+            Z = opt.read(i, C.NORMPRE_BUF_Z)
+            U = Q.astype(np.float64) @ Z[:, :nc].astype(np.float64)
+            assert principal_sine(U, sk["U_C"]) <= 1e-2, (cs.name, i)
+        dW = W1[i].astype(np.float64) - mats[i]["W"]
+        dW_ref = ref["W"] - mats[i]["W"]
+        if cs.w_dtype == "f32":
+            assert rel_fro(dW, dW_ref) <= w_tol, (cs.name, i, rel_fro(dW, dW_ref))
+        else:
+            _check_bf16_w(W1[i], ref["W"], dW_ref, w_tol, (cs.name, i), elem_tol=2.0 ** -7 + w_tol)
+
+
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED, ODD, TALL], ids=lambda c: c.name)
+@pytest.mark.parametrize("t", [0, 1])
+def test_l_bf16_psi(cfgset, t):
+    """Both contraction orientations of the bf16 kernel, ragged tiles and K
+    blocks, odd sketch widths (l = 19, 11), tall strips and 1-wide matrices."""
+    _check_l_bf16(cfgset, t)
+
+
+@pytest.mark.parametrize("t", [0, 1])
+@pytest.mark.parametrize("name,indices", [("gpt2_small_L", [0, 1, 2, 3, 47]), ("qwen3_1p7b", [0, 1, 4, 6])])
+def test_l_bf16_psi_full_size_sampled(name, indices, t):
+    """The GPT-2 and Qwen3 sets at full size in the bf16 mode (the Qwen3
+    configuration the benchmark runs), one matrix of each shape checked."""
+    import dataclasses
+    cs = dataclasses.replace(S.CONFIGS[name], rank=32, oversample=8)
+    _check_l_bf16(cs, t, indices=indices)
 
 
 # ---------------------------------------------------------------------------
@@ -692,10 +759,12 @@ def test_jacobi_sweep_cap_reports_numeric():
     opt.close()
 
 
-def test_bounded_wait_timeout_reports_and_recovers():
-    """The device-side timeout path of the tensor-core kernels: with test_stall,
-    one CTA of each group's first sketch contraction never gets its first copy;
-    its split warps give up after the bounded wait (about two seconds) and set
+@pytest.mark.parametrize("precision", [1, 0], ids=["fp32", "bf16_psi"])
+def test_bounded_wait_timeout_reports_and_recovers(precision):
+    """The device-side timeout path of the tensor-core kernels (the fp32
+    contraction, and the bf16-Psi one): with test_stall, one CTA of each
+    group's first sketch contraction never gets its first copy; the warp
+    waiting for it gives up after the bounded wait (about two seconds) and set
     the CTA's abort flag, every other role of that CTA leaves its loop at its
     next wait, thread 0 waits for the copies the CTA did issue, the tensor
     memory is freed and the kernel exits; the step reports
@@ -710,7 +779,7 @@ def test_bounded_wait_timeout_reports_and_recovers():
     W, G, M = to_device(mats, cs.g_dtype, cs.w_dtype)
     shapes = [(m.rows, m.cols) for m in cs.matrices]
     opt = _normpre(shapes, [cs.w_dtype] * cs.n_mats, [cs.g_dtype] * cs.n_mats, variant=C.NORMPRE_L,
-                   precision=1, rank=cs.rank, oversample=cs.oversample, seed=1234, test_stall=1)
+                   precision=precision, rank=cs.rank, oversample=cs.oversample, seed=1234, test_stall=1)
     t0 = time.perf_counter()
     opt.step(0, LR, W, G, M)
     torch.cuda.synchronize()
@@ -719,7 +788,10 @@ def test_bounded_wait_timeout_reports_and_recovers():
     assert "gave up" in C.normpre_last_error(opt.handle)
     assert 1.0 < waited < 60.0, waited
     opt.close()
-    _check_l(cs, 1)
+    if precision == 1:
+        _check_l(cs, 1)
+    else:
+        _check_l_bf16(cs, 1)
 
 
 # one GPT-2 Small attention qkv matrix (768 x 2304): Gamma is 768 x 768 at
