@@ -264,10 +264,11 @@ __global__ void __launch_bounds__(kCbThreads, 1) k_contract_bf(const __grid_cons
   }
 }
 
-bool contract_bf16_map(CUtensorMap* map, const void* psi, int64_t rows, int64_t cols, int64_t ld, int batch) {
+bool contract_bf16_map(CUtensorMap* map, const void* psi, int64_t rows, int64_t cols, int64_t ld, int batch,
+                       int box_rows) {
   const uint64_t dims[3] = {static_cast<uint64_t>(cols), static_cast<uint64_t>(rows), static_cast<uint64_t>(batch)};
   const uint64_t strides[2] = {static_cast<uint64_t>(ld) * 2, static_cast<uint64_t>(rows * ld) * 2};
-  const uint32_t box[3] = {64, 64, 1};
+  const uint32_t box[3] = {64, static_cast<uint32_t>(box_rows), 1};
   return (ld % 8 == 0) &&
          driver_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(psi), dims, strides, box, nullptr);
 }

@@ -265,7 +265,8 @@ struct SketchGroup {
   // same buffer), contracted by contract_bf16.cu (TMA map psi_map_bf, box
   // 64 x 64) against the bf16 hi / lo split of V in vb [batch][vb_bs]
   bool psi_bf16 = false;
-  CUtensorMap psi_map_bf;
+  CUtensorMap psi_map_bf;       // box 64 x 64 (contractions)
+  CUtensorMap psi_map_apply;    // box 64 x 32 (apply)
   void* vb = nullptr;
   int64_t vb_bs = 0;
 };
@@ -319,7 +320,8 @@ struct ContractBf16Launch {
   int* flags;
   int stall_first_copy;
 };
-bool contract_bf16_map(CUtensorMap* map, const void* psi, int64_t rows, int64_t cols, int64_t ld, int batch);
+bool contract_bf16_map(CUtensorMap* map, const void* psi, int64_t rows, int64_t cols, int64_t ld, int batch,
+                       int box_rows = 64);
 cudaError_t launch_contract_bf16(const ContractBf16Launch& c, cudaStream_t s);
 
 // Records the message returned by normpre_last_error(NULL) on this thread.
