@@ -793,12 +793,19 @@ __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramA
 }
 
 // Folds nsplit partial l x l sums into dst (shared, row stride ld), compensated.
-// Loads are issued eight at a time so their latencies overlap.
+// Loads are issued sixteen at a time so their latencies overlap.
 __device__ __forceinline__ void fold_partials(const float* part, int nsplit, int l, float* dst, int ld) {
   const int64_t stride = static_cast<int64_t>(l) * l;
   for (int e = threadIdx.x; e < l * l; e += blockDim.x) {
     Kahan k;
     int s = 0;
+    for (; s + 16 <= nsplit; s += 16) {
+      float v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] = __ldcg(part + (s + u) * stride + e);
+#pragma unroll
+      for (int u = 0; u < 16; ++u) k.add(v[u]);
+    }
     for (; s + 8 <= nsplit; s += 8) {
       float v[8];
 #pragma unroll
@@ -872,8 +879,9 @@ constexpr int kRfacStride = kLmax * kLmax + kLmax + 8;
 
 // One CTA per matrix: fold the Gram partials of the panel, factor G (+ shift)
 // = R^T R right-looking (one pivot per barrier), write R and 1 / R_ii.
+constexpr int kCholThreads = 1024;   // the fold of the Gram partials is latency-bound: many loads in flight
 template <int LP>
-__global__ void __launch_bounds__(256) k_chol_factor(const __grid_constant__ CholQRArgs a, float* rfac) {
+__global__ void __launch_bounds__(kCholThreads) k_chol_factor(const __grid_constant__ CholQRArgs a, float* rfac) {
   // G (row stride LP + 1) until the factorization ends
   __shared__ __align__(16) float GR[LP * (LP + 1)];
   __shared__ float Wm[LP][LP + 1];             // G + shift I, reduced in place
@@ -898,12 +906,12 @@ __global__ void __launch_bounds__(256) k_chol_factor(const __grid_constant__ Cho
   // right-looking Cholesky: at pivot j, W[p][q] -= W[j][p] W[j][q] / W[j][j]
   // for p, q > j (the whole trailing square, so W stays symmetric); row j is
   // final from then on and R[j][i] = W[j][i] / sqrt(W[j][j])
-  const int ty = tid >> 4, tx = tid & 15;
+  const int ty = tid >> 5, tx = tid & 31;
   const float small = 1e-6f * tr;
   bool bad = false;
   for (int attempt = 0; attempt < 2; ++attempt) {
     const float shift = attempt == 0 ? 0.f : 1e-5f * tr;
-    for (int e = tid; e < l * l; e += 256) {
+    for (int e = tid; e < l * l; e += kCholThreads) {
       const int i = e / l, j = e - i * l;
       Wm[i][j] = GR[i * (LP + 1) + j] + (i == j ? shift : 0.f);
     }
@@ -915,9 +923,9 @@ __global__ void __launch_bounds__(256) k_chol_factor(const __grid_constant__ Cho
       if (tiny) bad = true;
       // a dropped column eliminates nothing
       const float dinv = (tiny && a.drop) ? 0.f : 1.f / fmaxf(d, 1e-30f * tr);
-      for (int p = j + 1 + ty; p < l; p += 16) {
+      for (int p = j + 1 + ty; p < l; p += 32) {
         const float wp = Wm[j][p] * dinv;
-        for (int c = j + 1 + tx; c < l; c += 16) Wm[p][c] = fmaf(-wp, Wm[j][c], Wm[p][c]);
+        for (int c = j + 1 + tx; c < l; c += 32) Wm[p][c] = fmaf(-wp, Wm[j][c], Wm[p][c]);
       }
       __syncthreads();
     }
@@ -925,16 +933,16 @@ __global__ void __launch_bounds__(256) k_chol_factor(const __grid_constant__ Cho
   }
   if (tid == 0 && bad && !a.drop) raise_flag(a.flags, kFlagNumeric);
   // W[i][i] is pivot i; a dropped column gets 1 / R_ii = 0 (and so a zero row of R)
-  for (int i = tid; i < LP; i += 256) {
+  for (int i = tid; i < LP; i += kCholThreads) {
     const float d = (i < l) ? Wm[i][i] : 0.f;
     rinv[i] = (i >= l || (a.drop && !(d > small))) ? 0.f : 1.f / sqrtf(fmaxf(d, 1e-30f * tr));
   }
   __syncthreads();
-  for (int e = tid; e < LP * LP; e += 256) {
+  for (int e = tid; e < LP * LP; e += kCholThreads) {
     const int i = e / LP, j = e % LP;
     out[e] = (i < l && j < l && j > i) ? Wm[i][j] * rinv[i] : 0.f;
   }
-  for (int i = tid; i < LP; i += 256) out[LP * LP + i] = rinv[i];
+  for (int i = tid; i < LP; i += kCholThreads) out[LP * LP + i] = rinv[i];
   if (tid == 0) out[LP * LP + LP] = 0.f;
 }
 
@@ -1160,15 +1168,15 @@ __global__ void __launch_bounds__(256) k_rowmul(const __grid_constant__ RowMulAr
 
 // ---------------------------------------------------------------------------
 // Parallel cyclic Jacobi (round-robin pairing) of Gamma_Q in fp32, then the
-// descending sort, the selection C and K.  One CTA per matrix; a rotation
-// step has two phases.  First, thread k < n/2 owns pair k (its two players in
-// registers, advanced every step), computes the pair's rotation from the
-// current copy of A and publishes {c, s, i, j}.  Then the thread that owns
-// 2 x 2 block (k, k') of the n/2 x n/2 block grid writes J^T A J for it (rows
+// descending sort, the selection C and K.  One CTA per matrix.  The thread
+// that owns 2 x 2 block (k, k') of the n/2 x n/2 block grid keeps the players
+// of pairs k and k' in registers (advanced every step), forms both pairs'
+// rotations from the current copy of A itself (every owner of a pair forms
+// the same rotation from the same values), writes J^T A J for its block (rows
 // rotated by pair k, columns by pair k') into the other copy of A and rotates
-// rows k', k' + n/2 of V in pair k's columns.  With two copies of A each
-// phase ends in one barrier.  When l is odd the matrices are padded with a
-// zero row and column whose pair is never rotated.
+// rows k', k' + n/2 of V in pair k's columns: one barrier per rotation step.
+// When l is odd the matrices are padded with a zero row and column whose pair
+// is never rotated.
 // ---------------------------------------------------------------------------
 constexpr size_t kJacSmem = 3 * static_cast<size_t>(kLmax) * (kLmax + 1) * sizeof(float);
 struct EigArgs {
@@ -1244,36 +1252,37 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
   }
   // pair k plays (p, q) = (k or 0, n - 1 - k) at step 0; every step moves
   // each player but player 0 on by one place in 1 .. n - 1
-  __shared__ float4 rot4[kLmax / 2];
-  int pk = (tid == 0) ? 0 : tid, qk = n - 1 - tid;
   int bk[kJacBlocks], bk2[kJacBlocks];
+  int pa[kJacBlocks], qa[kJacBlocks], pb[kJacBlocks], qb[kJacBlocks];
 #pragma unroll
   for (int it = 0; it < kJacBlocks; ++it) {
     const int e = tid + nt * it;
     bk[it] = (e < npairs * npairs) ? e / npairs : -1;
     bk2[it] = (e < npairs * npairs) ? e % npairs : 0;
   }
+  auto advance = [&](int& p, int& q, int k) {
+    if (k != 0) p = (p == n - 1) ? 1 : p + 1;
+    q = (q == n - 1) ? 1 : q + 1;
+  };
   int sweep = 0;
   float off = frob2, prev = frob2;
   for (; sweep < a.max_sweeps; ++sweep) {
+#pragma unroll
+    for (int it = 0; it < kJacBlocks; ++it) {
+      const int k = bk[it] < 0 ? 0 : bk[it], k2 = bk2[it];
+      pa[it] = k; qa[it] = n - 1 - k;
+      pb[it] = k2; qb[it] = n - 1 - k2;
+    }
     for (int step = 0; step < n - 1; ++step) {
-      if (tid < npairs) {
-        const int i = min(pk, qk), j = max(pk, qk);
-        float c, s;
-        jac_rot(cur[i * ld + i], cur[j * ld + j], cur[i * ld + j], j >= l, c, s);
-        rot4[tid] = make_float4(c, s, __int_as_float(i), __int_as_float(j));
-        if (tid != 0) pk = (pk == n - 1) ? 1 : pk + 1;
-        qk = (qk == n - 1) ? 1 : qk + 1;
-      }
-      __syncthreads();
 #pragma unroll
       for (int it = 0; it < kJacBlocks; ++it) {
         const int k = bk[it], k2 = bk2[it];
         if (k >= 0) {
-          const float4 r1 = rot4[k], r2 = rot4[k2];
-          const int i = __float_as_int(r1.z), j = __float_as_int(r1.w);
-          const int i2 = __float_as_int(r2.z), j2 = __float_as_int(r2.w);
-          const float c = r1.x, s = r1.y, c2 = r2.x, s2 = r2.y;
+          const int i = min(pa[it], qa[it]), j = max(pa[it], qa[it]);
+          const int i2 = min(pb[it], qb[it]), j2 = max(pb[it], qb[it]);
+          float c, s, c2, s2;
+          jac_rot(cur[i * ld + i], cur[j * ld + j], cur[i * ld + j], j >= l, c, s);
+          jac_rot(cur[i2 * ld + i2], cur[j2 * ld + j2], cur[i2 * ld + j2], j2 >= l, c2, s2);
           const float* ri = cur + i * ld;
           const float* rj = cur + j * ld;
           const float a00 = ri[i2], a01 = ri[j2], a10 = rj[i2], a11 = rj[j2];
@@ -1292,6 +1301,8 @@ __global__ void __launch_bounds__(1024) k_jacobi(const __grid_constant__ EigArgs
             vr[i] = c * vi - s * vj;
             vr[j] = s * vi + c * vj;
           }
+          advance(pa[it], qa[it], k);
+          advance(pb[it], qb[it], k2);
         }
       }
       __syncthreads();
@@ -2156,7 +2167,7 @@ static cudaError_t launch_cholqr(const CholQRArgs& c, float* rfac, int batch, in
   switch (lp) {
 #define NP_CQ(N)                                                                                        \
   case N:                                                                                               \
-    k_chol_factor<N><<<batch, 256, 0, s>>>(c, rfac);                                                    \
+    k_chol_factor<N><<<batch, kCholThreads, 0, s>>>(c, rfac);                                                    \
     if (c.gram_out) {                                                                                   \
       const size_t sm = sizeof(float) * 256 * (N + 4);                                                  \
       static bool attr = false;                                                                         \
