@@ -163,6 +163,16 @@ CONFIGS: Dict[str, ParamSetConfig] = {
         grad_dist="normal", row_sigma=1.5, col_sigma=1.5, variants=("G", "L"),
         description="Qwen3 ~1.7B hidden matrices (28 layers, GQA k/v 2048x1024, MLP 6144), "
                     "bf16 grads N(0,1) x log-normal(1.5) row and column scales, bf16 weights"),
+    # the first two layers of the Qwen3 set: the same shapes, dtypes and value
+    # distributions at 1/14 of the size (100M elements, about 1 GB on the
+    # device, every per-step buffer still larger than L2), for kernel profiles
+    "qwen3_2layers": ParamSetConfig(
+        name="qwen3_2layers", matrices=_repeat(2, [MatrixSpec(2048, 2048, "q"), MatrixSpec(2048, 1024, "k"),
+                                                  MatrixSpec(2048, 1024, "v"), MatrixSpec(2048, 2048, "o"),
+                                                  MatrixSpec(2048, 6144, "gate"), MatrixSpec(2048, 6144, "up"),
+                                                  MatrixSpec(6144, 2048, "down")]),
+        g_dtype=BF16, w_dtype=BF16, grad_dist="normal", row_sigma=1.5, col_sigma=1.5, variants=("G", "L"),
+        description="two Qwen3 ~1.7B layers (the profiling case of the Qwen3 kernels)"),
 }
 
 
