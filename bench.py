@@ -398,12 +398,14 @@ def measure_variant(args, cfg, variant, host, dev):
     time.sleep(0.1)                     # let the sampler's first query land
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.nvtx.range_push("timed_" + variant)   # lets a profiler select the timed steps only
     ev0.record(stream)
     for _ in range(args.steps):
         opt.step(t, LR, W, G, M)
         t += 1
     ev1.record(stream)
     torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
     ms_total = ev0.elapsed_time(ev1)
     sampler.stop()
     counts = C.normpre_profile_read(h)  # launches of the timed region; resets the counters
@@ -515,12 +517,14 @@ def measure_muon(args, cfg, host):
         t += 1
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.nvtx.range_push("timed_muon")
     ev0.record(stream)
     for _ in range(args.steps):
         opt.step(t, LR, W, G, M)
         t += 1
     ev1.record(stream)
     torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
     ms = ev0.elapsed_time(ev1) / args.steps
     opt.status()
     opt.close()

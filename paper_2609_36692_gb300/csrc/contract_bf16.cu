@@ -41,20 +41,33 @@ __global__ void __launch_bounds__(256) k_vsplit_bf(const __grid_constant__ VSpli
   const int64_t k0 = static_cast<int64_t>(blockIdx.x) * 64;
   const int l = a.l;   // <= 64
   const float* v = a.v + b * a.v_bs + k0 * l;
-  const int64_t nvalid = (a.K - k0 < 64 ? a.K - k0 : 64) * l;   // contiguous floats of the block
-  for (int i = tid; i < 64 * l; i += 256) {
-    const int k = i / l, n = i - k * l;
-    tile[k][n] = i < nvalid ? v[i] : 0.f;
+  const int nvalid = static_cast<int>((a.K - k0 < 64 ? a.K - k0 : 64) * l);   // contiguous floats of the block
+  if ((l & 3) == 0 && (reinterpret_cast<uintptr_t>(v) & 15) == 0) {
+    for (int i4 = tid; i4 < 16 * l; i4 += 256) {          // 64 l / 4 float4s
+      const int i = 4 * i4;
+      const float4 x = i < nvalid ? __ldg(reinterpret_cast<const float4*>(v) + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int k = i / l, n = i - k * l;                   // l % 4 == 0: the 4 values share row k
+      tile[k][n] = x.x; tile[k][n + 1] = x.y; tile[k][n + 2] = x.z; tile[k][n + 3] = x.w;
+    }
+  } else {
+    for (int i = tid; i < 64 * l; i += 256) {
+      const int k = i / l, n = i - k * l;
+      tile[k][n] = i < nvalid ? v[i] : 0.f;
+    }
   }
   __syncthreads();
-  bf16* out = a.vb + b * a.vb_bs + k0;
-  for (int i = tid; i < a.np * 64; i += 256) {
-    const int n = i >> 6, k = i & 63;
-    const float x = n < l ? tile[k][n] : 0.f;
-    const bf16 hi = __float2bfloat16_rn(x);
-    const bf16 lo = __float2bfloat16_rn(x - __bfloat162float(hi));
-    out[static_cast<int64_t>(n) * a.kpad + k] = hi;
-    out[static_cast<int64_t>(a.np + n) * a.kpad + k] = lo;
+  // two K entries per thread: one 32-bit store of hi and one of lo
+  uint32_t* out = reinterpret_cast<uint32_t*>(a.vb + b * a.vb_bs + k0);
+  const int64_t rw = a.kpad / 2;                            // 32-bit words per row
+  for (int i = tid; i < a.np * 32; i += 256) {
+    const int n = i >> 5, k = 2 * (i & 31);
+    const float x0 = n < l ? tile[k][n] : 0.f, x1 = n < l ? tile[k + 1][n] : 0.f;
+    const bf16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+    const bf16 g0 = __float2bfloat16_rn(x0 - __bfloat162float(h0)), g1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
+    out[static_cast<int64_t>(n) * rw + (k >> 1)] =
+        static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
+    out[static_cast<int64_t>(a.np + n) * rw + (k >> 1)] =
+        static_cast<uint32_t>(__bfloat16_as_ushort(g0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(g1)) << 16);
   }
 }
 

@@ -710,6 +710,25 @@ __global__ void k_split_reduce(const __grid_constant__ SplitReduceArgs a) {
 // Split Gram sums: part[b][s] = sum over the rows of chunk s of y_i y_i^T,
 // fp32 over kGramRows rows.  Y is [N x l].
 // ---------------------------------------------------------------------------
+// The 4 x 4 tiles on or above the diagonal of an l4 x l4 tile grid, numbered
+// row by row: tile t -> (tp, tq) with tp <= tq, and back.  A Gram sum is
+// symmetric entry for entry (the product y_ip y_iq is the same float for (p, q)
+// and (q, p), added in the same order), so the kernels below sum only these
+// tiles and mirror them.
+__device__ __forceinline__ void upper_tile(int t, int l4, int& tp, int& tq) {
+  int r = 0;
+  while (t >= l4 - r) { t -= l4 - r; ++r; }
+  tp = r;
+  tq = r + t;
+}
+__device__ __forceinline__ int upper_index(int tp, int tq, int l4) { return tp * l4 - tp * (tp - 1) / 2 + (tq - tp); }
+// entry (p, q) of the l x l sum as (upper tile, position in it)
+__device__ __forceinline__ void upper_entry(int p, int q, int l4, int& tile, int& k) {
+  const int tp = p >> 2, tq = q >> 2;
+  if (tp <= tq) { tile = upper_index(tp, tq, l4); k = 4 * (p & 3) + (q & 3); }
+  else { tile = upper_index(tq, tp, l4); k = 4 * (q & 3) + (p & 3); }
+}
+
 struct GramArgs {
   const float* y; int64_t y_bs;
   float* part; int64_t part_bs;   // [nsplit][l][l] per matrix
@@ -730,16 +749,24 @@ __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramA
   const int64_t i0 = static_cast<int64_t>(s) * kGramRows;
   const int64_t nval = (a.n - i0 < kGramRows ? a.n - i0 : static_cast<int64_t>(kGramRows)) * l;   // valid floats of the chunk
   const float* y = a.y + b * a.y_bs + i0 * l;    // the chunk's rows are contiguous
-  for (int e = tid; e < kGramRows * l; e += blockDim.x) {
-    const int i = e / l, j = e - i * l;
-    ys[i * LD + j] = e < nval ? __ldg(y + e) : 0.f;
+  if ((l & 3) == 0 && (reinterpret_cast<uintptr_t>(y) & 15) == 0) {
+    for (int e4 = tid; e4 < kGramRows * l / 4; e4 += blockDim.x) {
+      const int e = 4 * e4, i = e / l, j = e - i * l;   // l % 4 == 0: one row per float4
+      const float4 v = e < nval ? __ldg(reinterpret_cast<const float4*>(y) + e4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      *reinterpret_cast<float4*>(ys + i * LD + j) = v;
+    }
+  } else {
+    for (int e = tid; e < kGramRows * l; e += blockDim.x) {
+      const int i = e / l, j = e - i * l;
+      ys[i * LD + j] = e < nval ? __ldg(y + e) : 0.f;
+    }
   }
   for (int e = tid; e < kGramRows * (lp - l); e += blockDim.x) {
     const int i = e / (lp - l), j = l + (e - i * (lp - l));
     ys[i * LD + j] = 0.f;
   }
   __syncthreads();
-  const int tiles = l4 * l4;
+  const int tiles = l4 * (l4 + 1) / 2;           // on or above the diagonal
   const int groups = tiles <= 64 ? 4 : (tiles <= 128 ? 2 : 1);
   const int rows_g = kGramRows / groups;
   float* out = a.part + b * a.part_bs + static_cast<int64_t>(s) * l * l;
@@ -747,7 +774,9 @@ __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramA
   int my_tile = -1, my_group = 0;
   for (int t = tid; t < tiles * groups; t += blockDim.x) {
     const int tile = t % tiles, g = t / tiles;
-    const int p0 = 4 * (tile / l4), q0 = 4 * (tile % l4);
+    int tp, tq;
+    upper_tile(tile, l4, tp, tq);
+    const int p0 = 4 * tp, q0 = 4 * tq;
 #pragma unroll
     for (int r = 0; r < 4; ++r)
 #pragma unroll
@@ -768,7 +797,10 @@ __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramA
       for (int r = 0; r < 4; ++r)
 #pragma unroll
         for (int c = 0; c < 4; ++c)
-          if (p0 + r < l && q0 + c < l) out[(p0 + r) * l + q0 + c] = acc[r][c];
+          if (p0 + r < l && q0 + c < l) {
+            out[(p0 + r) * l + q0 + c] = acc[r][c];
+            out[(q0 + c) * l + p0 + r] = acc[r][c];
+          }
     } else {
       my_tile = tile;     // one (tile, group) per thread when groups > 1
       my_group = g;
@@ -785,7 +817,8 @@ __global__ void __launch_bounds__(256) k_gram_part(const __grid_constant__ GramA
   __syncthreads();
   for (int e = tid; e < l * l; e += blockDim.x) {
     const int p = e / l, q = e - p * l;
-    const int tile = (p >> 2) * l4 + (q >> 2), k = 4 * (p & 3) + (q & 3);
+    int tile, k;
+    upper_entry(p, q, l4, tile, k);
     float v = 0.f;
     for (int g = 0; g < groups; ++g) v += ys[(g * tiles + tile) * 16 + k];
     out[e] = v;
@@ -1071,7 +1104,7 @@ __global__ void __launch_bounds__(256) k_chol_solve_gram(const __grid_constant__
   for (int j = 0; j < LP; j += 4)
     *reinterpret_cast<float4*>(X + tid * LDX + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
   __syncthreads();
-  constexpr int L4 = LP / 4, TILES = L4 * L4;
+  constexpr int L4 = LP / 4, TILES = L4 * (L4 + 1) / 2;   // tiles on or above the diagonal
   constexpr int GROUPS = TILES <= 64 ? 4 : (TILES <= 128 ? 2 : 1);
   constexpr int ROWS_G = 256 / GROUPS;
   float* out = a.gram_out + b * a.gram_bs + static_cast<int64_t>(blockIdx.x) * l * l;
@@ -1079,7 +1112,9 @@ __global__ void __launch_bounds__(256) k_chol_solve_gram(const __grid_constant__
   int my_tile = -1, my_group = 0;
   for (int t = tid; t < TILES * GROUPS; t += 256) {
     const int tile = t % TILES, g = t / TILES;
-    const int p0 = 4 * (tile / L4), q0 = 4 * (tile % L4);
+    int tp, tq;
+    upper_tile(tile, L4, tp, tq);
+    const int p0 = 4 * tp, q0 = 4 * tq;
 #pragma unroll
     for (int r = 0; r < 4; ++r)
 #pragma unroll
@@ -1100,7 +1135,10 @@ __global__ void __launch_bounds__(256) k_chol_solve_gram(const __grid_constant__
       for (int r = 0; r < 4; ++r)
 #pragma unroll
         for (int c = 0; c < 4; ++c)
-          if (p0 + r < l && q0 + c < l) out[(p0 + r) * l + q0 + c] = acc[r][c];
+          if (p0 + r < l && q0 + c < l) {
+            out[(p0 + r) * l + q0 + c] = acc[r][c];
+            out[(q0 + c) * l + p0 + r] = acc[r][c];
+          }
     } else {
       my_tile = tile;
       my_group = g;
@@ -1117,7 +1155,8 @@ __global__ void __launch_bounds__(256) k_chol_solve_gram(const __grid_constant__
   __syncthreads();
   for (int e = tid; e < l * l; e += 256) {
     const int p = e / l, qq = e - p * l;
-    const int tile = (p >> 2) * L4 + (qq >> 2), k = 4 * (p & 3) + (qq & 3);
+    int tile, k;
+    upper_entry(p, qq, L4, tile, k);
     float v = 0.f;
     for (int g = 0; g < GROUPS; ++g) v += X[(g * TILES + tile) * 16 + k];
     out[e] = v;
@@ -2500,17 +2539,24 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       NP_CHECK();
     }
   }
-  // QK = Q K  [m_a x l]
+  // K is symmetric (its entries are sums of products taken in the same order
+  // for (r, s) and (s, r)), so T_a = Psi_a + (Q K) B = Psi_a + Q (B^T K)^T: the
+  // l x l product is applied to the shorter of the two panels, Q [m_a x l] or
+  // B^T [n_a x l], into g.qk
+  const bool k_on_b = n_a < m_a;
   {
     RowMulArgs rm;
-    rm.y = g.q; rm.y_bs = vbs; rm.s = g.kmat; rm.s_bs = sq;
-    rm.out = g.qk; rm.out_bs = vbs; rm.n = m_a; rm.l = l;
-    k_rowmul<<<dim3(static_cast<unsigned>(cdiv(m_a * ((l + 7) / 8), 256)), B), 256, 0, s>>>(rm);
+    rm.y = k_on_b ? g.bt : g.q; rm.y_bs = vbs; rm.s = g.kmat; rm.s_bs = sq;
+    rm.out = g.qk; rm.out_bs = vbs; rm.n = k_on_b ? n_a : m_a; rm.l = l;
+    k_rowmul<<<dim3(static_cast<unsigned>(cdiv(rm.n * ((l + 7) / 8), 256)), B), 256, 0, s>>>(rm);
     NP_CHECK();
   }
   prof->end(kProfEig, s, (p.exact ? 1 : 3) + n_fold);
-  // T_s = Psi + Lm R^T with (Lm, R) = (QK, B^T) row-active or (B^T, QK) column-active,
-  // in launches of at most kMaxBatch matrices (W pointers travel as kernel arguments)
+  // T_s = Psi + Lm R^T with (Lm, R) = (QK, B^T) row-active or (B^T, QK)
+  // column-active; (Q, B^T K) and (B^T K, Q) when K went on B^T.  In launches
+  // of at most kMaxBatch matrices (W pointers travel as kernel arguments)
+  const float* u_a = k_on_b ? g.q : g.qk;    // the m_a-row factor
+  const float* u_b = k_on_b ? g.qk : g.bt;   // the n_a-row factor
   prof->begin(kProfApplyL, s);
   int n_apply = 0;
   const bool vec = (g.cols % 4 == 0) && (g.ld % 4 == 0);
@@ -2521,8 +2567,8 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     la.psi = g.psi_bf16 ? static_cast<const void*>(reinterpret_cast<const bf16*>(g.psi) + c0 * psi_bs)
                         : static_cast<const void*>(g.psi + c0 * psi_bs);
     la.psi_bs = psi_bs; la.psi_ld = g.ld; la.psi_bf16 = g.psi_bf16 ? 1 : 0;
-    la.lm = (rows_active ? g.qk : g.bt) + c0 * vbs; la.lm_bs = vbs;
-    la.rm = (rows_active ? g.bt : g.qk) + c0 * vbs; la.rm_bs = vbs;
+    la.lm = (rows_active ? u_a : u_b) + c0 * vbs; la.lm_bs = vbs;
+    la.rm = (rows_active ? u_b : u_a) + c0 * vbs; la.rm_bs = vbs;
     la.stats = g.stats + c0 * 8; la.stats_bs = 8;
     for (int i = 0; i < nb; ++i) la.W[i] = W[c0 + i];
     la.rows = g.rows; la.cols = g.cols; la.l = l;
