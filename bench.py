@@ -54,7 +54,12 @@ L2_BYTES = 129e6                                    # GB300 L2
 # absent until a capture of the current kernel exists (profiles/ keeps the
 # summaries).
 NCU_TRAFFIC_PER_LAUNCH = {
-    ("gpt2_small_G", "G"): 208.1e6,   # mean of 15 launches: Gram, poly and update of five NS iterations
+    # dram__bytes_read.sum + dram__bytes_write.sum per launch of the roofline
+    # kernel class, from one ncu capture of the timed steps (profiles/launches_*.md)
+    ("gpt2_small_G", "G"): 207.9e6,      # mean of 45 launches: Gram, poly and update of five NS iterations, 3 steps
+    ("qwen3_1p7b", "G"): 4519e6,         # the same on the Qwen3 set
+    ("qwen3_1p7b", "L", "normalize"): 1.687e9,   # a row-active and a column-active step over their 28 launches
+    ("gpt2_small_L", "L", "contract"): 56.0e6,   # 78 launches: contractions and split-K reductions, 3 steps
 }
 
 
