@@ -1881,38 +1881,9 @@ static size_t abf_smem(int natoms) {
          static_cast<size_t>(abf_stages<TW>()) * abf_stage_bytes<TW>() + 512;
 }
 
-// rows [r0, r0 + R) of a panel rounded to TF32 into one swizzled K-major tile
-template <int R>
-__device__ __forceinline__ void abf_round_rows(const float* panel, int64_t r0, int64_t nrows, int l, uint8_t* hi,
-                                               int atom_bytes, int ptid) {
-  constexpr int NT = 64, B = 8;
-  const int l4 = l >> 2;
-  const int n = R * l4;
-  const float* src = panel + r0 * l;
-  const int64_t valid = (nrows - r0) * l4;
-  for (int base = ptid; base < n; base += B * NT) {
-    float4 x[B];
-#pragma unroll
-    for (int k = 0; k < B; ++k) {
-      const int idx = base + k * NT;
-      x[k] = (idx < n && idx < valid) ? __ldg(reinterpret_cast<const float4*>(src) + idx)
-                                      : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-#pragma unroll
-    for (int k = 0; k < B; ++k) {
-      const int idx = base + k * NT;
-      if (idx < n) {
-        const int r = idx / l4, c4 = idx - r * l4;
-        const int kk = 4 * c4;
-        const uint32_t off = static_cast<uint32_t>((kk >> 5) * atom_bytes) + sw128(r, (kk & 31) >> 2);
-        *reinterpret_cast<float4*>(hi + off) = x[k];   // the MMA reads fp32 storage at TF32 precision
-      }
-    }
-  }
-}
-
 struct ApplyBfArgs {
   CUtensorMap psi_map;             // bf16 Psi {cols, rows, batch}, box 64 x 32
+  CUtensorMap lm_map, rm_map;      // fp32 panels {l, rows / cols, launch batch}, boxes 32 x 256 / 32 x 128
   CUtensorMap w_map[kMaxBatch];    // W of each matrix {cols, rows}, box (128 bytes) x 32
   int psi_b0;                      // batch coordinate of the launch's first matrix in psi_map
 };
@@ -1936,6 +1907,7 @@ __global__ void __launch_bounds__(kAbfThreads, 1) k_apply_bf(const __grid_consta
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sempty + S);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [S] last parity + 1
+  uint32_t op_issued = 0;                                           // operand copies: last parity + 1 (thread 0)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t rt = (a.rows + kAtcRows - 1) / kAtcRows, ct = (a.cols + kAtcCols - 1) / kAtcCols;
@@ -1949,7 +1921,7 @@ __global__ void __launch_bounds__(kAbfThreads, 1) k_apply_bf(const __grid_consta
     j0 = (rem % ct) * kAtcCols;
   };
   if (threadIdx.x == 0) {
-    tc::mbar_init(opfull, kAtcProd);
+    tc::mbar_init(opfull, 1);
     tc::mbar_init(opfree, 1);
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&tfull[i], 1);
@@ -1981,24 +1953,37 @@ __global__ void __launch_bounds__(kAbfThreads, 1) k_apply_bf(const __grid_consta
   constexpr int WBOX = 128 / static_cast<int>(sizeof(TW));   // W columns per 128-byte box row
 
   if (warp < kAtcProd) {
-    // ---------------- operand rounding ----------------
-    const int ptid = threadIdx.x;
+    // ---------------- operand tiles by TMA (warp 0; warp 1 has no role) ----------------
+    // The MMA reads fp32 storage at TF32 precision, so the panels' 32-wide K
+    // slabs are copied as they are: a box of 32 floats x R rows with the
+    // 128-byte swizzle is exactly one K-major atom, K past l reads zero
     bool ok = true;
-    int64_t b_key = -1;
-    uint32_t it = 0;
-    for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
-      int b;
-      int64_t i0, j0;
-      unit_of(u, b, i0, j0);
-      ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(opfree, (it & 1) ^ 1u, abort_flag));
-      if (!ok) break;
-      const int64_t key = static_cast<int64_t>(b) * rt + i0 / kAtcRows;
-      if (key != b_key) abf_round_rows<kAtcRows>(a.lm + b * a.lm_bs, i0, a.rows, l, b_hi, kAtcAtomB, ptid);
-      b_key = key;
-      abf_round_rows<kAtcCols>(a.rm + b * a.rm_bs, j0, a.cols, l, a_hi, kAtcAtomA, ptid);
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(opfull);
+    if (warp == 0) {
+      if (lane == 0) {
+        tc::prefetch_map(&m.lm_map);
+        tc::prefetch_map(&m.rm_map);
+      }
+      int64_t b_key = -1;
+      uint32_t it = 0;
+      for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
+        int b;
+        int64_t i0, j0;
+        unit_of(u, b, i0, j0);
+        ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(opfree, (it & 1) ^ 1u, abort_flag));
+        if (!ok) break;
+        const int64_t key = static_cast<int64_t>(b) * rt + i0 / kAtcRows;
+        const bool new_b = key != b_key;
+        b_key = key;
+        if (lane == 0) {
+          tc::mbar_expect_tx(opfull, static_cast<uint32_t>(natoms * (kAtcAtomA + (new_b ? kAtcAtomB : 0))));
+          op_issued = (it & 1) + 1;
+          for (int at = 0; at < natoms; ++at) {
+            tc::tma_load_3d(a_hi + at * kAtcAtomA, &m.rm_map, opfull, 32 * at, static_cast<int>(j0), b);
+            if (new_b) tc::tma_load_3d(b_hi + at * kAtcAtomB, &m.lm_map, opfull, 32 * at, static_cast<int>(i0), b);
+          }
+        }
+        __syncwarp();
+      }
     }
     if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
   } else if (warp == kAtcProd) {
@@ -2156,10 +2141,11 @@ __global__ void __launch_bounds__(kAbfThreads, 1) k_apply_bf(const __grid_consta
   }
   __syncthreads();
   if (threadIdx.x == 0 && *abort_flag) {
-    // let every bulk copy still in flight land before the CTA exits
+    // let every TMA copy still in flight land before the CTA exits
     volatile int never = 0;
     for (int i = 0; i < S; ++i)
       if (issued[i]) tc::mbar_wait(&sfull[i], issued[i] - 1, &never);
+    if (op_issued) tc::mbar_wait(opfull, op_issued - 1, &never);
   }
   __syncthreads();
   if (warp == kAtcProd) {
@@ -2595,6 +2581,14 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       for (int i = 0; i < nb && use_bf; ++i)
         use_bf = driver_encode_tiled(&ma.w_map[i], g.w_dtype ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
                                      2, la.W[i], wd, ws, wbox, nullptr);
+      // the fp32 panels (l % 4 == 0 and 16-byte matrix strides: vec_panels)
+      const uint64_t pst[2] = {static_cast<uint64_t>(l) * 4, static_cast<uint64_t>(vbs) * 4};
+      const uint64_t ld_[3] = {static_cast<uint64_t>(l), static_cast<uint64_t>(g.rows), static_cast<uint64_t>(nb)};
+      const uint64_t rd_[3] = {static_cast<uint64_t>(l), static_cast<uint64_t>(g.cols), static_cast<uint64_t>(nb)};
+      const uint32_t lbox[3] = {32, static_cast<uint32_t>(kAtcRows), 1}, rbox[3] = {32, static_cast<uint32_t>(kAtcCols), 1};
+      use_bf = use_bf &&
+               driver_encode_tiled(&ma.lm_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(la.lm), ld_, pst, lbox, nullptr) &&
+               driver_encode_tiled(&ma.rm_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(la.rm), rd_, pst, rbox, nullptr);
     }
     if (use_bf) {
       const int natoms = (l + 31) / 32;
