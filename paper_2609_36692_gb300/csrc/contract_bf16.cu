@@ -26,8 +26,9 @@ namespace normpre {
 // ---------------------------------------------------------------------------
 // V [K x l] fp32 (row stride l) -> vb [2 np][kpad] bf16: row n < np holds
 // hi(V[:, n]), row np + n holds lo(V[:, n]); columns n >= l and K rows >= K
-// are zero.  One CTA per 64 K rows of a matrix, the 64 x l block staged in
-// shared memory so that both the read and the transposed write are coalesced.
+// are zero.  One CTA per 256 K rows of a matrix, in four 64-row blocks each
+// staged in shared memory so that both the read and the transposed write are
+// coalesced; a thread writes eight K entries of one row as one 16-byte store.
 // ---------------------------------------------------------------------------
 struct VSplitArgs {
   const float* v; int64_t v_bs;
@@ -35,39 +36,48 @@ struct VSplitArgs {
   int l, np;
   bf16* vb; int64_t vb_bs, kpad;
 };
+constexpr int kVsRows = 256;
 __global__ void __launch_bounds__(256) k_vsplit_bf(const __grid_constant__ VSplitArgs a) {
   __shared__ float tile[64][64 + 1];
   const int b = blockIdx.y, tid = threadIdx.x;
-  const int64_t k0 = static_cast<int64_t>(blockIdx.x) * 64;
   const int l = a.l;   // <= 64
-  const float* v = a.v + b * a.v_bs + k0 * l;
-  const int nvalid = static_cast<int>((a.K - k0 < 64 ? a.K - k0 : 64) * l);   // contiguous floats of the block
-  if ((l & 3) == 0 && (reinterpret_cast<uintptr_t>(v) & 15) == 0) {
-    for (int i4 = tid; i4 < 16 * l; i4 += 256) {          // 64 l / 4 float4s
-      const int i = 4 * i4;
-      const float4 x = i < nvalid ? __ldg(reinterpret_cast<const float4*>(v) + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
-      const int k = i / l, n = i - k * l;                   // l % 4 == 0: the 4 values share row k
-      tile[k][n] = x.x; tile[k][n + 1] = x.y; tile[k][n + 2] = x.z; tile[k][n + 3] = x.w;
+  for (int blk = 0; blk < kVsRows / 64; ++blk) {
+    const int64_t k0 = static_cast<int64_t>(blockIdx.x) * kVsRows + 64 * blk;
+    if (k0 >= a.kpad) break;
+    const float* v = a.v + b * a.v_bs + k0 * l;
+    const int64_t left = a.K - k0;
+    const int nvalid = left <= 0 ? 0 : static_cast<int>((left < 64 ? left : 64) * l);   // contiguous floats
+    if (blk) __syncthreads();          // the previous block's tile is read
+    if ((l & 3) == 0 && (reinterpret_cast<uintptr_t>(v) & 15) == 0) {
+      for (int i4 = tid; i4 < 16 * l; i4 += 256) {          // 64 l / 4 float4s
+        const int i = 4 * i4;
+        const float4 x = i < nvalid ? __ldg(reinterpret_cast<const float4*>(v) + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
+        const int k = i / l, n = i - k * l;                   // l % 4 == 0: the 4 values share row k
+        tile[k][n] = x.x; tile[k][n + 1] = x.y; tile[k][n + 2] = x.z; tile[k][n + 3] = x.w;
+      }
+    } else {
+      for (int i = tid; i < 64 * l; i += 256) {
+        const int k = i / l, n = i - k * l;
+        tile[k][n] = i < nvalid ? v[i] : 0.f;
+      }
     }
-  } else {
-    for (int i = tid; i < 64 * l; i += 256) {
-      const int k = i / l, n = i - k * l;
-      tile[k][n] = i < nvalid ? v[i] : 0.f;
+    __syncthreads();
+    // thread: row n = item / 8, K entries 8 (item % 8) .. + 7 of the block
+    bf16* out = a.vb + b * a.vb_bs + k0;
+    for (int item = tid; item < a.np * 8; item += 256) {
+      const int n = item >> 3, kk = 8 * (item & 7);
+      uint32_t hw[4], lw[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float x0 = n < l ? tile[kk + 2 * e][n] : 0.f, x1 = n < l ? tile[kk + 2 * e + 1][n] : 0.f;
+        const bf16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+        const bf16 g0 = __float2bfloat16_rn(x0 - __bfloat162float(h0)), g1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
+        hw[e] = static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
+        lw[e] = static_cast<uint32_t>(__bfloat16_as_ushort(g0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(g1)) << 16);
+      }
+      *reinterpret_cast<uint4*>(out + static_cast<int64_t>(n) * a.kpad + kk) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+      *reinterpret_cast<uint4*>(out + static_cast<int64_t>(a.np + n) * a.kpad + kk) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
     }
-  }
-  __syncthreads();
-  // two K entries per thread: one 32-bit store of hi and one of lo
-  uint32_t* out = reinterpret_cast<uint32_t*>(a.vb + b * a.vb_bs + k0);
-  const int64_t rw = a.kpad / 2;                            // 32-bit words per row
-  for (int i = tid; i < a.np * 32; i += 256) {
-    const int n = i >> 5, k = 2 * (i & 31);
-    const float x0 = n < l ? tile[k][n] : 0.f, x1 = n < l ? tile[k + 1][n] : 0.f;
-    const bf16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
-    const bf16 g0 = __float2bfloat16_rn(x0 - __bfloat162float(h0)), g1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
-    out[static_cast<int64_t>(n) * rw + (k >> 1)] =
-        static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
-    out[static_cast<int64_t>(a.np + n) * rw + (k >> 1)] =
-        static_cast<uint32_t>(__bfloat16_as_ushort(g0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(g1)) << 16);
   }
 }
 
@@ -305,7 +315,7 @@ cudaError_t launch_contract_bf16(const ContractBf16Launch& c, cudaStream_t s) {
   VSplitArgs vs;
   vs.v = c.v; vs.v_bs = c.v_bs; vs.K = c.K; vs.l = c.l; vs.np = np;
   vs.vb = static_cast<bf16*>(c.vb); vs.vb_bs = c.vb_bs; vs.kpad = kpad;
-  k_vsplit_bf<<<dim3(static_cast<unsigned>(kpad / 64), static_cast<unsigned>(c.batch)), 256, 0, s>>>(vs);
+  k_vsplit_bf<<<dim3(static_cast<unsigned>(cdiv(kpad, kVsRows)), static_cast<unsigned>(c.batch)), 256, 0, s>>>(vs);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   ContractBfArgs a;
