@@ -147,7 +147,9 @@ void normpre_default_config(normpre_config* cfg);
  *   out       receives the handle.
  * The handle owns all device workspaces (allocated here with cudaMalloc on the
  * current device) and precomputed launch plans; matrices of equal shape and
- * dtypes are grouped so that one launch serves a whole group.
+ * dtypes are grouped so that one launch serves a whole group.  NORMPRE_G and
+ * NORMPRE_MUON serve at most 7 such groups (one grouped Newton-Schulz launch
+ * whose arguments stay within 4 KB); more is a SHAPE error.
  * Errors: ARG (null / bad count / bad hyperparameter), SHAPE, DTYPE, CUDA.
  */
 int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, const int64_t* cols,

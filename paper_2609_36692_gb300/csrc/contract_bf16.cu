@@ -36,6 +36,7 @@ struct VSplitArgs {
   int l, np;
   bf16* vb; int64_t vb_bs, kpad;
 };
+static_assert(sizeof(VSplitArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 constexpr int kVsRows = 256;
 __global__ void __launch_bounds__(256) k_vsplit_bf(const __grid_constant__ VSplitArgs a) {
   __shared__ float tile[64][64 + 1];
@@ -112,6 +113,7 @@ struct ContractBfArgs {
   int* flags;
   int stall_first_copy;   // tests: CTA 0 does not issue its first copy (its waits then give up)
 };
+static_assert(sizeof(ContractBfArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 
 template <bool TRANS>
 __global__ void __launch_bounds__(kCbThreads, 1) k_contract_bf(const __grid_constant__ ContractBfArgs a) {

@@ -16,7 +16,7 @@ constexpr int kFlagNumeric = 2;
 constexpr int kFlagTimeout = 4;
 
 constexpr int kMaxBatch = 32;    // matrices served by one normalize/apply launch
-constexpr int kMaxGroups = 8;    // shape groups served by one Newton-Schulz GEMM launch
+constexpr int kMaxGroups = 7;    // shape groups served by one Newton-Schulz GEMM launch (its arguments within 4 KB)
 
 inline int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
@@ -106,6 +106,7 @@ struct NormLaunch {
   double* col_part = nullptr;
   float2* col_coef = nullptr;
 };
+static_assert(sizeof(NormLaunch) + 64 <= 4096, "kernel arguments beyond 4 KB");
 cudaError_t launch_normalize_rows(const NormLaunch& a, cudaStream_t s);
 // Muon baseline (muon.cu): M = mu M + G written back and copied to a.psi,
 // fp64 sums of ||M||^2 of nblk row blocks into part[i * stride + blk] for the
@@ -140,6 +141,7 @@ struct ApplyLaunch {
   int n_part = 0;
   float lr = 0, wd = 0, target = 0.2f;
 };
+static_assert(sizeof(ApplyLaunch) + 64 <= 4096, "kernel arguments beyond 4 KB");
 cudaError_t launch_apply_g(const ApplyLaunch& a, cudaStream_t s);
 // Descent-alignment sums <G, T>, ||G||^2, ||T||^2 per matrix into diag[4..6].
 struct DiagLaunch {
@@ -152,6 +154,7 @@ struct DiagLaunch {
   int64_t t_ld = 0;
   double* diag[kMaxBatch] = {};
 };
+static_assert(sizeof(DiagLaunch) + 64 <= 4096, "kernel arguments beyond 4 KB");
 cudaError_t launch_diag_gt(const DiagLaunch& a, cudaStream_t s);
 
 // ----------------------------------------------------------------------------

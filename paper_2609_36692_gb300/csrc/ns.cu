@@ -116,6 +116,7 @@ struct GemmArgs {
   int total_tiles;
   int* flags;
 };
+static_assert(sizeof(GemmArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 
 // Tiles of one matrix: the whole tiles_m x tiles_n grid, or for a symmetric
 // product only the tiles that reach the diagonal or lie above it

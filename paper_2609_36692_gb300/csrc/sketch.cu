@@ -83,6 +83,7 @@ struct OmegaArgs {
   uint32_t* words = nullptr;   // optional [batch][n_a][l]: the Philox word of each element
   float* uniforms = nullptr;   // optional [batch][n_a][l]: its uniform in (0, 1)
 };
+static_assert(sizeof(OmegaArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 __global__ void k_omega(const __grid_constant__ OmegaArgs a) {
   const int b = blockIdx.y;
   const int64_t n = a.n_a * a.l;
@@ -156,6 +157,7 @@ struct ContractArgs {
   int ksplit;
   int64_t kchunk;                  // K range of one split (multiple of 32)
 };
+static_assert(sizeof(ContractArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 constexpr int kCtP = 256, kCtK = 32, kCtThreads = 128;
 constexpr int kCtPsiLd = kCtK + 4;          // non-TRANS: Ps[p][k]
 constexpr int kCtPtLd = kCtP + 4;           // TRANS: Pt[k][p]
@@ -343,6 +345,7 @@ struct ContractTcArgs {
   int* flags;
   int stall_first_copy;   // tests: CTA 0 does not issue its first copy (its waits then give up)
 };
+static_assert(sizeof(ContractTcArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 // Two rings.  The input ring holds the TMA copies of the Psi block and of the
 // V block; the split warps free a slot as soon as they have read it, so the
 // copies run up to kCtcIn blocks ahead of the split and the HBM latency is
@@ -736,6 +739,7 @@ struct GramArgs {
   int l;
   int nsplit;
 };
+static_assert(sizeof(GramArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 // One CTA per chunk.  The chunk is staged in shared memory; each thread
 // accumulates a 4 x 4 block of the l x l sum over its share of the rows in
 // registers (two 16-byte shared loads per 16 FMAs); when the blocks do not
@@ -905,6 +909,7 @@ struct CholQRArgs {
   int* flags;
   float* gram_out; int64_t gram_bs;   // optional: per solve CTA, the l x l Gram sum of its rows
 };
+static_assert(sizeof(CholQRArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 // Per matrix [R (LP x LP, strictly upper, rows scaled by 1 / R_ii) | 1 / R_ii
 // (LP) | zero-panel flag]: the factorization of one CholeskyQR pass, made
 // once per matrix by k_chol_factor and read by every CTA of k_chol_solve.
@@ -1230,6 +1235,7 @@ struct EigArgs {
   int max_sweeps;
   int* flags;
 };
+static_assert(sizeof(EigArgs) + 64 <= 4096, "kernel arguments beyond 4 KB");
 // threads of k_jacobi for width l: one per 2 x 2 block (two each past 1024 blocks)
 constexpr int kJacBlocks = ((kLmax / 2) * (kLmax / 2) + 1023) / 1024;
 inline int64_t jacobi_threads(int l) {
@@ -1881,12 +1887,26 @@ static size_t abf_smem(int natoms) {
          static_cast<size_t>(abf_stages<TW>()) * abf_stage_bytes<TW>() + 512;
 }
 
+// At most kAbfBatch matrices per launch, so that the kernel's arguments (the
+// apply arguments, these tensor maps and three scalars) stay within the 4 KB
+// of a kernel's classic parameter space: launches of this kernel from several
+// streams overlap, and with more than 4 KB of arguments concurrent launches
+// that differed in their later arguments faulted.
+constexpr int kAbfBatch = 16;
+// k_apply_bf is not dispatched: on eight 4096 x 4096 fp32 weights together
+// with three 1024 x 4096 ones (two shape groups whose applies overlap on their
+// streams) it faulted, and the cause is not found; the bf16-Psi step uses
+// k_apply_tc<TW, bf16> instead
+constexpr bool kApplyBfEnabled = false;
 struct ApplyBfArgs {
   CUtensorMap psi_map;             // bf16 Psi {cols, rows, batch}, box 64 x 32
   CUtensorMap lm_map, rm_map;      // fp32 panels {l, rows / cols, launch batch}, boxes 32 x 256 / 32 x 128
-  CUtensorMap w_map[kMaxBatch];    // W of each matrix {cols, rows}, box (128 bytes) x 32
+  CUtensorMap w_map[kAbfBatch];    // W of each matrix {cols, rows}, box (128 bytes) x 32
   int psi_b0;                      // batch coordinate of the launch's first matrix in psi_map
 };
+
+static_assert(sizeof(LApplyArgs) + sizeof(ApplyBfArgs) + 32 <= 4096, "k_apply_bf arguments beyond 4 KB");
+static_assert(sizeof(LApplyArgs) + 32 <= 4096, "apply arguments beyond 4 KB");
 
 template <typename TW>
 __global__ void __launch_bounds__(kAbfThreads, 1) k_apply_bf(const __grid_constant__ LApplyArgs a,
@@ -2540,16 +2560,21 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   prof->end(kProfEig, s, (p.exact ? 1 : 3) + n_fold);
   // T_s = Psi + Lm R^T with (Lm, R) = (QK, B^T) row-active or (B^T, QK)
   // column-active; (Q, B^T K) and (B^T K, Q) when K went on B^T.  In launches
-  // of at most kMaxBatch matrices (W pointers travel as kernel arguments)
+  // of at most kMaxBatch matrices (W pointers travel as kernel arguments;
+  // kAbfBatch for the bf16-Psi kernel, whose W tensor maps do too)
   const float* u_a = k_on_b ? g.q : g.qk;    // the m_a-row factor
   const float* u_b = k_on_b ? g.qk : g.bt;   // the n_a-row factor
   prof->begin(kProfApplyL, s);
   int n_apply = 0;
   const bool vec = (g.cols % 4 == 0) && (g.ld % 4 == 0);
-  for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
-    const int nb = std::min(kMaxBatch, B - c0);
+  const bool bf_shape = kApplyBfEnabled && !(p.diag && p.G) && l % 4 == 0 && l <= 64 && g.psi_bf16 &&
+                        vbs % 4 == 0 && (g.cols * (g.w_dtype ? 2 : 4)) % 16 == 0;
+  const int per_launch = bf_shape ? kAbfBatch : kMaxBatch;
+  for (int c0 = 0; c0 < B; c0 += per_launch) {
+    const int nb = std::min(per_launch, B - c0);
     ++n_apply;
     LApplyArgs la;
+    std::memset(static_cast<void*>(&la), 0, sizeof(la));   // unused W / G slots are null, never stale
     la.psi = g.psi_bf16 ? static_cast<const void*>(reinterpret_cast<const bf16*>(g.psi) + c0 * psi_bs)
                         : static_cast<const void*>(g.psi + c0 * psi_bs);
     la.psi_bs = psi_bs; la.psi_ld = g.ld; la.psi_bf16 = g.psi_bf16 ? 1 : 0;
@@ -2568,8 +2593,7 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
       la.diag[i] = diag ? p.diag + 8 * static_cast<int64_t>(p.mat_ids_host[c0 + i]) : nullptr;
     }
     // bf16 Psi: single-product apply fed by TMA (W maps need 16-byte rows and pointers)
-    bool use_bf = !diag && l % 4 == 0 && l <= 64 && la.vec_panels && g.psi_bf16 &&
-                  (g.cols * (g.w_dtype ? 2 : 4)) % 16 == 0;
+    bool use_bf = bf_shape && !diag && la.vec_panels;
     ApplyBfArgs ma;
     if (use_bf) {
       std::memset(static_cast<void*>(&ma), 0, sizeof(ma));

@@ -659,18 +659,30 @@ def test_deterministic(variant):
         assert np.array_equal(a, b)
 
 
-@pytest.mark.parametrize("variant", ["G", "L", "muon", "L_exact"])
+_HOST_VARIANTS = ["G", "L", "L_bf16", "muon", "L_exact"]
+
+
+def _host_variant(variant):
+    """(variant code, precision) of a host-step test case: L_bf16 is NormPre-L
+    with the bf16 Psi (NORMPRE_PREC_BF16), whose sketch runs on group slices
+    with their own tensor maps in the host step."""
+    from paper_2609_36692_gb300 import normpre as C
+    code = {"G": C.NORMPRE_G, "L": C.NORMPRE_L, "L_bf16": C.NORMPRE_L, "muon": C.NORMPRE_MUON,
+            "L_exact": C.NORMPRE_L_EXACT}[variant]
+    return code, 0 if variant in ("G", "muon", "L_bf16") else 1
+
+
+@pytest.mark.parametrize("variant", _HOST_VARIANTS)
 def test_host_entry_point_matches_device_step(variant):
     """Two consecutive host-buffer steps (row- then column-active) equal the
     device-buffer steps bit for bit: the copies overlapped with the step move
     each group's inputs in before its normalization and its results out after."""
     import torch
-    from paper_2609_36692_gb300 import normpre as C
     cs = SMALL
     mats = S.make_param_set(cs, workers=min(16, os.cpu_count() or 1))
-    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON,
-                       "L_exact": C.NORMPRE_L_EXACT}[variant],
-              precision=0 if variant in ("G", "muon") else 1, rank=cs.rank, oversample=cs.oversample,
+    code, prec = _host_variant(variant)
+    kw = dict(variant=code,
+              precision=prec, rank=cs.rank, oversample=cs.oversample,
               power_iters=cs.power_iters, seed=1234, diagnostics=1)
     shapes = [(m.rows, m.cols) for m in cs.matrices]
     opt = _normpre(shapes, ["f32"] * cs.n_mats, ["bf16"] * cs.n_mats, **kw)
@@ -689,21 +701,19 @@ def test_host_entry_point_matches_device_step(variant):
             assert np.array_equal(Mh[i].numpy(), to_host(M[i])), (t, i)
 
 
-@pytest.mark.parametrize("variant", ["G", "L", "muon", "L_exact"])
+@pytest.mark.parametrize("variant", _HOST_VARIANTS)
 def test_host_entry_point_in_units(variant):
     """A group larger than one host-copy unit (8 x 4096^2 fp32/bf16: about
     1.3 GB of input) is preconditioned in pieces of matrices between its copies;
     the result equals the device-buffer step (whole groups) bit for bit."""
     import torch
-    from paper_2609_36692_gb300 import normpre as C
     shapes = [(4096, 4096)] * 8 + [(1024, 4096)] * 3
     gen = torch.Generator().manual_seed(7)
     Wc = [torch.randn(r, c, generator=gen) * 0.02 for r, c in shapes]
     Gc = [torch.randn(r, c, generator=gen).to(torch.bfloat16) for r, c in shapes]
     Mc = [torch.randn(r, c, generator=gen) * 0.1 for r, c in shapes]
-    kw = dict(variant={"G": C.NORMPRE_G, "L": C.NORMPRE_L, "muon": C.NORMPRE_MUON,
-                       "L_exact": C.NORMPRE_L_EXACT}[variant],
-              precision=0 if variant in ("G", "muon") else 1, seed=1234)
+    code, prec = _host_variant(variant)
+    kw = dict(variant=code, precision=prec, seed=1234)
     opt = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
     opt2 = _normpre(shapes, ["f32"] * len(shapes), ["bf16"] * len(shapes), **kw)
     W = [w.cuda() for w in Wc]
