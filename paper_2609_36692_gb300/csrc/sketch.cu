@@ -1857,325 +1857,6 @@ __global__ void __launch_bounds__(kAtcThreads, 1) k_apply_tc(const __grid_consta
 }
 
 // ---------------------------------------------------------------------------
-// Fused apply for a bf16 Psi (NORMPRE_PREC_BF16; l % 4 == 0, l <= 64, no
-// diagnostics, cols % 8 == 0, 16-byte aligned W).  Psi carries bf16 rounding
-// (2^-8 of each entry), so the rank-l correction Lm Rm^T runs as one TF32
-// product (2^-11 of the correction) instead of the three-product split: the
-// operand tiles hold hi only, which leaves room for a ring of Psi / W tiles in
-// shared memory.  A loader warp fills the ring with TMA copies (32 rows x 128
-// columns of Psi and of W per stage: 64-column boxes of Psi through the
-// group's map, 128-byte-wide boxes of W through one map per matrix, 128-byte
-// swizzle, zero fill past the edges), so the loads are coalesced and cost no
-// registers, and the epilogue reads them column-wise (lane = W column, as the
-// TMEM lanes) from shared memory.
-//
-// Same units, MMA shape and TMEM use as k_apply_tc: D = Rm_tile Lm_tile^T,
-// M = 128 W columns (TMEM lanes), N = 256 W rows (TMEM columns); warps 0-1
-// split, warp 2 issues the MMAs, warp 3 loads, warps 4-11 drain.  Within a
-// unit the eight 32-row stages are loaded in the order 0, 4, 1, 5, 2, 6, 3, 7
-// so that both row halves of the drain (rows 0-127 and 128-255) are fed.
-// ---------------------------------------------------------------------------
-constexpr int kAbfThreads = 32 * 12;
-constexpr int kAbfEpi = 8;
-template <typename TW>
-__host__ __device__ constexpr int abf_stages() { return sizeof(TW) == 2 ? 7 : 5; }
-template <typename TW>
-__host__ __device__ constexpr int abf_stage_bytes() { return 32 * 128 * (2 + static_cast<int>(sizeof(TW))); }
-template <typename TW>
-static size_t abf_smem(int natoms) {
-  return 1024 + static_cast<size_t>(natoms) * (kAtcAtomA + kAtcAtomB) +
-         static_cast<size_t>(abf_stages<TW>()) * abf_stage_bytes<TW>() + 512;
-}
-
-// At most kAbfBatch matrices per launch, so that the kernel's arguments (the
-// apply arguments, these tensor maps and three scalars) stay within the 4 KB
-// of a kernel's classic parameter space: launches of this kernel from several
-// streams overlap, and with more than 4 KB of arguments concurrent launches
-// that differed in their later arguments faulted.
-constexpr int kAbfBatch = 16;
-// k_apply_bf is not dispatched: on eight 4096 x 4096 fp32 weights together
-// with three 1024 x 4096 ones (two shape groups whose applies overlap on their
-// streams) it faulted, and the cause is not found; the bf16-Psi step uses
-// k_apply_tc<TW, bf16> instead
-constexpr bool kApplyBfEnabled = false;
-struct ApplyBfArgs {
-  CUtensorMap psi_map;             // bf16 Psi {cols, rows, batch}, box 64 x 32
-  CUtensorMap lm_map, rm_map;      // fp32 panels {l, rows / cols, launch batch}, boxes 32 x 256 / 32 x 128
-  CUtensorMap w_map[kAbfBatch];    // W of each matrix {cols, rows}, box (128 bytes) x 32
-  int psi_b0;                      // batch coordinate of the launch's first matrix in psi_map
-};
-
-static_assert(sizeof(LApplyArgs) + sizeof(ApplyBfArgs) + 32 <= 4096, "k_apply_bf arguments beyond 4 KB");
-static_assert(sizeof(LApplyArgs) + 32 <= 4096, "apply arguments beyond 4 KB");
-
-template <typename TW>
-__global__ void __launch_bounds__(kAbfThreads, 1) k_apply_bf(const __grid_constant__ LApplyArgs a,
-                                                              const __grid_constant__ ApplyBfArgs m, int nmat,
-                                                              int natoms, int* flags) {
-  constexpr int S = abf_stages<TW>(), SB = abf_stage_bytes<TW>();
-  extern __shared__ uint8_t abf_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(abf_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* a_hi = smem;                                   // Rm tile (128 W columns)
-  uint8_t* b_hi = a_hi + natoms * kAtcAtomA;              // Lm tile (256 W rows)
-  uint8_t* ring = b_hi + natoms * kAtcAtomB;              // S stages: Psi boxes (2 x 4 KB) | W boxes
-  uint64_t* opfull = reinterpret_cast<uint64_t*>(ring + S * SB);
-  uint64_t* opfree = opfull + 1;
-  uint64_t* tfull = opfree + 1;                           // [2]
-  uint64_t* tempty = tfull + 2;                           // [2]
-  uint64_t* sfull = tempty + 2;                           // [S] stage landed
-  uint64_t* sempty = sfull + S;                           // [S] stage read by its 4 drain warps
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sempty + S);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  uint32_t* issued = reinterpret_cast<uint32_t*>(tmem_slot + 2);   // [S] last parity + 1
-  uint32_t op_issued = 0;                                           // operand copies: last parity + 1 (thread 0)
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t rt = (a.rows + kAtcRows - 1) / kAtcRows, ct = (a.cols + kAtcCols - 1) / kAtcCols;
-  const int64_t per_mat = rt * ct;
-  const int64_t units = per_mat * nmat;
-  const int64_t u0 = units * blockIdx.x / gridDim.x, u1 = units * (blockIdx.x + 1) / gridDim.x;
-  auto unit_of = [&](int64_t u, int& b, int64_t& i0, int64_t& j0) {
-    b = static_cast<int>(u / per_mat);
-    const int64_t rem = u - b * per_mat;
-    i0 = (rem / ct) * kAtcRows;
-    j0 = (rem % ct) * kAtcCols;
-  };
-  if (threadIdx.x == 0) {
-    tc::mbar_init(opfull, 1);
-    tc::mbar_init(opfree, 1);
-    for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(&tfull[i], 1);
-      tc::mbar_init(&tempty[i], kAbfEpi);
-    }
-    for (int i = 0; i < S; ++i) {
-      tc::mbar_init(&sfull[i], 1);
-      tc::mbar_init(&sempty[i], 4);
-      issued[i] = 0;
-    }
-    *abort_flag = 0;
-    tc::fence_barrier_init();
-  }
-  if (warp == kAtcProd) {
-    tc::tmem_alloc(tmem_slot, 512);
-    tc::tmem_relinquish();
-    tc::fence_before();
-  }
-  // K columns past l up to the next multiple of 8 enter the last MMA K step
-  // and are never written below: zero the operand tiles once
-  for (int i = threadIdx.x; i < natoms * (kAtcAtomA + kAtcAtomB) / 16; i += blockDim.x)
-    reinterpret_cast<float4*>(smem)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  __syncthreads();
-  tc::fence_after();
-  const uint32_t tmem_base = *tmem_slot;
-  const int l = a.l;
-  const int ksteps = (l + 7) / 8;
-  constexpr int WBOX = 128 / static_cast<int>(sizeof(TW));   // W columns per 128-byte box row
-
-  if (warp < kAtcProd) {
-    // ---------------- operand tiles by TMA (warp 0; warp 1 has no role) ----------------
-    // The MMA reads fp32 storage at TF32 precision, so the panels' 32-wide K
-    // slabs are copied as they are: a box of 32 floats x R rows with the
-    // 128-byte swizzle is exactly one K-major atom, K past l reads zero
-    bool ok = true;
-    if (warp == 0) {
-      if (lane == 0) {
-        tc::prefetch_map(&m.lm_map);
-        tc::prefetch_map(&m.rm_map);
-      }
-      int64_t b_key = -1;
-      uint32_t it = 0;
-      for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
-        int b;
-        int64_t i0, j0;
-        unit_of(u, b, i0, j0);
-        ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(opfree, (it & 1) ^ 1u, abort_flag));
-        if (!ok) break;
-        const int64_t key = static_cast<int64_t>(b) * rt + i0 / kAtcRows;
-        const bool new_b = key != b_key;
-        b_key = key;
-        if (lane == 0) {
-          tc::mbar_expect_tx(opfull, static_cast<uint32_t>(natoms * (kAtcAtomA + (new_b ? kAtcAtomB : 0))));
-          op_issued = (it & 1) + 1;
-          for (int at = 0; at < natoms; ++at) {
-            tc::tma_load_3d(a_hi + at * kAtcAtomA, &m.rm_map, opfull, 32 * at, static_cast<int>(j0), b);
-            if (new_b) tc::tma_load_3d(b_hi + at * kAtcAtomB, &m.lm_map, opfull, 32 * at, static_cast<int>(i0), b);
-          }
-        }
-        __syncwarp();
-      }
-    }
-    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
-  } else if (warp == kAtcProd) {
-    // ---------------- MMA issuer: one TF32 product per K step ----------------
-    const uint32_t idesc = tc::idesc_tf32(kAtcCols, kAtcRows, 0, 0);
-    bool ok = true;
-    uint32_t it = 0;
-    for (int64_t u = u0; u < u1 && ok; ++u, ++it) {
-      const int acc = it & 1;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(opfull, it & 1, abort_flag));
-      if (!ok) break;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(&tempty[acc], ((it >> 1) & 1) ^ 1u, abort_flag));
-      if (!ok) break;
-      tc::fence_after();
-      if (lane == 0) {
-        const uint32_t d = tmem_base + static_cast<uint32_t>(256 * acc);
-        for (int kk = 0; kk < ksteps; ++kk) {
-          const uint32_t off = static_cast<uint32_t>(kk & 3) * 32u;
-          const uint32_t aa = static_cast<uint32_t>(kk >> 2) * kAtcAtomA + off;
-          const uint32_t bb = static_cast<uint32_t>(kk >> 2) * kAtcAtomB + off;
-          tc::mma_tf32(d, tc::sdesc(tc::su32(a_hi) + aa, 16, 1024), tc::sdesc(tc::su32(b_hi) + bb, 16, 1024), idesc,
-                       kk > 0 ? 1u : 0u);
-        }
-        tc::mma_commit(opfree);
-        tc::mma_commit(&tfull[acc]);
-      }
-      __syncwarp();
-    }
-    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
-  } else if (warp == kAtcProd + 1) {
-    // ---------------- loader: the Psi and W boxes of each 32-row stage ----------------
-    bool ok = true;
-    uint32_t it = 0;
-    if (lane == 0) {
-      tc::prefetch_map(&m.psi_map);
-      for (int i = 0; i < nmat; ++i) tc::prefetch_map(&m.w_map[i]);
-    }
-    for (int64_t u = u0; u < u1 && ok; ++u) {
-      int b;
-      int64_t i0, j0;
-      unit_of(u, b, i0, j0);
-      for (int kp = 0; kp < 8 && ok; ++kp, ++it) {
-        const int c = (kp & 1) ? 4 + (kp >> 1) : (kp >> 1);   // stage rows 32 c .. 32 c + 31 of the unit
-        const int sl = static_cast<int>(it % S);
-        const uint32_t ph = (it / S) & 1;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(&sempty[sl], ph ^ 1u, abort_flag));
-        if (!ok) break;
-        if (lane == 0) {
-          uint8_t* st = ring + sl * SB;
-          const int r0 = static_cast<int>(i0) + 32 * c, jc = static_cast<int>(j0);
-          tc::mbar_expect_tx(&sfull[sl], static_cast<uint32_t>(SB));   // boxes past the edges are zero-filled
-          issued[sl] = ph + 1;
-#pragma unroll
-          for (int i = 0; i < 2; ++i) tc::tma_load_3d(st + i * 4096, &m.psi_map, &sfull[sl], jc + 64 * i, r0, m.psi_b0 + b);
-#pragma unroll
-          for (int i = 0; i < 128 / WBOX; ++i) tc::tma_load_2d(st + 8192 + i * 4096, &m.w_map[b], &sfull[sl], jc + WBOX * i, r0);
-        }
-        __syncwarp();
-      }
-    }
-    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
-  } else {
-    // ---------------- epilogue: W <- (1 - lr wd) W - lr s (Psi + D) ----------------
-    const int e = warp - kAtcProd - 2;
-    const int q = warp & 3;          // TMEM lane quarter = W columns 32 q .. 32 q + 31 of the tile
-    const int h = e >> 2;            // W rows 128 h .. 128 h + 127 of the tile
-    const double mn = static_cast<double>(a.rows) * static_cast<double>(a.cols);
-    const float cw = 1.f - a.lr * a.wd;
-    bool ok = true;
-    int cur_b = -1;
-    float ctt = 0.f;
-    uint32_t uit = 0;
-    // swizzled byte offsets of this lane's Psi and W columns, per row & 7
-    uint32_t po[8], wo[8];
-    {
-      const int pcb = 2 * (32 * (q & 1) + lane);
-      const int wcb = static_cast<int>(sizeof(TW)) * ((32 * q + lane) % WBOX);
-#pragma unroll
-      for (int r = 0; r < 8; ++r) {
-        po[r] = static_cast<uint32_t>((((pcb >> 4) ^ r) << 4) + (pcb & 15));
-        wo[r] = static_cast<uint32_t>((((wcb >> 4) ^ r) << 4) + (wcb & 15));
-      }
-    }
-    for (int64_t u = u0; u < u1 && ok; ++u, ++uit) {
-      const int acc = uit & 1;
-      int b;
-      int64_t i0, j0;
-      unit_of(u, b, i0, j0);
-      if (b != cur_b) {
-        // fp64 throughput is low on this part: one lane per warp forms the
-        // scale of a new matrix and broadcasts it
-        float scale = 0.f;
-        if (lane == 0) {
-          const float nrm2 = a.stats[b * a.stats_bs + 2];
-          scale = nrm2 > 0.f ? static_cast<float>(a.target * sqrt(mn / nrm2)) : 0.f;
-        }
-        ctt = -a.lr * __shfl_sync(0xffffffffu, scale, 0);
-        cur_b = b;
-      }
-      const int64_t j = j0 + 32 * q + lane;
-      const bool jok = j < a.cols;
-      TW* W = static_cast<TW*>(a.W[b]) + j;
-      for (int cc = 0; cc < 4 && ok; ++cc) {
-        const uint32_t it = uit * 8u + static_cast<uint32_t>(2 * cc + h);   // stage of rows 32 (4 h + cc)
-        const int sl = static_cast<int>(it % S);
-        if (cc == 0) {
-          ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(&tfull[acc], (uit >> 1) & 1, abort_flag));
-          if (!ok) break;
-          tc::fence_after();
-        }
-        ok = __all_sync(0xffffffffu, tc::mbar_wait_idle(&sfull[sl], (it / S) & 1, abort_flag));
-        if (!ok) break;
-        uint32_t v[32];
-        tc::tmem_ld32(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(256 * acc + 128 * h + 32 * cc), v);
-        tc::tmem_ld_wait();
-        if (cc == 3) {
-          // the accumulator is read: the MMAs of unit uit + 2 may overwrite it
-          tc::fence_before();
-          __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&tempty[acc]);
-        }
-        // this lane's column 32 q + lane: Psi box (q / 2), byte column 2 (32 (q & 1) + lane);
-        // W box (32 q + lane) / WBOX.  Row rr of a box sits at rr * 128 plus a
-        // swizzled column offset that depends on rr & 7 only (po / wo below).
-        const uint8_t* st = ring + sl * SB;
-        const uint8_t* ps = st + (q >> 1) * 4096;
-        const uint8_t* ws = st + 8192 + ((32 * q + lane) / WBOX) * 4096;
-        const int64_t r0 = i0 + 128 * h + 32 * cc;
-        const int nr = (r0 < a.rows && jok) ? static_cast<int>(a.rows - r0 < 32 ? a.rows - r0 : 32) : 0;
-        TW* wrow = W + r0 * a.cols;
-        if (nr == 32) {
-#pragma unroll
-          for (int rr = 0; rr < 32; ++rr) {
-            const float p = to_f32(*reinterpret_cast<const bf16*>(ps + rr * 128 + po[rr & 7]));
-            const float w = to_f32(*reinterpret_cast<const TW*>(ws + rr * 128 + wo[rr & 7]));
-            *wrow = from_f32<TW>(fmaf(cw, w, ctt * (p + __uint_as_float(v[rr]))));
-            wrow += a.cols;
-          }
-        } else {
-#pragma unroll
-          for (int rr = 0; rr < 32; ++rr) {
-            if (rr < nr) {
-              const float p = to_f32(*reinterpret_cast<const bf16*>(ps + rr * 128 + po[rr & 7]));
-              const float w = to_f32(*reinterpret_cast<const TW*>(ws + rr * 128 + wo[rr & 7]));
-              *wrow = from_f32<TW>(fmaf(cw, w, ctt * (p + __uint_as_float(v[rr]))));
-            }
-            wrow += a.cols;
-          }
-        }
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&sempty[sl]);
-      }
-    }
-    if (!ok && lane == 0) { *abort_flag = 1; raise_flag(flags, kFlagTimeout); }
-  }
-  __syncthreads();
-  if (threadIdx.x == 0 && *abort_flag) {
-    // let every TMA copy still in flight land before the CTA exits
-    volatile int never = 0;
-    for (int i = 0; i < S; ++i)
-      if (issued[i]) tc::mbar_wait(&sfull[i], issued[i] - 1, &never);
-    if (op_issued) tc::mbar_wait(opfull, op_issued - 1, &never);
-  }
-  __syncthreads();
-  if (warp == kAtcProd) {
-    __syncwarp();
-    tc::fence_after();
-    tc::tmem_dealloc(tmem_base, 512);
-  }
-}
-
-// ---------------------------------------------------------------------------
 // host orchestration
 // ---------------------------------------------------------------------------
 #define NP_FOR_LP(X) X(8) X(16) X(24) X(32) X(40) X(48) X(56) X(64) X(72)
@@ -2560,18 +2241,14 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
   prof->end(kProfEig, s, (p.exact ? 1 : 3) + n_fold);
   // T_s = Psi + Lm R^T with (Lm, R) = (QK, B^T) row-active or (B^T, QK)
   // column-active; (Q, B^T K) and (B^T K, Q) when K went on B^T.  In launches
-  // of at most kMaxBatch matrices (W pointers travel as kernel arguments;
-  // kAbfBatch for the bf16-Psi kernel, whose W tensor maps do too)
+  // of at most kMaxBatch matrices (W pointers travel as kernel arguments)
   const float* u_a = k_on_b ? g.q : g.qk;    // the m_a-row factor
   const float* u_b = k_on_b ? g.qk : g.bt;   // the n_a-row factor
   prof->begin(kProfApplyL, s);
   int n_apply = 0;
   const bool vec = (g.cols % 4 == 0) && (g.ld % 4 == 0);
-  const bool bf_shape = kApplyBfEnabled && !(p.diag && p.G) && l % 4 == 0 && l <= 64 && g.psi_bf16 &&
-                        vbs % 4 == 0 && (g.cols * (g.w_dtype ? 2 : 4)) % 16 == 0;
-  const int per_launch = bf_shape ? kAbfBatch : kMaxBatch;
-  for (int c0 = 0; c0 < B; c0 += per_launch) {
-    const int nb = std::min(per_launch, B - c0);
+  for (int c0 = 0; c0 < B; c0 += kMaxBatch) {
+    const int nb = std::min(kMaxBatch, B - c0);
     ++n_apply;
     LApplyArgs la;
     std::memset(static_cast<void*>(&la), 0, sizeof(la));   // unused W / G slots are null, never stale
@@ -2591,47 +2268,6 @@ cudaError_t run_sketch_group(SketchGroup& g, const SketchParams& p, const int* m
     for (int i = 0; i < nb; ++i) {
       la.G[i] = diag ? p.G[c0 + i] : nullptr;
       la.diag[i] = diag ? p.diag + 8 * static_cast<int64_t>(p.mat_ids_host[c0 + i]) : nullptr;
-    }
-    // bf16 Psi: single-product apply fed by TMA (W maps need 16-byte rows and pointers)
-    bool use_bf = bf_shape && !diag && la.vec_panels;
-    ApplyBfArgs ma;
-    if (use_bf) {
-      std::memset(static_cast<void*>(&ma), 0, sizeof(ma));
-      ma.psi_map = g.psi_map_apply;
-      ma.psi_b0 = c0;
-      const uint64_t wd[2] = {static_cast<uint64_t>(g.cols), static_cast<uint64_t>(g.rows)};
-      const uint64_t ws[1] = {static_cast<uint64_t>(g.cols) * (g.w_dtype ? 2 : 4)};
-      const uint32_t wbox[2] = {static_cast<uint32_t>(g.w_dtype ? 64 : 32), 32};
-      for (int i = 0; i < nb && use_bf; ++i)
-        use_bf = driver_encode_tiled(&ma.w_map[i], g.w_dtype ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
-                                     2, la.W[i], wd, ws, wbox, nullptr);
-      // the fp32 panels (l % 4 == 0 and 16-byte matrix strides: vec_panels)
-      const uint64_t pst[2] = {static_cast<uint64_t>(l) * 4, static_cast<uint64_t>(vbs) * 4};
-      const uint64_t ld_[3] = {static_cast<uint64_t>(l), static_cast<uint64_t>(g.rows), static_cast<uint64_t>(nb)};
-      const uint64_t rd_[3] = {static_cast<uint64_t>(l), static_cast<uint64_t>(g.cols), static_cast<uint64_t>(nb)};
-      const uint32_t lbox[3] = {32, static_cast<uint32_t>(kAtcRows), 1}, rbox[3] = {32, static_cast<uint32_t>(kAtcCols), 1};
-      use_bf = use_bf &&
-               driver_encode_tiled(&ma.lm_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(la.lm), ld_, pst, lbox, nullptr) &&
-               driver_encode_tiled(&ma.rm_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(la.rm), rd_, pst, rbox, nullptr);
-    }
-    if (use_bf) {
-      const int natoms = (l + 31) / 32;
-      static bool attr_bf[2] = {false, false};
-      const int wi = g.w_dtype != 0 ? 1 : 0;
-      if (!attr_bf[wi]) {
-        e = wi ? cudaFuncSetAttribute(k_apply_bf<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      static_cast<int>(abf_smem<bf16>(2)))
-               : cudaFuncSetAttribute(k_apply_bf<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      static_cast<int>(abf_smem<float>(2)));
-        if (e != cudaSuccess) return e;
-        attr_bf[wi] = true;
-      }
-      const int64_t units = cdiv(g.rows, kAtcRows) * cdiv(g.cols, kAtcCols) * nb;
-      const unsigned ctas = static_cast<unsigned>(std::min<int64_t>(units, device_sm_count()));
-      if (wi) k_apply_bf<bf16><<<ctas, kAbfThreads, abf_smem<bf16>(natoms), s>>>(la, ma, nb, natoms, flags);
-      else k_apply_bf<float><<<ctas, kAbfThreads, abf_smem<float>(natoms), s>>>(la, ma, nb, natoms, flags);
-      NP_CHECK();
-      continue;
     }
     if (!diag && l % 4 == 0 && l <= 64 && la.vec_panels) {
       // tensor-core apply: one persistent CTA per SM over the launch's units
