@@ -92,6 +92,10 @@ SINGLE = S.CONFIGS["single_256x1024"]
 # the CholeskyQR rows are not float4-aligned
 ODD = S.custom_config("odd_width", [(96, 160), (160, 96), (19, 300), (250, 11), (45, 45)],
                       g_dtype="f32", w_dtype="f32", row_sigma=1.0, col_sigma=1.0, rank=13, oversample=6)
+# bf16 weights of even and odd widths and ragged row counts in the bf16 mode
+RAGGED_BF16W = S.custom_config("ragged_bf16w", [(50, 202), (203, 50), (131, 130), (64, 77), (300, 256)],
+                               g_dtype="bf16", w_dtype="bf16", row_sigma=1.0, col_sigma=1.0,
+                               rank=4, oversample=4)
 # tall column-active strips: clusters of 4, 8 and 12 CTAs (the last with a
 # partial row block) and one matrix whose column count is not a multiple of 32
 TALL = S.custom_config("tall_cols", [(1000, 40), (4100, 64), (6144, 32), (2056, 24)],
@@ -420,11 +424,12 @@ def _check_l_bf16(cs, t, indices=None, w_tol=3e-3):
             _check_bf16_w(W1[i], ref["W"], dW_ref, w_tol, (cs.name, i), elem_tol=2.0 ** -7 + w_tol)
 
 
-@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED, ODD, TALL], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfgset", [SINGLE, SMALL, RAGGED, ODD, TALL, RAGGED_BF16W], ids=lambda c: c.name)
 @pytest.mark.parametrize("t", [0, 1])
 def test_l_bf16_psi(cfgset, t):
     """Both contraction orientations of the bf16 kernel, ragged tiles and K
-    blocks, odd sketch widths (l = 19, 11), tall strips and 1-wide matrices."""
+    blocks, odd sketch widths (l = 19, 11), tall strips, 1-wide matrices and
+    bf16 weights of even and odd widths."""
     _check_l_bf16(cfgset, t)
 
 
