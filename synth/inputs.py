@@ -203,7 +203,8 @@ def make_matrix(cfg: ParamSetConfig, index: int, seed: Optional[int] = None,
     """Draw (G, M_prev, W) for matrix ``index`` of parameter set ``cfg``.
 
     Returns float32 arrays holding values exactly representable in the storage
-    dtype (``cfg.g_dtype`` for G, float32 for M, ``cfg.w_dtype`` for W).
+    dtype: ``cfg.g_dtype`` for G and for M (a gradient draw, kept in an fp32
+    momentum buffer), ``cfg.w_dtype`` for W.
     """
     s = cfg.seed if seed is None else seed
     spec = cfg.matrices[index]
