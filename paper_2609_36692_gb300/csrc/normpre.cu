@@ -187,10 +187,11 @@ const char* normpre_last_error(const normpre_handle* h) {
   return h ? h->err.c_str() : g_thread_error.c_str();
 }
 
-void normpre_free(normpre_handle* h) {
-  if (!h) return;
-  cudaSetDevice(h->device);
-  cudaDeviceSynchronize();
+namespace {
+
+// Everything a handle holds, on the current device: what normpre_free
+// releases, and what a normpre_init that fails part way has created so far.
+void release_handle(normpre_handle* h) {
   h->ns.reset();
   for (cudaStream_t st : h->side) cudaStreamDestroy(st);
   for (cudaEvent_t ev : h->side_done) cudaEventDestroy(ev);
@@ -205,6 +206,19 @@ void normpre_free(normpre_handle* h) {
   for (cudaStream_t st : {h->h2d, h->d2h})
     if (st) cudaStreamDestroy(st);
   delete h;
+}
+
+struct HandleRelease {
+  void operator()(normpre_handle* h) const { release_handle(h); }
+};
+
+}  // namespace
+
+void normpre_free(normpre_handle* h) {
+  if (!h) return;
+  cudaSetDevice(h->device);
+  cudaDeviceSynchronize();
+  release_handle(h);
 }
 
 int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, const int64_t* cols,
@@ -224,7 +238,8 @@ int normpre_init(const normpre_config* cfg, int n_mats, const int64_t* rows, con
     if ((w_dtype[i] != NORMPRE_F32 && w_dtype[i] != NORMPRE_BF16) || (g_dtype[i] != NORMPRE_F32 && g_dtype[i] != NORMPRE_BF16))
       return fail(nullptr, NORMPRE_ERR_DTYPE, "matrix " + std::to_string(i) + ": dtype must be NORMPRE_F32 or NORMPRE_BF16");
   }
-  std::unique_ptr<normpre_handle> h(new normpre_handle());
+  // an init that fails part way frees what it has created
+  std::unique_ptr<normpre_handle, HandleRelease> h(new normpre_handle());
   h->cfg = *cfg;
   h->n_mats = n_mats;
   cudaError_t e = cudaGetDevice(&h->device);
