@@ -646,7 +646,21 @@ struct HostPipe : StepHooks {
   }
 };
 
-cudaError_t host_pipe_alloc(normpre_handle* h) {
+// The staging buffers (indexed by matrix), copy streams and step events of
+// the host-buffer entry point; all or nothing, so that a retry after a failed
+// allocation starts from empty vectors.
+void host_pipe_release(normpre_handle* h) {
+  for (auto* v : {&h->stage_w, &h->stage_g, &h->stage_m}) {
+    for (void* p : *v) cudaFree(p);
+    v->clear();
+  }
+  for (cudaEvent_t* ev : {&h->start_ev, &h->out_ev})
+    if (*ev) { cudaEventDestroy(*ev); *ev = nullptr; }
+  for (cudaStream_t* st : {&h->h2d, &h->d2h})
+    if (*st) { cudaStreamDestroy(*st); *st = nullptr; }
+}
+
+cudaError_t host_pipe_alloc_all(normpre_handle* h) {
   cudaError_t e;
   for (int i = 0; i < h->n_mats; ++i) {
     const MatInfo& m = h->mats[i];
@@ -663,6 +677,12 @@ cudaError_t host_pipe_alloc(normpre_handle* h) {
   if ((e = cudaStreamCreateWithFlags(&h->d2h, cudaStreamNonBlocking))) return e;
   if ((e = cudaEventCreateWithFlags(&h->start_ev, cudaEventDisableTiming))) return e;
   return cudaEventCreateWithFlags(&h->out_ev, cudaEventDisableTiming);
+}
+
+cudaError_t host_pipe_alloc(normpre_handle* h) {
+  const cudaError_t e = host_pipe_alloc_all(h);
+  if (e != cudaSuccess) host_pipe_release(h);
+  return e;
 }
 
 // The units of a host-buffer step, largest groups first.
