@@ -19,6 +19,9 @@
  *   - Matrices are dense, row-major, contiguous, `rows x cols` as stored.
  *   - Device pointers are CUDA device addresses on the current device and must
  *     be 16-byte aligned.  Host pointers are ordinary host addresses.
+ *   - A handle belongs to the device that was current at normpre_init; every
+ *     call on it makes that device current for its own duration and gives
+ *     the caller's current device back before it returns.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
  *     Calls enqueue work on it and return without synchronizing unless the
  *     description says otherwise.

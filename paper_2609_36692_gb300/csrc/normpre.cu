@@ -189,6 +189,24 @@ const char* normpre_last_error(const normpre_handle* h) {
 
 namespace {
 
+// Makes the handle's device current for one entry point and gives the caller
+// its own current device back on the way out.
+class DeviceGuard {
+ public:
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev_) == cudaSuccess && prev_ != dev) changed_ = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    if (changed_) cudaSetDevice(prev_);
+  }
+  DeviceGuard(const DeviceGuard&) = delete;
+  DeviceGuard& operator=(const DeviceGuard&) = delete;
+
+ private:
+  int prev_ = 0;
+  bool changed_ = false;
+};
+
 // Everything a handle holds, on the current device: what normpre_free
 // releases, and what a normpre_init that fails part way has created so far.
 void release_handle(normpre_handle* h) {
@@ -216,7 +234,7 @@ struct HandleRelease {
 
 void normpre_free(normpre_handle* h) {
   if (!h) return;
-  cudaSetDevice(h->device);
+  DeviceGuard device_guard(h->device);
   cudaDeviceSynchronize();
   release_handle(h);
 }
@@ -341,7 +359,7 @@ int step_impl(normpre_handle* h, int64_t t, float lr, void* const* W, const void
     if (!aligned16(W[i]) || !aligned16(G[i]) || !aligned16(M[i]))
       return fail(h, NORMPRE_ERR_ALIGN, "matrix " + std::to_string(i) + ": tensors must be 16-byte aligned");
   }
-  cudaSetDevice(h->device);
+  DeviceGuard device_guard(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const normpre_config& c = h->cfg;
   const int k = orientation_of(c, t);
@@ -581,7 +599,7 @@ int normpre_profile(normpre_handle* h, int enable) {
 int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* launches) {
   if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
   if (n_classes < 0 || (n_classes > 0 && (!ms || !launches))) return fail(h, NORMPRE_ERR_ARG, "bad output arrays");
-  cudaSetDevice(h->device);
+  DeviceGuard device_guard(h->device);
   h->prof.collect();
   for (int i = 0; i < n_classes; ++i) {
     ms[i] = i < kProfClasses ? h->prof.ms[i] : 0.0;
@@ -593,7 +611,7 @@ int normpre_profile_read(normpre_handle* h, int n_classes, double* ms, int64_t* 
 
 int normpre_sync_status(normpre_handle* h, void* stream) {
   if (!h) return fail(nullptr, NORMPRE_ERR_ARG, "null handle");
-  cudaSetDevice(h->device);
+  DeviceGuard device_guard(h->device);
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e) return cuda_fail(h, e, "cudaStreamSynchronize");
   int flags = 0;
@@ -714,7 +732,7 @@ int normpre_step_host(normpre_handle* h, int64_t t, float lr, void* const* W_hos
   if (!W_host || !G_host || !M_host) return fail(h, NORMPRE_ERR_ARG, "null pointer array");
   for (int i = 0; i < h->n_mats; ++i)
     if (!W_host[i] || !G_host[i] || !M_host[i]) return fail(h, NORMPRE_ERR_ARG, "null host tensor pointer");
-  cudaSetDevice(h->device);
+  DeviceGuard device_guard(h->device);
   cudaError_t e;
   if (!h->h2d && (e = host_pipe_alloc(h))) return cuda_fail(h, e, "host-buffer staging");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -822,7 +840,7 @@ int normpre_read(normpre_handle* h, int mat, int what, void* dst, int64_t capaci
   if (rc) return rc;
   const size_t el = dsize(dt);
   if (capacity_bytes < static_cast<int64_t>(r * c * el)) return fail(h, NORMPRE_ERR_ARG, "destination too small");
-  cudaSetDevice(h->device);
+  DeviceGuard device_guard(h->device);
   cudaError_t e = cudaDeviceSynchronize();
   if (e) return cuda_fail(h, e, "cudaDeviceSynchronize");
   const MatInfo& m = h->mats[mat];

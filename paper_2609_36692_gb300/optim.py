@@ -122,6 +122,8 @@ class NormPreOptimizer(_torch_optimizer_base()):
                         variant=variant, config=dict(config))
         super().__init__(params, defaults)
         for group in self.param_groups:
+            if len({p.device for p in group["params"]}) > 1:
+                raise ValueError("the matrices of a parameter group must share one CUDA device")
             for p in group["params"]:
                 if p.dim() != 2:
                     raise ValueError("NormPreOptimizer takes 2-D matrices only (got shape %s); give "
@@ -136,7 +138,10 @@ class NormPreOptimizer(_torch_optimizer_base()):
         self._plans = {}
 
     def _plan(self, gi: int, group, params):
-        key = (tuple(id(p) for p in params), tuple(repr(group[k]) for k in self._FIXED))
+        # a plan is fixed to its matrices, their weight and gradient dtypes and
+        # the group's hyperparameters other than lr
+        key = (tuple(id(p) for p in params), tuple((_dtype_code(p), _dtype_code(p.grad)) for p in params),
+               tuple(repr(group[k]) for k in self._FIXED))
         plan = self._plans.get(gi)
         if plan is None or plan[0] != key:
             cfg = dict(group["config"])
@@ -165,21 +170,25 @@ class NormPreOptimizer(_torch_optimizer_base()):
                     st = self.state[p]
                     if "momentum_buffer" not in st:
                         st["momentum_buffer"] = torch.zeros(p.shape, dtype=torch.float32, device=p.device)
-                plan = self._plan(gi, group, params)
-                plan.step(group["t"], float(group["lr"]), params, [p.grad for p in params],
-                          [self.state[p]["momentum_buffer"] for p in params])
-                group["t"] += 1
-                if self.check_status:
-                    plan.status()
+                # the library works on the current device: make it the matrices'
+                with torch.cuda.device(params[0].device):
+                    plan = self._plan(gi, group, params)
+                    plan.step(group["t"], float(group["lr"]), params, [p.grad for p in params],
+                              [self.state[p]["momentum_buffer"] for p in params])
+                    group["t"] += 1
+                    if self.check_status:
+                        plan.status()
         return loss
 
     def diagnostics(self):
         """Per matrix of the last step: NORMPRE_BUF_DIAG as a dict (spectral
         energies with variant "L_exact", descent alignment with
         diagnostics=1), plus the mean alignment over the matrices (App. E)."""
+        import torch
         out, cos = {}, []
         for gi, (key, plan, params) in self._plans.items():
-            plan.status()
+            with torch.cuda.device(params[0].device):
+                plan.status()
             for i, p in enumerate(params):
                 d = plan.read(i, C.NORMPRE_BUF_DIAG)[0]
                 rec = dict(zip(("E_top", "E_remain", "E_sub", "E_global", "align", "grad_norm",

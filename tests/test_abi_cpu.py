@@ -138,3 +138,7 @@ def test_torch_optimizer_validates_parameters():
         NormPreOptimizer([torch.nn.Parameter(torch.zeros(3, 4))])
     with pytest.raises(ValueError, match="variant"):
         NormPreOptimizer([torch.nn.Parameter(torch.zeros(3, 4))], variant="X")
+    # one plan serves a group on one device
+    with pytest.raises(ValueError, match="one CUDA device"):
+        NormPreOptimizer([torch.nn.Parameter(torch.zeros(3, 4)),
+                          torch.nn.Parameter(torch.zeros(3, 4, device="meta"))])
