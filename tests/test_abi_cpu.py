@@ -142,3 +142,39 @@ def test_torch_optimizer_validates_parameters():
     with pytest.raises(ValueError, match="one CUDA device"):
         NormPreOptimizer([torch.nn.Parameter(torch.zeros(3, 4)),
                           torch.nn.Parameter(torch.zeros(3, 4, device="meta"))])
+
+
+def _header_without_comments():
+    return re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+
+
+def test_binding_enums_mirror_the_header(lib):
+    """Every enumerator the header defines has the same value in the binding."""
+    src = _header_without_comments()
+    values = {}
+    for body in re.findall(r"\benum\s+\w+\s*\{(.*?)\}", src, flags=re.S):
+        for name, val in re.findall(r"\b(NORMPRE_\w+)\s*=\s*(\d+)", body):
+            values[name] = int(val)
+    assert len(values) >= 30
+    mirrored = {n: v for n, v in values.items() if not n.startswith("NORMPRE_PROF_")}
+    for name, val in mirrored.items():
+        assert getattr(lib, name) == val, name
+    assert lib.STATUS_NAMES == {v: n[len("NORMPRE_"):] for n, v in values.items()
+                                if n == "NORMPRE_OK" or n.startswith("NORMPRE_ERR_")}
+
+
+def test_binding_config_struct_mirrors_the_header(lib):
+    """normpre_config: the binding's ctypes fields in the header's order and
+    types, so that the library reads every hyperparameter where it was put."""
+    src = _header_without_comments()
+    body = re.search(r"typedef\s+struct\s+normpre_config\s*\{(.*?)\}\s*normpre_config\s*;", src, flags=re.S).group(1)
+    fields = re.findall(r"(\w+)\s+(\w+)(\[\d+\])?\s*;", body)
+    c_types = {"int": ctypes.c_int, "float": ctypes.c_float, "uint64_t": ctypes.c_uint64}
+    want = [(name, c_types[ty] * int(arr[1:-1]) if arr else c_types[ty]) for ty, name, arr in fields]
+    got = lib.normpre_config._fields_
+    assert [n for n, _ in got] == [n for n, _ in want]
+    for (n, t_got), (_, t_want) in zip(got, want):
+        if hasattr(t_want, "_length_"):      # a fixed-size array field
+            assert t_got._length_ == t_want._length_ and t_got._type_ is t_want._type_, n
+        else:
+            assert t_got is t_want, n
